@@ -1,0 +1,383 @@
+"""Pins of the fp64 oracle against facts fixed outside the oracle itself.
+
+Each ``check_*`` function raises AssertionError when the oracle disagrees with
+a hand-derived fixture (tests/golden), a closed form, an invariant, a special
+case that reduces to something simpler, or an independent library routine.
+``test_planted_mistakes_are_caught`` plants plausible mistakes in the oracle
+(on the CPU) and asserts that at least one check fails for each of them.
+"""
+import dataclasses
+import hashlib
+
+import numpy as np
+import pytest
+
+import oracle.sp_oracle as so
+from conftest import read_golden
+from paper_2608_28099_gb300 import workloads as wl
+
+
+# --------------------------------------------------------------------------- #
+# helpers (no method arithmetic: only build inputs)
+# --------------------------------------------------------------------------- #
+@dataclasses.dataclass
+class W:
+    w_q: np.ndarray
+    w_k: np.ndarray
+    w_v: np.ndarray
+    w_o: np.ndarray
+    w_gate: np.ndarray
+    w_up: np.ndarray
+    w_down: np.ndarray
+    g_in: np.ndarray
+    g_post: np.ndarray
+    soft_prompt: np.ndarray
+    head_w: np.ndarray
+    head_b: np.ndarray = None
+
+
+def f32(a):
+    return np.asarray(a, dtype=np.float32)
+
+
+def random_layer(seed, d=16, hq=4, hkv=2, dh=8, f=24, k=3, C=3, pool=wl.POOL_MEAN, eps=1e-6):
+    rng = np.random.default_rng(seed)
+    sh = wl.Shape(d, hq, hkv, dh, f, k, C, rope_theta=100.0, rms_eps=eps,
+                  w_dtype=wl.F32, kv_dtype=wl.F32, pool=pool)
+    n = lambda *s: f32(rng.standard_normal(s) * 0.4)
+    w = W(n(hq * dh, d), n(hkv * dh, d), n(hkv * dh, d), n(d, hq * dh), n(f, d), n(f, d), n(d, f),
+          f32(1 + 0.1 * rng.standard_normal(d)), f32(1 + 0.1 * rng.standard_normal(d)),
+          n(k, d), n(C, d), f32(rng.standard_normal(C)))
+    return sh, w
+
+
+def hand_layer():
+    sh = wl.Shape(2, 1, 1, 2, 1, 1, 2, rope_theta=10000.0, rms_eps=0.0,
+                  w_dtype=wl.F32, kv_dtype=wl.F32, pool=wl.POOL_LAST)
+    I2 = f32(np.eye(2))
+    w = W(I2, I2, I2, I2, f32([[1, 0]]), f32([[0, 1]]), f32([[1], [0]]),
+          f32([1, 1]), f32([1, 1]), f32([[1, 1]]), np.eye(2), None)
+    return sh, w
+
+
+# --------------------------------------------------------------------------- #
+# checks
+# --------------------------------------------------------------------------- #
+def check_hand_example():
+    g = read_golden("hand_example_L2_k1.txt")
+    sh, w = hand_layer()
+    layer = so.Layer(sh, w)
+    kc = np.array([[[1.0, 0.0]], [[0.0, 1.0]]])
+    vc = kc.copy()
+    tr = {}
+    h2 = layer.rows_with_cache(layer.soft_prompt, kc, vc, trace=tr)
+    np.testing.assert_allclose(tr["q"].ravel(), g["q"], atol=1e-9)
+    np.testing.assert_allclose(tr["k_new"].ravel(), g["q"], atol=1e-9)
+    np.testing.assert_allclose(tr["p"].ravel(), g["p"], atol=1e-9)
+    np.testing.assert_allclose(tr["o"].ravel(), g["o"], atol=1e-9)
+    np.testing.assert_allclose(layer.readout(h2), g["logits"], atol=1e-9)
+
+
+def check_rope_pairs():
+    g = read_golden("rope_pairs_dh4.txt")
+    x = np.eye(4)[:3].reshape(3, 1, 1, 4)            # three inputs, T=1, H=1
+    y = np.stack([so.rope(x[i], np.array([1]), 1.0e4) for i in range(3)]).reshape(3, 4)
+    np.testing.assert_allclose(y[0], g["e0"], atol=1e-12)
+    np.testing.assert_allclose(y[1], g["e1"], atol=1e-12)
+    np.testing.assert_allclose(y[2], g["e2"], atol=1e-12)
+
+
+def check_rope_relative_and_norm():
+    """Rotation keeps norms and the score depends on position differences only."""
+    rng = np.random.default_rng(5)
+    q = rng.standard_normal((1, 1, 8))
+    k = rng.standard_normal((1, 1, 8))
+    np.testing.assert_allclose(np.linalg.norm(so.rope(q, np.array([37]), 100.0)), np.linalg.norm(q),
+                               rtol=1e-12)
+    s1 = np.sum(so.rope(q, np.array([40]), 100.0) * so.rope(k, np.array([33]), 100.0))
+    s2 = np.sum(so.rope(q, np.array([107]), 100.0) * so.rope(k, np.array([100]), 100.0))
+    np.testing.assert_allclose(s1, s2, rtol=1e-10)
+
+
+def check_softmax_rows_sum_to_one():
+    sh, w = random_layer(1)
+    layer = so.Layer(sh, w)
+    rng = np.random.default_rng(2)
+    L = 11
+    kc = rng.standard_normal((L, sh.n_kv_heads, sh.head_dim))
+    tr = {}
+    layer.rows_with_cache(layer.soft_prompt, kc, kc * 0.5, trace=tr)
+    sums = tr["p"].sum(axis=-1)
+    np.testing.assert_allclose(sums, 1.0, atol=1e-12)
+    # row r sees exactly L + r + 1 keys
+    for r in range(sh.k_rows):
+        nz = np.count_nonzero(tr["p"][r], axis=-1)
+        assert np.all(nz == L + r + 1), (r, nz)
+
+
+def check_incremental_equals_full_recompute():
+    """Cache path == full causal layer over [context ; soft rows] (Eq. 1-3)."""
+    cases = [dict(L=0), dict(L=1), dict(L=7), dict(L=2, k=5), dict(L=9, hq=2, hkv=2),
+             dict(L=6, hq=6, hkv=2, k=1), dict(L=5, dh=4)]
+    for i, c in enumerate(cases):
+        L = c.pop("L")
+        sh, w = random_layer(10 + i, **c)
+        layer = so.Layer(sh, w)
+        rng = np.random.default_rng(100 + i)
+        ctx = rng.standard_normal((L, sh.d_model))
+        kc, vc = layer.build_cache(ctx)
+        inc = layer.rows_with_cache(layer.soft_prompt, kc, vc)
+        full = layer.full_causal(np.concatenate([ctx, layer.soft_prompt], axis=0))[L:]
+        np.testing.assert_allclose(inc, full, rtol=1e-10, atol=1e-10)
+
+
+def check_gqa_equals_mha_with_repeated_kv():
+    sh, w = random_layer(3, hq=6, hkv=2)
+    G = sh.group
+    sh_mha = dataclasses.replace(sh, n_kv_heads=sh.n_q_heads)
+    dh = sh.head_dim
+    rep = lambda m: np.repeat(m.reshape(sh.n_kv_heads, dh, -1), G, axis=0).reshape(-1, m.shape[1])
+    w_mha = dataclasses.replace(w, w_k=rep(w.w_k), w_v=rep(w.w_v))
+    rng = np.random.default_rng(4)
+    kc = rng.standard_normal((9, sh.n_kv_heads, dh))
+    vc = rng.standard_normal((9, sh.n_kv_heads, dh))
+    a = so.Layer(sh, w).rows_with_cache(so.to_f64(w.soft_prompt, wl.F32), kc, vc)
+    b = so.Layer(sh_mha, w_mha).rows_with_cache(so.to_f64(w.soft_prompt, wl.F32),
+                                                np.repeat(kc, G, axis=1), np.repeat(vc, G, axis=1))
+    np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-12)
+
+
+def check_attention_matches_torch_sdpa():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(6)
+    R, Hq, Hkv, dh, L = 4, 6, 2, 16, 13
+    q = rng.standard_normal((R, Hq, dh))
+    keys = rng.standard_normal((L + R, Hkv, dh))
+    vals = rng.standard_normal((L + R, Hkv, dh))
+    visible = np.arange(L + R)[None, :] <= (L + np.arange(R))[:, None]
+    o = so.attention(q, keys, vals, visible, Hq // Hkv)
+    tq = torch.from_numpy(q).permute(1, 0, 2)[None]                       # [1, Hq, R, dh]
+    tk = torch.from_numpy(keys).permute(1, 0, 2).repeat_interleave(Hq // Hkv, 0)[None]
+    tv = torch.from_numpy(vals).permute(1, 0, 2).repeat_interleave(Hq // Hkv, 0)[None]
+    ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv,
+                                                           attn_mask=torch.from_numpy(visible))
+    np.testing.assert_allclose(o, ref[0].permute(1, 0, 2).numpy(), rtol=1e-12, atol=1e-12)
+
+
+def check_uniform_keys_give_mean_of_values():
+    rng = np.random.default_rng(7)
+    R, Hq, Hkv, dh, L = 3, 4, 2, 8, 10
+    q = rng.standard_normal((R, Hq, dh))
+    keys = np.tile(rng.standard_normal((1, Hkv, dh)), (L + R, 1, 1))
+    vals = rng.standard_normal((L + R, Hkv, dh))
+    visible = np.arange(L + R)[None, :] <= (L + np.arange(R))[:, None]
+    o = so.attention(q, keys, vals, visible, 2)
+    for r in range(R):
+        for h in range(Hq):
+            np.testing.assert_allclose(o[r, h], vals[: L + r + 1, h // 2].mean(axis=0),
+                                       rtol=1e-12, atol=1e-12)
+
+
+def check_rms_norm():
+    rng = np.random.default_rng(8)
+    x = rng.standard_normal((5, 32))
+    y = so.rms_norm(x, np.ones(32), 0.0)
+    np.testing.assert_allclose(np.sqrt(np.mean(y * y, axis=-1)), 1.0, rtol=1e-12)
+    np.testing.assert_allclose(so.rms_norm(3.5 * x, np.ones(32), 0.0), y, rtol=1e-12)
+    # eps enters inside the root: a constant row c gives c / sqrt(c^2 + eps)
+    c = np.full((1, 4), 0.5)
+    np.testing.assert_allclose(so.rms_norm(c, np.ones(4), 0.75), 0.5 / 1.0, rtol=1e-12)
+
+
+def check_silu():
+    np.testing.assert_allclose(so.silu(np.array([1.0])), [0.7310585786300049], rtol=1e-14)
+    z = np.linspace(-6, 6, 25)
+    np.testing.assert_allclose(so.silu(z) - so.silu(-z), z, atol=1e-12)
+    assert so.silu(np.array([0.0]))[0] == 0.0
+
+
+def check_swiglu_block_by_hand():
+    """d=2, d_ff=1 layer with zero attention output: h2 = h1 + W_down a with
+    a = silu(n_0) * n_1 computed by hand from n = h1 / rms(h1)."""
+    sh, w = hand_layer()
+    layer = so.Layer(sh, w)
+    x = np.array([[3.0, -1.0]])
+    h2 = layer.finish(x, np.zeros((1, 1, 2)))
+    rms = np.sqrt((9 + 1) / 2)
+    n0, n1 = 3 / rms, -1 / rms
+    a = n0 / (1 + np.exp(-n0)) * n1
+    np.testing.assert_allclose(h2, [[3.0 + a, -1.0]], rtol=1e-12)
+
+
+def check_readout_pooling():
+    sh, w = random_layer(9, pool=wl.POOL_MEAN)
+    h2 = np.random.default_rng(1).standard_normal((sh.k_rows, sh.d_model))
+    lm = so.Layer(sh, w).readout(h2)
+    ll = so.Layer(dataclasses.replace(sh, pool=wl.POOL_LAST), w).readout(h2)
+    hw = np.asarray(w.head_w, np.float64)
+    np.testing.assert_allclose(lm, hw @ h2.mean(axis=0) + w.head_b, rtol=1e-12)
+    np.testing.assert_allclose(ll, hw @ h2[-1] + w.head_b, rtol=1e-12)
+    # zero head gives the bias
+    w0 = dataclasses.replace(w, head_w=np.zeros_like(w.head_w))
+    np.testing.assert_allclose(so.Layer(sh, w0).readout(h2), w.head_b, rtol=0, atol=0)
+
+
+def check_k1_mean_equals_last():
+    sh, w = random_layer(12, k=1)
+    w = dataclasses.replace(w, soft_prompt=w.soft_prompt[:1])
+    rng = np.random.default_rng(3)
+    kc = rng.standard_normal((5, sh.n_kv_heads, sh.head_dim))
+    a = so.Layer(sh, w)
+    b = so.Layer(dataclasses.replace(sh, pool=wl.POOL_LAST), w)
+    np.testing.assert_allclose(a.readout(a.rows_with_cache(a.soft_prompt, kc, kc)),
+                               b.readout(b.rows_with_cache(b.soft_prompt, kc, kc)), rtol=1e-14)
+
+
+def check_paged_gather_matches_contiguous():
+    sh = wl.Shape(64, 4, 2, 16, 64, 2, 2, w_dtype=wl.BF16, kv_dtype=wl.BF16)
+    w = wl.custom(sh, [0, 1, 15, 16, 17, 40], wl.LAYOUT_CONTIGUOUS, 21)
+    paged = wl.contiguous_to_paged(w.cache, 16, 5)
+    for b in range(6):
+        k1, v1 = so.sequence_kv(w.cache, b)
+        k2, v2 = so.sequence_kv(paged, b)
+        assert k1.shape == (int(w.cache.seq_lens[b]), 2, 16)
+        assert np.array_equal(k1, k2) and np.array_equal(v1, v2)
+
+
+def check_cache_untouched():
+    sh = wl.Shape(64, 4, 2, 16, 64, 2, 2, w_dtype=wl.BF16, kv_dtype=wl.BF16)
+    w = wl.custom(sh, [5, 33], wl.LAYOUT_PAGED, 22)
+    before = hashlib.sha256(w.cache.k_pool.tobytes() + w.cache.v_pool.tobytes()).hexdigest()
+    so.classify(so.Layer(sh, w.weights), w.cache, w.seq_ids)
+    after = hashlib.sha256(w.cache.k_pool.tobytes() + w.cache.v_pool.tobytes()).hexdigest()
+    assert before == after
+
+
+ALL_CHECKS = [check_hand_example, check_rope_pairs, check_rope_relative_and_norm,
+              check_softmax_rows_sum_to_one, check_incremental_equals_full_recompute,
+              check_gqa_equals_mha_with_repeated_kv, check_attention_matches_torch_sdpa,
+              check_uniform_keys_give_mean_of_values, check_rms_norm, check_silu,
+              check_swiglu_block_by_hand, check_readout_pooling, check_k1_mean_equals_last,
+              check_paged_gather_matches_contiguous, check_cache_untouched]
+
+
+@pytest.mark.parametrize("check", ALL_CHECKS, ids=lambda f: f.__name__)
+def test_pin(check):
+    check()
+
+
+# --------------------------------------------------------------------------- #
+# planted mistakes: every one must trip at least one pin
+# --------------------------------------------------------------------------- #
+# Each factory takes the original function and returns a wrong variant of it.
+def _rope_flipped(orig):
+    return lambda x, positions, theta: orig(x, -np.asarray(positions), theta)
+
+
+def _rope_interleaved(orig):
+    def f(x, positions, theta):
+        dh = x.shape[-1]
+        perm = np.concatenate([np.arange(0, dh, 2), np.arange(1, dh, 2)])
+        return orig(x[..., perm], positions, theta)[..., np.argsort(perm)]
+    return f
+
+
+def _scale_1_over_dh(orig):
+    return lambda q, keys, visible, group: orig(q / np.sqrt(q.shape[-1]), keys, visible, group)
+
+
+def _no_causal_mask(orig):
+    return lambda q, keys, values, visible, group: orig(q, keys, values, np.ones_like(visible),
+                                                         group)
+
+
+def _gqa_modulo(orig):
+    def f(q, keys, visible, group):
+        # query head h reads KV head h % Hkv instead of h // group
+        Hq, Hkv = q.shape[1], keys.shape[1]
+        expanded = keys[:, [h % Hkv for h in range(Hq)]]
+        return orig(q, expanded, visible, 1)
+    return f
+
+
+def _rms_sum(orig):
+    return lambda x, gain, eps: x / np.sqrt(np.sum(x * x, axis=-1, keepdims=True) + eps) * gain
+
+
+def _rms_eps_outside(orig):
+    return lambda x, gain, eps: x / (np.sqrt(np.mean(x * x, axis=-1, keepdims=True)) + eps) * gain
+
+
+def _silu_sigmoid(orig):
+    return lambda z: 1.0 / (1.0 + np.exp(-z))
+
+
+def _positions_from_zero(orig):
+    def f(self, x, k_cache, v_cache, trace=None):
+        saved = self.project_qkv
+        L = k_cache.shape[0]
+        self.project_qkv = lambda xx, pos: saved(xx, np.asarray(pos) - L)
+        try:
+            return orig(self, x, k_cache, v_cache, trace)
+        finally:
+            del self.project_qkv
+    return f
+
+
+def _residual_dropped(orig):
+    def f(self, x, o):
+        return orig(self, np.zeros_like(x), o) + 0.0 * x
+    return f
+
+
+def _gate_up_swapped(orig):
+    def f(self, x, o):
+        self.w_gate, self.w_up = self.w_up, self.w_gate
+        try:
+            return orig(self, x, o)
+        finally:
+            self.w_gate, self.w_up = self.w_up, self.w_gate
+    return f
+
+
+def _readout_first_row(orig):
+    return lambda self, h2: self.head_w @ h2[0] + self.head_b
+
+
+def _gather_reversed(orig):
+    def f(cache, seq_id):
+        k, v = orig(cache, seq_id)
+        if cache.layout == so.LAYOUT_PAGED:
+            k, v = k[::-1].copy(), v[::-1].copy()
+        return k, v
+    return f
+
+
+MUTANTS = {
+    "rope_direction_flipped": (so, "rope", _rope_flipped),
+    "rope_interleaved_pairs": (so, "rope", _rope_interleaved),
+    "softmax_scale_1_over_dh": (so, "attention_probs", _scale_1_over_dh),
+    "no_causal_mask": (so, "attention", _no_causal_mask),
+    "gqa_head_modulo": (so, "attention_probs", _gqa_modulo),
+    "rms_sum_not_mean": (so, "rms_norm", _rms_sum),
+    "rms_eps_outside_root": (so, "rms_norm", _rms_eps_outside),
+    "silu_is_sigmoid": (so, "silu", _silu_sigmoid),
+    "positions_from_zero": (so.Layer, "rows_with_cache", _positions_from_zero),
+    "residual_dropped": (so.Layer, "finish", _residual_dropped),
+    "gate_up_swapped": (so.Layer, "finish", _gate_up_swapped),
+    "readout_first_row": (so.Layer, "readout", _readout_first_row),
+    "paged_gather_reversed": (so, "sequence_kv", _gather_reversed),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_planted_mistakes_are_caught(name, monkeypatch):
+    owner, attr, factory = MUTANTS[name]
+    monkeypatch.setattr(owner, attr, factory(getattr(owner, attr)))
+    failed = []
+    for check in ALL_CHECKS:
+        try:
+            check()
+        except AssertionError:
+            failed.append(check.__name__)
+    assert failed, f"planted mistake {name!r} passed every pin"
