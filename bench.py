@@ -1,0 +1,408 @@
+#!/usr/bin/env python
+"""Throughput of the Speculative Probing classify path on one GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 4b] [--impl ours|reference]
+
+One step = one sp_classify call over one batch of the named seeded workload
+(every stage of the path: input norm, Q/K/V projection, rotation, split-KV
+attention over the resident cache, merge, output projection, post-norm,
+gate/up, SwiGLU, down projection, pooling and readout).  Inputs are resident
+in HBM before timing; L2 is flushed (a 256 MiB write) between steps; each step
+is timed with CUDA events on the launching stream.  Prints one JSON line.
+
+Multi-GPU: the path shards by sequence with no exchange step, so N ranks run N
+independent replicas (weak scaling) and `value` counts all ranks' sequences
+over the slowest rank's time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "classified sequences/sec and µs/call at 1 GB300; achieved HBM GB/s vs 8 TB/s"
+UNIT = "sequences/s"
+FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS = 6800.0, 1900.0
+FLUSH_BYTES = 256 << 20
+
+# DRAM traffic per launch of the dominant kernel from an ncu capture of the same
+# kernel build (profiles/); None until one is taken for the current kernel.
+TRAFFIC_BYTES = {}
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--workload", default="4b")
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--rows", default="per-seq", choices=["per-seq", "shared"],
+                   help="per-seq: per-sequence input rows (full layer per call); "
+                        "shared: the soft prompt, whose Q/K/V projection is precomputed")
+    p.add_argument("--cpu-seconds", type=float, default=12.0)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            mp = json.load(f)
+        return float(mp["hbm_gbs"]), float(mp["bf16_tflops"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+
+
+# --------------------------------------------------------------------------- #
+# the algorithmic work model (bytes and flops every stage must move/do)
+# --------------------------------------------------------------------------- #
+def work_model(w, per_seq_rows: bool):
+    sh = w.shape
+    B, k, d = len(w.seq_ids), sh.k_rows, sh.d_model
+    hq, hkv, dh, f, C = sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.d_ff, sh.n_classes
+    es = 2 if sh.w_dtype == 1 else 4
+    kes = 2 if sh.kv_dtype == 1 else 4
+    M = B * k
+    lens = w.cache.seq_lens[w.seq_ids].astype(np.int64)
+    nqkv = (hq + 2 * hkv) * dh
+
+    def gemm(N, K):
+        return {"bytes": N * K * es + M * K * es + M * N * es, "flops": 2 * M * N * K}
+
+    st = {}
+    if per_seq_rows:
+        st["qkv"] = gemm(nqkv, d)
+    kv_bytes = int(lens.sum()) * hkv * dh * 2 * kes
+    st["attention"] = {"bytes": kv_bytes + M * nqkv * 4 + M * hq * dh * 4,
+                       "flops": int(4 * dh * hq * (k * lens.sum() + B * k * (k + 1) // 2))}
+    st["o_proj"] = gemm(d, hq * dh)
+    st["gate_up"] = gemm(2 * f, d)
+    st["down"] = gemm(d, f)
+    st["readout"] = {"bytes": C * d * 4 + M * d * 4, "flops": 2 * B * C * d}
+    total_bytes = sum(v["bytes"] for v in st.values())
+    weight_bytes = ((nqkv * d if per_seq_rows else 0) + d * hq * dh + 3 * f * d) * es + C * d * 4
+    return st, {"kv_bytes": kv_bytes, "weight_bytes": weight_bytes, "total_bytes": total_bytes,
+                "total_flops": sum(v["flops"] for v in st.values())}
+
+
+# --------------------------------------------------------------------------- #
+# clocks
+# --------------------------------------------------------------------------- #
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.out,
+                stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.3)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.out.close()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- #
+# reference arm: the fp64 oracle on the host cores
+# --------------------------------------------------------------------------- #
+def cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def oracle_rate(w, per_seq_rows: bool, seconds: float, max_seqs: int | None = None):
+    """Sequences/s of the oracle over successive sequences of the workload."""
+    import oracle.sp_oracle as so
+    layer = so.Layer(w.shape, w.weights)
+    n = 0
+    t0 = time.perf_counter()
+    B = len(w.seq_ids)
+    while True:
+        i = n % B
+        rows = w.rows[i:i + 1] if (per_seq_rows and w.rows is not None) else None
+        so.classify(layer, w.cache, w.seq_ids[i:i + 1], rows)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or (max_seqs is not None and n >= max_seqs):
+            return n / el, n, el
+
+
+def run_reference(args, spec, w, rank, world):
+    if rank != 0:
+        return
+    per_seq = args.rows == "per-seq"
+    import oracle.sp_oracle as so
+    layer = so.Layer(w.shape, w.weights)
+    B = len(w.seq_ids)
+    times, counts = [], []
+    per_step = max(1, min(B, 2))
+    for step in range(args.warmup + args.steps):
+        ids = [(step * per_step + j) % B for j in range(per_step)]
+        rows = w.rows[ids] if (per_seq and w.rows is not None) else None
+        t0 = time.perf_counter()
+        so.classify(layer, w.cache, w.seq_ids[ids], rows)
+        el = time.perf_counter() - t0
+        if step >= args.warmup:
+            times.append(el)
+            counts.append(per_step)
+    value = sum(counts) / sum(times)
+    sample = (f"{per_step} sequence(s) of workload {spec.name} per step, "
+              f"{args.steps} steps after {args.warmup} warm-up")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(spec, w, args),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(spec, w, args):
+    sh = w.shape
+    lens = w.cache.seq_lens[w.seq_ids]
+    return {"workload": spec.name, "batch": len(w.seq_ids),
+            "seq_len": (f"{spec.len_lo}" if spec.len_lo == spec.len_hi
+                        else f"U[{spec.len_lo},{spec.len_hi}] mean {float(lens.mean()):.0f}"),
+            "d_model": sh.d_model, "heads": f"{sh.n_q_heads}q/{sh.n_kv_heads}kv",
+            "head_dim": sh.head_dim, "d_ff": sh.d_ff, "k_rows": sh.k_rows,
+            "n_classes": sh.n_classes,
+            "kv_layout": "paged16" if w.cache.layout == 1 else "contiguous",
+            "rows": args.rows, "seed": spec.seed,
+            "l2": "flushed between steps (256 MiB write)", "timing": "CUDA events per step"}
+
+
+# --------------------------------------------------------------------------- #
+# our arm
+# --------------------------------------------------------------------------- #
+def run_ours(args, spec, w, rank, world):
+    import torch
+    import torch.distributed as dist
+
+    import paper_2608_28099_gb300 as sp
+    from paper_2608_28099_gb300 import build_lib
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if rank == 0:
+        build_lib.build()
+    if world > 1:
+        dist.barrier()
+    sp.load_library()
+    per_seq = args.rows == "per-seq"
+    B = len(w.seq_ids)
+    lens = w.cache.seq_lens
+    model = sp.Model(w.shape, w.weights, B, int(lens.max(initial=0)))
+    h = model.handle
+    cache = sp.DeviceCache(w.cache)
+    ids = torch.from_numpy(np.ascontiguousarray(w.seq_ids, dtype=np.int32)).cuda()
+    rows = None
+    if per_seq:
+        r = np.ascontiguousarray(w.rows)
+        rows = torch.from_numpy(r.view(np.int16) if r.dtype == np.uint16 else r).cuda()
+    logits = torch.empty((B, w.shape.n_classes), dtype=torch.float32, device="cuda")
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step():
+        sp.sp_classify(h, stream, B, ids, cache.seq_lens, cache.desc, rows, logits)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    assert sp.sp_check_status(h) == 0, sp.sp_last_error()
+    launches_per_step = sp.sp_last_launch_count(h)
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record(stream)
+        step()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    clk = clocks.stop()
+    ms = sum(step_ms) / len(step_ms)
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    # per-stage device times from events the library records on the same stream
+    sp.sp_set_option(h, sp.SP_OPT_PROFILE, 1)
+    acc = {}
+    for i in range(args.steps):
+        flush.zero_()
+        step()
+        for name, v in sp.sp_stage_times(h).items():
+            acc.setdefault(name, []).append(v)
+    sp.sp_set_option(h, sp.SP_OPT_PROFILE, 0)
+    stage_ms = {k: sum(v) / len(v) for k, v in acc.items()}
+
+    # end to end through the host entry point: pinned inputs up, logits down
+    h_ids = torch.from_numpy(np.ascontiguousarray(w.seq_ids, dtype=np.int32)).pin_memory()
+    h_lens = torch.from_numpy(np.ascontiguousarray(lens[w.seq_ids], dtype=np.int32)).pin_memory()
+    h_rows = rows.cpu().pin_memory() if rows is not None else None
+    h_logits = torch.empty((B, w.shape.n_classes), dtype=torch.float32).pin_memory()
+    e2e_s = []
+    for i in range(args.warmup + args.steps):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        sp.sp_classify_host(h, stream, B, h_ids, h_lens, cache.desc, h_rows, h_logits)
+        el = time.perf_counter() - t0
+        if i >= args.warmup:
+            e2e_s.append(el)
+    e2e_mean = sum(e2e_s) / len(e2e_s)
+    if world > 1:
+        t = torch.tensor([e2e_mean], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_mean = float(t.item())
+    h2d = h_ids.numel() * 4 + h_lens.numel() * 4 + (h_rows.numel() * h_rows.element_size()
+                                                     if h_rows is not None else 0)
+    d2h = h_logits.numel() * 4
+
+    if rank != 0:
+        model.close()
+        return
+    hbm, tfl, peak_src = peaks()
+    st_work, totals = work_model(w, per_seq)
+    # dominant kernel: the stage with the largest device time
+    named = {"attention": "attention", "qkv": "qkv", "o_proj": "o_proj", "gate_up": "gate_up",
+             "down": "down", "readout": "readout"}
+    cand = {k: v for k, v in stage_ms.items() if k in named and k in st_work}
+    dom = max(cand, key=cand.get)
+    wk = st_work[dom]
+    dur_s = stage_ms[dom] / 1e3
+    intensity = wk["flops"] / wk["bytes"]
+    ridge = tfl * 1e12 / (hbm * 1e9)
+    if intensity > ridge:
+        bound, ach, peak, unit = "tensor", wk["flops"] / dur_s / 1e12, tfl, "TFLOP/s"
+    else:
+        bound, ach, peak, unit = "hbm", wk["bytes"] / dur_s / 1e9, hbm, "GB/s"
+    traffic = TRAFFIC_BYTES.get((spec.name, dom))
+    roofline = {"bound": bound, "kernel": dom, "achieved": ach, "peak": peak, "unit": unit,
+                "frac": ach / peak, "traffic": traffic,
+                "peak_source": f"{peak_src} ({'hbm_gbs' if bound == 'hbm' else 'bf16_tflops'})",
+                "algorithmic_bytes": wk["bytes"], "algorithmic_flops": wk["flops"],
+                "ms": stage_ms[dom]}
+    path_bytes = totals["total_bytes"]
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        rate, n, el = oracle_rate(w, per_seq, args.cpu_seconds)
+        cpu = {"value": rate, "unit": UNIT, "cores": cores(), "kind": "oracle",
+               "sample": f"{n} sequences of workload {spec.name} one at a time, {el:.1f} s"}
+    value = world * B / (ms / 1e3)
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "us_per_call": ms * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16"
+            if w.shape.w_dtype == 1 else "f32", "data": "synthetic (seeded, random-init)",
+            "config": workload_config(spec, w, args),
+            "hbm": {"algorithmic_bytes_per_call": path_bytes,
+                    "gbs": path_bytes / (ms / 1e3) / 1e9,
+                    "frac_of_8tbs": path_bytes / (ms / 1e3) / 8e12,
+                    "frac_of_measured": path_bytes / (ms / 1e3) / (hbm * 1e9),
+                    "kv_bytes": totals["kv_bytes"], "weight_bytes": totals["weight_bytes"]},
+            "roofline": roofline,
+            "stages_ms": stage_ms,
+            "cpu_baseline": cpu,
+            "e2e": {"value": world * B / e2e_mean, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "ms_per_step": e2e_mean * 1e3},
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clk}
+    print(json.dumps(line), flush=True)
+    model.close()
+
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        if args.impl == "reference":
+            if rank != 0:
+                return
+        else:
+            import torch
+            torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+            dist.init_process_group("nccl")
+    from paper_2608_28099_gb300 import workloads as wl
+    spec = wl.named(args.workload, rows_per_seq=(args.rows == "per-seq"))
+    w = wl.generate(spec)
+    if args.impl == "reference":
+        run_reference(args, spec, w, rank, world)
+    else:
+        run_ours(args, spec, w, rank, world)
+    if world > 1 and args.impl != "reference":
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,257 @@
+/*
+ * sp.h -- C ABI of the Speculative Probing classify path (libsp.so).
+ *
+ * Speculative Probing (Sec. 3.2) classifies a sequence by appending k learned
+ * soft-prompt rows after it and running the frozen single decoder layer of the
+ * speculative-decoding draft head (Sec. 3.1) over those rows.  Their attention
+ * reads the sequence's keys/values already resident in the draft head's cache
+ * (Sec. 3.3, Eq. 1-3); a linear head then reads class logits from the pooled
+ * outputs (Sec. 3.2, "Classification head").  This library evaluates that path
+ * on one GPU, in hand-written CUDA for sm_103a.
+ *
+ * Per row r = 0..k-1 of sequence b (cached length L_b, position L_b + r):
+ *   x_hat = RMSNorm(x_r; g_in)
+ *   q, k', v' = W_q x_hat, W_k x_hat, W_v x_hat; q, k' rotated at L_b + r
+ *   o = softmax(q [K_cache ; k'_0..r]^T / sqrt(dh)) [V_cache ; v'_0..r]
+ *   h1 = x_r + W_o o ;  n = RMSNorm(h1; g_post)
+ *   h2_r = h1 + W_down (silu(W_gate n) * W_up n)
+ * logits_b = W_head pool_r(h2_r) + head_b      (pool: mean over r, or r = k-1)
+ * Query head h reads KV head h / (n_q_heads / n_kv_heads).  Rotation is the
+ * rotate-half form: pair (i, i + dh/2) turns by (L_b + r) * theta^(-2i/dh).
+ *
+ * Conventions for every entry point:
+ *  - Host pointers are named h_*, device pointers d_*; the stream argument is a
+ *    cudaStream_t (NULL = the legacy default stream).
+ *  - Calls that take a stream are asynchronous on it unless stated otherwise;
+ *    they neither synchronise nor allocate.
+ *  - Arguments are validated on the host before any launch; a rejected call
+ *    returns SP_ERR_INVALID_ARG or SP_ERR_UNSUPPORTED and launches nothing.
+ *  - Problems only the device can see (a sequence id or cached length out of
+ *    range, a page id outside the pool) never fault: the kernels skip the bad
+ *    access, treat it as masked, and set bits of a device status word that
+ *    sp_check_status() returns as SP_ERR_DEVICE_STATUS.
+ *  - sp_last_error() returns a per-thread description of the last failure.
+ *  - The caches passed in are only read, never written (Sec. 3.3, "Monitoring
+ *    does not disturb speculative decoding"): the k new keys/values go to
+ *    library-owned scratch memory.
+ */
+#ifndef SP_H
+#define SP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SP_API __attribute__((visibility("default")))
+#else
+#define SP_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct sp_handle sp_handle;
+typedef struct CUstream_st *sp_stream; /* identical to cudaStream_t */
+
+typedef enum sp_status {
+    SP_OK = 0,
+    SP_ERR_INVALID_ARG = 1,   /* bad pointer, size or enum; nothing launched        */
+    SP_ERR_UNSUPPORTED = 2,   /* valid but not implemented (e.g. head_dim 96)       */
+    SP_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed                  */
+    SP_ERR_OOM = 4,           /* device allocation failed in sp_create              */
+    SP_ERR_DEVICE_STATUS = 5  /* the device reported bad ids/lengths/pages          */
+} sp_status;
+
+enum { SP_F32 = 0, SP_BF16 = 1 };              /* element types                  */
+enum { SP_POOL_MEAN = 0, SP_POOL_LAST = 1 };   /* which outputs the head reads   */
+enum { SP_KV_CONTIGUOUS = 0, SP_KV_PAGED = 1 };/* cache addressing               */
+
+/* Device status bits (OR-ed together). */
+enum {
+    SP_DEV_BAD_SEQ_ID = 1,    /* a sequence id was outside [0, n_seqs)               */
+    SP_DEV_BAD_LENGTH = 2,    /* a cached length was < 0 or > max_seq_len            */
+    SP_DEV_BAD_PAGE = 4       /* a page-table entry was outside [0, n_pages)         */
+};
+
+/* Shapes of the frozen layer and of the probe (Sec. 3.1, 3.2). */
+typedef struct sp_config {
+    int d_model;      /* hidden size d; multiple of 8                                */
+    int n_q_heads;    /* query heads Hq; a multiple of n_kv_heads                    */
+    int n_kv_heads;   /* key/value heads Hkv (grouped-query attention)               */
+    int head_dim;     /* dh: 32, 64 or 128                                           */
+    int d_ff;         /* SwiGLU intermediate size; multiple of 8                     */
+    int k_rows;       /* soft-prompt rows k appended per sequence, 1..32             */
+    int n_classes;    /* C >= 1 rows of the linear head                              */
+    float rope_theta; /* rotary base theta                                           */
+    float rms_eps;    /* RMSNorm epsilon (added to the mean square)                  */
+    int pool;         /* SP_POOL_MEAN or SP_POOL_LAST                                */
+    int w_dtype;      /* SP_F32 or SP_BF16: layer matrices, soft prompt, input rows  */
+    int kv_dtype;     /* SP_F32 or SP_BF16: cached keys/values                       */
+    int max_batch;    /* largest batch passed to sp_classify (sizes the scratch)     */
+    int max_seq_len;  /* largest cached length L_b (sizes the split plan)            */
+} sp_config;
+
+/* Layer and probe parameters: HOST pointers, read once by sp_create and
+ * copied to the device (the caller may free them afterwards).  Matrices are
+ * row-major [out][in] in w_dtype (bf16 as raw 16-bit patterns):
+ *   w_q [Hq*dh][d], w_k [Hkv*dh][d], w_v [Hkv*dh][d], w_o [d][Hq*dh],
+ *   w_gate [d_ff][d], w_up [d_ff][d], w_down [d][d_ff],
+ *   soft_prompt [k][d] (w_dtype), g_in [d], g_post [d] (float),
+ *   head_w [C][d] (float), head_b [C] (float, may be NULL = zero bias). */
+typedef struct sp_weights {
+    const void *w_q, *w_k, *w_v, *w_o, *w_gate, *w_up, *w_down;
+    const float *g_in, *g_post;
+    const void *soft_prompt;
+    const float *head_w, *head_b;
+} sp_weights;
+
+/* A resident key/value cache (Sec. 3.3): DEVICE pointers, borrowed for the
+ * duration of the stream work of one call and never written.  Keys are stored
+ * already rotated at their own positions 0..L_b-1.
+ *  SP_KV_CONTIGUOUS: k_seq/v_seq are DEVICE arrays of n_seqs device pointers;
+ *    sequence s is token-major [L_s][Hkv][dh] in kv_dtype.
+ *  SP_KV_PAGED: k_pool/v_pool hold n_pages pages laid out
+ *    [page][Hkv][page_size][dh]; page_table is a DEVICE int32 array
+ *    [n_seqs][max_pages_per_seq]; token t of sequence s sits in page
+ *    page_table[s][t / page_size], slot t % page_size.  Entries past
+ *    ceil(L_s / page_size) are never read; a length that would need more than
+ *    max_pages_per_seq pages is reported as SP_DEV_BAD_PAGE and the excess is
+ *    masked.  page_size: 16, 32 or 64.
+ *  A contiguous buffer must hold min(L_s, max_seq_len) tokens: its size is not
+ *  known to the library, so a length beyond it cannot be detected. */
+typedef struct sp_kv_cache {
+    int layout;
+    const void *const *k_seq;
+    const void *const *v_seq;
+    const void *k_pool;
+    const void *v_pool;
+    const int *page_table;
+    int page_size;
+    int n_pages;
+    int max_pages_per_seq;
+    int n_seqs;
+} sp_kv_cache;
+
+/* Build a handle on the current CUDA device: validates the shapes, copies the
+ * weights, precomputes the projections of the shared soft prompt and sizes all
+ * scratch memory for cfg->max_batch.  The handle owns every device buffer it
+ * allocates.  One handle serves one stream at a time (its scratch is shared by
+ * consecutive calls).  Returns SP_OK and *out, or an error with *out = NULL. */
+SP_API sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out);
+
+/* Free a handle and everything it owns; waits for the device to go idle first.
+ * NULL is accepted and ignored. */
+SP_API sp_status sp_destroy(sp_handle *h);
+
+/* The classify path (Sec. 3.2-3.3): logits for `batch` sequences of a resident
+ * cache, enqueued on `stream`, no synchronisation, no allocation.
+ *   d_seq_ids  [batch] int32 device: which cache sequences to classify
+ *              (NULL: sequences 0..batch-1).
+ *   d_seq_lens [kv->n_seqs] int32 device: cached length of every sequence;
+ *              only the entries of the classified ids are read.
+ *   kv         the cache (see sp_kv_cache); kv_dtype must match the handle.
+ *   d_rows     [batch][k][d] device, w_dtype: the per-sequence input rows of
+ *              the layer (e.g. an MTP head's fused inputs), or NULL: every
+ *              sequence uses the handle's shared soft prompt rows.
+ *   d_logits   [batch][C] float device, caller-owned: raw class logits.
+ * 1 <= batch <= max_batch.  Device-side range problems are reported through
+ * sp_check_status(). */
+SP_API sp_status sp_classify(sp_handle *h, sp_stream stream, int batch, const int *d_seq_ids,
+                      const int *d_seq_lens, const sp_kv_cache *kv, const void *d_rows,
+                      float *d_logits);
+
+/* sp_classify from HOST buffers: copies h_seq_ids [batch] (NULL = 0..batch-1),
+ * h_seq_lens [batch] (the cached length of each classified sequence, in batch
+ * order) and h_rows [batch][k][d] (NULL = shared prompt) to
+ * handle-owned device staging, runs the path, copies the logits back to
+ * h_logits [batch][C] and synchronises `stream`.  The cache stays on the
+ * device.  Also returns any device status as SP_ERR_DEVICE_STATUS.  Pinned host
+ * buffers make the copies asynchronous DMA transfers. */
+SP_API sp_status sp_classify_host(sp_handle *h, sp_stream stream, int batch, const int *h_seq_ids,
+                           const int *h_seq_lens, const sp_kv_cache *kv, const void *h_rows,
+                           float *h_logits);
+
+/* Synchronise `stream`, read and clear the handle's device status word.
+ * Returns SP_OK, or SP_ERR_DEVICE_STATUS with the SP_DEV_* bits in *bits. */
+SP_API sp_status sp_check_status(sp_handle *h, sp_stream stream, int *bits);
+
+/* Per-thread text describing the last failure of any entry point. */
+SP_API const char *sp_last_error(void);
+
+/* Options (tests and benchmarks).  Returns SP_ERR_INVALID_ARG for an unknown
+ * key or value. */
+enum {
+    SP_OPT_SPLIT_TOKENS = 1,  /* attention tokens per split-KV work unit (multiple
+                                 of 64), 0 = automatic plan                      */
+    SP_OPT_GEMM_PATH = 2,     /* 0 = automatic, 1 = CUDA-core kernels only,
+                                 2 = tensor-core kernels wherever supported       */
+    SP_OPT_ATTN_PATH = 3,     /* 0 = automatic, 1 = CUDA-core kernel only,
+                                 2 = tensor-core kernel wherever supported        */
+    SP_OPT_PROFILE = 4        /* 1 = record CUDA events around every stage of
+                                 sp_classify on its stream, 0 = off (default)    */
+};
+
+/* Stages of sp_classify, in launch order. */
+enum {
+    SP_STAGE_INPUT_NORM = 0,  /* a1: RMSNorm of per-sequence rows                    */
+    SP_STAGE_QKV = 1,         /* a2: Q/K/V projection (skipped for the shared prompt) */
+    SP_STAGE_ROPE = 2,        /* a2: rotation at L_b + r, new keys to scratch        */
+    SP_STAGE_ATTN = 3,        /* a3: split-KV attention over [cache ; new keys]      */
+    SP_STAGE_MERGE = 4,       /* a3: log-sum-exp merge of the splits                 */
+    SP_STAGE_O_PROJ = 5,      /* a4: output projection                               */
+    SP_STAGE_POST_NORM = 6,   /* a4: residual + post-norm                            */
+    SP_STAGE_GATE_UP = 7,     /* a5: gate/up projection                              */
+    SP_STAGE_SWIGLU = 8,      /* a5: SwiGLU                                          */
+    SP_STAGE_DOWN = 9,        /* a6: down projection                                 */
+    SP_STAGE_READOUT = 10,    /* a6-a7: residual, pooling, linear head               */
+    SP_N_STAGES = 11
+};
+
+/* With SP_OPT_PROFILE on: synchronise on the last call's events and write the
+ * device time (ms) of each stage of that call to ms[0..n-1] (-1 for a stage the
+ * call did not run).  Returns SP_ERR_INVALID_ARG when profiling is off. */
+SP_API sp_status sp_stage_times(sp_handle *h, float *ms, int n);
+SP_API sp_status sp_set_option(sp_handle *h, int key, int value);
+
+/* Number of kernel launches the last sp_classify enqueued. */
+SP_API int sp_last_launch_count(const sp_handle *h);
+
+/* ------------------------------------------------------------------------- */
+/* The attention step alone (Eq. 1-3), for step-level checks and for callers  */
+/* that run their own projections.                                            */
+/* ------------------------------------------------------------------------- */
+typedef struct sp_attn_dims {
+    int n_q_heads, n_kv_heads, head_dim; /* as in sp_config                         */
+    int k_rows;                          /* query rows per sequence (k), 1..32      */
+    int kv_dtype;                        /* SP_F32 or SP_BF16                       */
+    int max_seq_len;                     /* bound on the cached lengths             */
+    int split_tokens;                    /* tokens per split-KV work unit (multiple
+                                            of 64), 0 = automatic plan              */
+} sp_attn_dims;
+
+/* Bytes of device scratch sp_attend needs for `batch` sequences (256-byte
+ * aligned start required); 0 for invalid dims. */
+SP_API size_t sp_attend_workspace_bytes(const sp_attn_dims *dims, int batch);
+
+/* Attention of k rotated query rows per sequence over [cache ; new keys]:
+ *   d_q     [batch][k][Hq][dh] float device (already rotated)
+ *   d_k_new [batch][k][Hkv][dh] float device (already rotated), d_v_new same
+ *   d_out   [batch][k][Hq][dh], float (out_dtype SP_F32) or bf16 (SP_BF16)
+ * Row r of sequence b sees the L_b cached tokens and new tokens 0..r.
+ * d_workspace: caller-allocated, >= sp_attend_workspace_bytes(dims, batch).
+ * d_status: optional device int (OR-ed SP_DEV_* bits), NULL = not recorded.
+ * d_gathered_pages: optional device int32 [batch][kv->max_pages_per_seq]
+ *   (paged caches only): entry [i][j] receives the physical page id the kernel
+ *   read for logical page j of the i-th sequence; entries it did not read are
+ *   left untouched.  NULL = not recorded. */
+SP_API sp_status sp_attend(sp_stream stream, const sp_attn_dims *dims, int batch, const int *d_seq_ids,
+                    const int *d_seq_lens, const sp_kv_cache *kv, const float *d_q,
+                    const float *d_k_new, const float *d_v_new, void *d_out, int out_dtype,
+                    void *d_workspace, size_t workspace_bytes, int *d_status,
+                    int *d_gathered_pages);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SP_H */

@@ -1,0 +1,606 @@
+// C ABI of libsp.so: handle lifetime, argument checks, the classify launch
+// sequence (Sec. 3.2-3.3) and the stand-alone attention step (Eq. 1-3).
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <string>
+#include <vector>
+
+#include "sp_common.cuh"
+#include "sp_gemm.cuh"
+
+using namespace sp;
+
+namespace {
+
+thread_local std::string g_err;
+
+sp_status fail(sp_status st, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return st;
+}
+
+#define SP_CUDA(call)                                                                       \
+    do {                                                                                    \
+        cudaError_t e_ = (call);                                                            \
+        if (e_ != cudaSuccess)                                                              \
+            return fail(SP_ERR_CUDA, "%s failed: %s (%s:%d)", #call, cudaGetErrorString(e_), \
+                        __FILE__, __LINE__);                                                \
+    } while (0)
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// One device allocation carved into 256-byte aligned pieces.
+struct Arena {
+    char *base = nullptr;
+    size_t used = 0, cap = 0;
+    void *take(size_t bytes) {
+        void *p = base + used;
+        used += align256(bytes);
+        return p;
+    }
+};
+
+}  // namespace
+
+struct sp_handle {
+    sp_config cfg;
+    int device = 0, n_sm = 148;
+    int es = 2;        // bytes per weight/activation element
+    int nqkv = 0;      // (Hq + 2 Hkv) dh
+    int gu_blk = 0;    // gate/up interleave block (columns)
+    // weights
+    void *w_qkv = nullptr, *w_o = nullptr, *w_gu = nullptr, *w_down = nullptr;
+    float *g_in = nullptr, *g_post = nullptr, *head_w = nullptr, *head_b = nullptr;
+    void *soft_prompt = nullptr;
+    float *qkv_shared = nullptr;  // [k][nqkv] projections of the shared soft prompt
+    float2 *rope_cs = nullptr;    // [max_seq_len + k][dh/2]
+    // scratch
+    Arena arena;
+    void *xn = nullptr;           // [M][d] activation dtype
+    float *y = nullptr;           // [M][max N] projection output
+    float *q = nullptr, *k_new = nullptr, *v_new = nullptr;
+    void *attn_ws = nullptr;
+    size_t attn_ws_bytes = 0;
+    void *o = nullptr;            // [M][Hq dh]
+    float *h1 = nullptr;          // [M][d]
+    void *n = nullptr;            // [M][d]
+    void *a = nullptr;            // [M][d_ff]
+    int *status = nullptr;
+    int *stage_ids = nullptr, *stage_lens = nullptr;
+    void *stage_rows = nullptr;
+    float *stage_logits = nullptr;
+    GemmPlanner gemm;
+    // options
+    int opt_split = 0, opt_gemm = 0, opt_attn = 0, opt_profile = 0;
+    int last_launches = 0;
+    cudaEvent_t ev[SP_N_STAGES][2] = {};
+    bool ev_used[SP_N_STAGES] = {};
+    std::vector<void *> allocs;
+};
+
+namespace {
+
+sp_status dev_alloc(sp_handle *h, void **p, size_t bytes) {
+    *p = nullptr;
+    if (bytes == 0) bytes = 256;
+    cudaError_t e = cudaMalloc(p, bytes);
+    if (e != cudaSuccess) {
+        *p = nullptr;
+        return fail(SP_ERR_OOM, "cudaMalloc(%zu) failed: %s", bytes, cudaGetErrorString(e));
+    }
+    h->allocs.push_back(*p);
+    return SP_OK;
+}
+
+sp_status upload(sp_handle *h, void **dst, const void *src, size_t bytes) {
+    sp_status st = dev_alloc(h, dst, bytes);
+    if (st != SP_OK) return st;
+    SP_CUDA(cudaMemcpy(*dst, src, bytes, cudaMemcpyHostToDevice));
+    return SP_OK;
+}
+
+sp_status check_config(const sp_config *c) {
+    if (!c) return fail(SP_ERR_INVALID_ARG, "config is NULL");
+    if (c->d_model <= 0 || c->d_model % 8) return fail(SP_ERR_INVALID_ARG, "d_model must be a positive multiple of 8");
+    if (c->n_kv_heads <= 0 || c->n_q_heads <= 0 || c->n_q_heads % c->n_kv_heads)
+        return fail(SP_ERR_INVALID_ARG, "n_q_heads must be a positive multiple of n_kv_heads");
+    if (c->head_dim != 32 && c->head_dim != 64 && c->head_dim != 128)
+        return fail(SP_ERR_UNSUPPORTED, "head_dim %d unsupported (32, 64, 128)", c->head_dim);
+    if (c->d_ff <= 0 || c->d_ff % 8) return fail(SP_ERR_INVALID_ARG, "d_ff must be a positive multiple of 8");
+    if (c->k_rows < 1 || c->k_rows > 32) return fail(SP_ERR_INVALID_ARG, "k_rows must be in 1..32");
+    if (c->n_classes < 1) return fail(SP_ERR_INVALID_ARG, "n_classes must be >= 1");
+    if (c->pool != SP_POOL_MEAN && c->pool != SP_POOL_LAST) return fail(SP_ERR_INVALID_ARG, "bad pool");
+    if (c->w_dtype != SP_F32 && c->w_dtype != SP_BF16) return fail(SP_ERR_INVALID_ARG, "bad w_dtype");
+    if (c->kv_dtype != SP_F32 && c->kv_dtype != SP_BF16) return fail(SP_ERR_INVALID_ARG, "bad kv_dtype");
+    if (c->max_batch < 1) return fail(SP_ERR_INVALID_ARG, "max_batch must be >= 1");
+    if (c->max_seq_len < 0) return fail(SP_ERR_INVALID_ARG, "max_seq_len must be >= 0");
+    if (!(c->rope_theta > 0.f) || !(c->rms_eps >= 0.f)) return fail(SP_ERR_INVALID_ARG, "bad theta/eps");
+    const int R = (c->n_q_heads / c->n_kv_heads) * c->k_rows;
+    if (R * c->head_dim > 128 * 128)
+        return fail(SP_ERR_UNSUPPORTED, "query group x k_rows x head_dim too large (%d rows)", R);
+    return SP_OK;
+}
+
+sp_status check_kv(const sp_kv_cache *kv, int kv_dtype) {
+    (void)kv_dtype;
+    if (!kv) return fail(SP_ERR_INVALID_ARG, "kv cache descriptor is NULL");
+    if (kv->n_seqs < 1) return fail(SP_ERR_INVALID_ARG, "kv->n_seqs must be >= 1");
+    if (kv->layout == SP_KV_CONTIGUOUS) {
+        if (!kv->k_seq || !kv->v_seq) return fail(SP_ERR_INVALID_ARG, "contiguous cache needs k_seq and v_seq");
+    } else if (kv->layout == SP_KV_PAGED) {
+        if (!kv->k_pool || !kv->v_pool || !kv->page_table)
+            return fail(SP_ERR_INVALID_ARG, "paged cache needs k_pool, v_pool and page_table");
+        if (kv->page_size != 16 && kv->page_size != 32 && kv->page_size != 64)
+            return fail(SP_ERR_UNSUPPORTED, "page_size %d unsupported (16, 32, 64)", kv->page_size);
+        if (kv->n_pages < 1 || kv->max_pages_per_seq < 1)
+            return fail(SP_ERR_INVALID_ARG, "n_pages and max_pages_per_seq must be >= 1");
+    } else {
+        return fail(SP_ERR_INVALID_ARG, "bad kv layout %d", kv->layout);
+    }
+    return SP_OK;
+}
+
+KVDev to_dev(const sp_kv_cache *kv) {
+    KVDev d;
+    d.layout = kv->layout;
+    d.k_seq = kv->k_seq;
+    d.v_seq = kv->v_seq;
+    d.k_pool = kv->k_pool;
+    d.v_pool = kv->v_pool;
+    d.page_table = kv->page_table;
+    d.page_size = kv->page_size;
+    d.n_pages = kv->n_pages;
+    d.max_pages = kv->max_pages_per_seq;
+    d.n_seqs = kv->n_seqs;
+    return d;
+}
+
+int sm_count() {
+    int dev = 0, n = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess)
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    return n;
+}
+
+// Largest attention workspace over every batch size up to max_batch.
+size_t max_attention_ws(const sp_config &c, int n_sm, int forced_split) {
+    const int G = c.n_q_heads / c.n_kv_heads;
+    size_t best = 0;
+    for (int B = 1; B <= c.max_batch; ++B) {
+        int split, ns;
+        plan_attention(B, c.n_kv_heads, c.k_rows, c.max_seq_len, forced_split, n_sm, &split, &ns);
+        size_t b = attention_workspace_bytes(B, c.n_kv_heads, G * c.k_rows, c.head_dim, ns);
+        if (b > best) best = b;
+    }
+    return best;
+}
+
+// Enqueue the attention step (split units + merge) for AttnArgs with the
+// partial buffers taken from `ws`.
+sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_path, int *launches,
+                            cudaStream_t st, cudaEvent_t *ev_attn = nullptr,
+                            cudaEvent_t *ev_merge = nullptr) {
+    const size_t need = attention_workspace_bytes(a.B, a.Hkv, a.R, a.dh, a.n_splits);
+    if (ws_bytes < need) return fail(SP_ERR_INVALID_ARG, "attention workspace too small (%zu < %zu)", ws_bytes, need);
+    a.part_o = (float *)ws;
+    a.part_ml = (float *)((char *)ws + align256((size_t)a.B * a.Hkv * a.n_splits * a.R * a.dh * sizeof(float)));
+    (void)attn_path;
+    if (ev_attn) cudaEventRecord(ev_attn[0], st);
+    SP_CUDA(launch_attention_simt(a, st));
+    if (ev_attn) cudaEventRecord(ev_attn[1], st);
+    if (ev_merge) cudaEventRecord(ev_merge[0], st);
+    SP_CUDA(launch_attention_merge(a, st));
+    if (ev_merge) cudaEventRecord(ev_merge[1], st);
+    *launches += 2;
+    return SP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *sp_last_error(void) { return g_err.c_str(); }
+
+sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) {
+    if (!out) return fail(SP_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    sp_status st = check_config(cfg);
+    if (st != SP_OK) return st;
+    if (!w || !w->w_q || !w->w_k || !w->w_v || !w->w_o || !w->w_gate || !w->w_up || !w->w_down ||
+        !w->g_in || !w->g_post || !w->soft_prompt || !w->head_w)
+        return fail(SP_ERR_INVALID_ARG, "a required weight pointer is NULL");
+
+    sp_handle *h = new sp_handle();
+    h->cfg = *cfg;
+    const sp_config &c = h->cfg;
+    cudaGetDevice(&h->device);
+    h->n_sm = sm_count();
+    h->es = c.w_dtype == SP_BF16 ? 2 : 4;
+    const int d = c.d_model, hq = c.n_q_heads, hkv = c.n_kv_heads, dh = c.head_dim, f = c.d_ff;
+    const int k = c.k_rows, C = c.n_classes;
+    h->nqkv = (hq + 2 * hkv) * dh;
+    h->gu_blk = f;  // gate block then up block (no interleave)
+    const size_t es = h->es;
+    auto cleanup = [&](sp_status s) {
+        sp_destroy(h);
+        return s;
+    };
+
+    // weights: [W_q; W_k; W_v] and [W_gate; W_up] concatenated along the output dim
+    {
+        std::vector<char> buf((size_t)h->nqkv * d * es);
+        memcpy(buf.data(), w->w_q, (size_t)hq * dh * d * es);
+        memcpy(buf.data() + (size_t)hq * dh * d * es, w->w_k, (size_t)hkv * dh * d * es);
+        memcpy(buf.data() + (size_t)(hq + hkv) * dh * d * es, w->w_v, (size_t)hkv * dh * d * es);
+        if ((st = upload(h, &h->w_qkv, buf.data(), buf.size())) != SP_OK) return cleanup(st);
+    }
+    {
+        std::vector<char> buf((size_t)2 * f * d * es);
+        memcpy(buf.data(), w->w_gate, (size_t)f * d * es);
+        memcpy(buf.data() + (size_t)f * d * es, w->w_up, (size_t)f * d * es);
+        if ((st = upload(h, &h->w_gu, buf.data(), buf.size())) != SP_OK) return cleanup(st);
+    }
+    if ((st = upload(h, &h->w_o, w->w_o, (size_t)d * hq * dh * es)) != SP_OK) return cleanup(st);
+    if ((st = upload(h, &h->w_down, w->w_down, (size_t)d * f * es)) != SP_OK) return cleanup(st);
+    if ((st = upload(h, (void **)&h->g_in, w->g_in, d * sizeof(float))) != SP_OK) return cleanup(st);
+    if ((st = upload(h, (void **)&h->g_post, w->g_post, d * sizeof(float))) != SP_OK) return cleanup(st);
+    if ((st = upload(h, &h->soft_prompt, w->soft_prompt, (size_t)k * d * es)) != SP_OK) return cleanup(st);
+    if ((st = upload(h, (void **)&h->head_w, w->head_w, (size_t)C * d * sizeof(float))) != SP_OK)
+        return cleanup(st);
+    if (w->head_b &&
+        (st = upload(h, (void **)&h->head_b, w->head_b, C * sizeof(float))) != SP_OK)
+        return cleanup(st);
+
+    // rotary table: angle (position p, pair i) = p * theta^(-2i/dh), evaluated in double
+    {
+        const int npos = c.max_seq_len + k, half = dh / 2;
+        std::vector<float2> cs((size_t)npos * half);
+        std::vector<double> freq(half);
+        for (int i = 0; i < half; ++i) freq[i] = pow((double)c.rope_theta, -2.0 * i / dh);
+        for (int p = 0; p < npos; ++p)
+            for (int i = 0; i < half; ++i) {
+                const double ang = (double)p * freq[i];
+                cs[(size_t)p * half + i] = make_float2((float)cos(ang), (float)sin(ang));
+            }
+        if ((st = upload(h, (void **)&h->rope_cs, cs.data(), cs.size() * sizeof(float2))) != SP_OK)
+            return cleanup(st);
+    }
+
+    // scratch for max_batch sequences
+    const size_t M = (size_t)c.max_batch * k;
+    size_t maxN = (size_t)h->nqkv;
+    if ((size_t)d > maxN) maxN = d;
+    if ((size_t)2 * f > maxN) maxN = 2 * (size_t)f;
+    h->attn_ws_bytes = max_attention_ws(c, h->n_sm, 0);
+    h->gemm.init(h->n_sm);
+    const size_t gemm_ws = h->gemm.workspace_bytes(M, maxN);
+    size_t total = 0;
+    const size_t sizes[] = {M * d * es,                 // xn
+                            M * maxN * 4 + gemm_ws,     // y (+ split-K partials)
+                            M * hq * dh * 4,            // q
+                            M * hkv * dh * 4,           // k_new
+                            M * hkv * dh * 4,           // v_new
+                            h->attn_ws_bytes,           // attention partials
+                            M * hq * dh * es,           // o
+                            M * d * 4,                  // h1
+                            M * d * es,                 // n
+                            M * f * es,                 // a
+                            256,                        // status
+                            (size_t)c.max_batch * 4,    // stage ids
+                            (size_t)c.max_batch * 4,    // stage lens
+                            M * d * es,                 // stage rows
+                            (size_t)c.max_batch * C * 4,  // stage logits
+                            (size_t)k * h->nqkv * 4};   // qkv_shared
+    for (size_t s : sizes) total += align256(s);
+    void *arena = nullptr;
+    if ((st = dev_alloc(h, &arena, total)) != SP_OK) return cleanup(st);
+    h->arena.base = (char *)arena;
+    h->arena.cap = total;
+    h->xn = h->arena.take(sizes[0]);
+    h->y = (float *)h->arena.take(sizes[1]);
+    h->q = (float *)h->arena.take(sizes[2]);
+    h->k_new = (float *)h->arena.take(sizes[3]);
+    h->v_new = (float *)h->arena.take(sizes[4]);
+    h->attn_ws = h->arena.take(sizes[5]);
+    h->o = h->arena.take(sizes[6]);
+    h->h1 = (float *)h->arena.take(sizes[7]);
+    h->n = h->arena.take(sizes[8]);
+    h->a = h->arena.take(sizes[9]);
+    h->status = (int *)h->arena.take(sizes[10]);
+    h->stage_ids = (int *)h->arena.take(sizes[11]);
+    h->stage_lens = (int *)h->arena.take(sizes[12]);
+    h->stage_rows = h->arena.take(sizes[13]);
+    h->stage_logits = (float *)h->arena.take(sizes[14]);
+    h->qkv_shared = (float *)h->arena.take(sizes[15]);
+    if (cudaMemset(h->status, 0, 256) != cudaSuccess) return cleanup(fail(SP_ERR_CUDA, "memset failed"));
+
+    // projections of the shared soft prompt rows (they do not depend on the sequence)
+    {
+        const int wb = c.w_dtype == SP_BF16;
+        cudaError_t e = launch_rmsnorm_rows(wb, h->soft_prompt, 0, h->g_in, c.rms_eps, k, d, h->xn, 0);
+        if (e == cudaSuccess)
+            e = launch_gemm_simt(wb, h->xn, h->w_qkv, h->qkv_shared, k, h->nqkv, d, 0);
+        if (e == cudaSuccess) e = cudaDeviceSynchronize();
+        if (e != cudaSuccess)
+            return cleanup(fail(SP_ERR_CUDA, "shared prompt projection failed: %s", cudaGetErrorString(e)));
+    }
+    *out = h;
+    return SP_OK;
+}
+
+sp_status sp_destroy(sp_handle *h) {
+    if (!h) return SP_OK;
+    cudaDeviceSynchronize();
+    for (auto &pair : h->ev)
+        for (cudaEvent_t &e : pair)
+            if (e) cudaEventDestroy(e);
+    for (void *p : h->allocs) cudaFree(p);
+    delete h;
+    return SP_OK;
+}
+
+sp_status sp_set_option(sp_handle *h, int key, int value) {
+    if (!h) return fail(SP_ERR_INVALID_ARG, "handle is NULL");
+    switch (key) {
+    case SP_OPT_SPLIT_TOKENS: {
+        if (value < 0 || value % 64) return fail(SP_ERR_INVALID_ARG, "split tokens must be a multiple of 64");
+        const size_t need = max_attention_ws(h->cfg, h->n_sm, value);
+        if (need > h->attn_ws_bytes)
+            return fail(SP_ERR_INVALID_ARG, "split of %d tokens needs more scratch than sp_create sized", value);
+        h->opt_split = value;
+        return SP_OK;
+    }
+    case SP_OPT_GEMM_PATH:
+        if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad gemm path");
+        h->opt_gemm = value;
+        return SP_OK;
+    case SP_OPT_ATTN_PATH:
+        if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad attention path");
+        h->opt_attn = value;
+        return SP_OK;
+    case SP_OPT_PROFILE:
+        if (value != 0 && value != 1) return fail(SP_ERR_INVALID_ARG, "bad profile flag");
+        if (value && !h->ev[0][0]) {
+            for (auto &pair : h->ev)
+                for (cudaEvent_t &e : pair) SP_CUDA(cudaEventCreate(&e));
+        }
+        h->opt_profile = value;
+        return SP_OK;
+    default:
+        return fail(SP_ERR_INVALID_ARG, "unknown option %d", key);
+    }
+}
+
+int sp_last_launch_count(const sp_handle *h) { return h ? h->last_launches : -1; }
+
+sp_status sp_stage_times(sp_handle *h, float *ms, int n) {
+    if (!h || !ms || n < 0) return fail(SP_ERR_INVALID_ARG, "bad arguments");
+    if (!h->opt_profile) return fail(SP_ERR_INVALID_ARG, "profiling is off (SP_OPT_PROFILE)");
+    for (int i = 0; i < n; ++i) {
+        ms[i] = -1.f;
+        if (i >= SP_N_STAGES || !h->ev_used[i]) continue;
+        SP_CUDA(cudaEventSynchronize(h->ev[i][1]));
+        SP_CUDA(cudaEventElapsedTime(&ms[i], h->ev[i][0], h->ev[i][1]));
+    }
+    return SP_OK;
+}
+
+static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const int *d_seq_ids,
+                               const int *d_seq_lens, int lens_by_batch, const sp_kv_cache *kv,
+                               const void *d_rows, float *d_logits) {
+    if (!h) return fail(SP_ERR_INVALID_ARG, "handle is NULL");
+    const sp_config &c = h->cfg;
+    if (batch < 1 || batch > c.max_batch)
+        return fail(SP_ERR_INVALID_ARG, "batch %d outside 1..max_batch (%d)", batch, c.max_batch);
+    if (!d_seq_lens || !d_logits) return fail(SP_ERR_INVALID_ARG, "seq_lens and logits are required");
+    sp_status s = check_kv(kv, c.kv_dtype);
+    if (s != SP_OK) return s;
+    if (!d_seq_ids && batch > kv->n_seqs)
+        return fail(SP_ERR_INVALID_ARG, "batch %d exceeds n_seqs %d with implicit ids", batch, kv->n_seqs);
+
+    const int d = c.d_model, hq = c.n_q_heads, hkv = c.n_kv_heads, dh = c.head_dim, f = c.d_ff;
+    const int k = c.k_rows, C = c.n_classes, G = hq / hkv;
+    const int M = batch * k;
+    const int wb = c.w_dtype == SP_BF16;
+    int launches = 0;
+    for (bool &u : h->ev_used) u = false;
+    auto mark = [&](int stage, int end) {
+        if (!h->opt_profile) return;
+        cudaEventRecord(h->ev[stage][end], st);
+        h->ev_used[stage] = true;
+    };
+
+    // a1-a2: pre-norm, Q/K/V projection, rotation at positions L_b + r
+    const float *yqkv = h->qkv_shared;
+    if (d_rows) {
+        mark(SP_STAGE_INPUT_NORM, 0);
+        SP_CUDA(launch_rmsnorm_rows(wb, d_rows, 0, h->g_in, c.rms_eps, M, d, h->xn, st));
+        mark(SP_STAGE_INPUT_NORM, 1);
+        ++launches;
+        mark(SP_STAGE_QKV, 0);
+        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->nqkv, d, st, &launches);
+        mark(SP_STAGE_QKV, 1);
+        if (s != SP_OK) return s;
+        yqkv = h->y;
+    }
+    QkvRopeArgs r;
+    r.y = yqkv;
+    r.shared = d_rows ? 0 : 1;
+    r.B = batch; r.k = k; r.Hq = hq; r.Hkv = hkv; r.dh = dh;
+    r.seq_ids = d_seq_ids; r.seq_lens = d_seq_lens; r.lens_by_batch = lens_by_batch;
+    r.n_seqs = kv->n_seqs; r.max_seq_len = c.max_seq_len;
+    r.rope_cs = h->rope_cs;
+    r.q = h->q; r.k_new = h->k_new; r.v_new = h->v_new;
+    r.status = h->status;
+    mark(SP_STAGE_ROPE, 0);
+    SP_CUDA(launch_qkv_rope(r, st));
+    mark(SP_STAGE_ROPE, 1);
+    ++launches;
+
+    // a3: attention over [cache ; new keys]
+    AttnArgs a;
+    memset(&a, 0, sizeof a);
+    a.B = batch; a.Hq = hq; a.Hkv = hkv; a.dh = dh; a.k = k; a.G = G; a.R = G * k;
+    a.kv_bf16 = c.kv_dtype == SP_BF16;
+    plan_attention(batch, hkv, k, c.max_seq_len, h->opt_split, h->n_sm, &a.split_tokens, &a.n_splits);
+    a.max_seq_len = c.max_seq_len;
+    a.seq_ids = d_seq_ids; a.seq_lens = d_seq_lens; a.lens_by_batch = lens_by_batch;
+    a.kv = to_dev(kv);
+    a.q = h->q; a.k_new = h->k_new; a.v_new = h->v_new;
+    a.status = h->status;
+    a.gathered = nullptr;
+    a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+    a.out = h->o;
+    a.out_bf16 = wb;
+    s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, &launches, st,
+                          h->opt_profile ? h->ev[SP_STAGE_ATTN] : nullptr,
+                          h->opt_profile ? h->ev[SP_STAGE_MERGE] : nullptr);
+    if (s != SP_OK) return s;
+    if (h->opt_profile) h->ev_used[SP_STAGE_ATTN] = h->ev_used[SP_STAGE_MERGE] = true;
+
+    // a4: output projection + residual, post-norm
+    const void *x = d_rows ? d_rows : h->soft_prompt;
+    const int row_mod = d_rows ? 0 : k;
+    mark(SP_STAGE_O_PROJ, 0);
+    s = h->gemm.run(wb, h->opt_gemm, h->o, h->w_o, h->y, M, d, hq * dh, st, &launches);
+    mark(SP_STAGE_O_PROJ, 1);
+    if (s != SP_OK) return s;
+    mark(SP_STAGE_POST_NORM, 0);
+    SP_CUDA(launch_residual_norm(wb, h->y, x, row_mod, h->g_post, c.rms_eps, M, d, h->h1, h->n, st));
+    mark(SP_STAGE_POST_NORM, 1);
+    ++launches;
+    // a5: gate/up + SwiGLU
+    mark(SP_STAGE_GATE_UP, 0);
+    s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, M, 2 * f, d, st, &launches);
+    mark(SP_STAGE_GATE_UP, 1);
+    if (s != SP_OK) return s;
+    mark(SP_STAGE_SWIGLU, 0);
+    SP_CUDA(launch_swiglu(wb, h->y, M, f, h->gu_blk, h->a, st));
+    mark(SP_STAGE_SWIGLU, 1);
+    ++launches;
+    // a6-a7: down projection + residual, pooling, linear head
+    mark(SP_STAGE_DOWN, 0);
+    s = h->gemm.run(wb, h->opt_gemm, h->a, h->w_down, h->y, M, d, f, st, &launches);
+    mark(SP_STAGE_DOWN, 1);
+    if (s != SP_OK) return s;
+    mark(SP_STAGE_READOUT, 0);
+    SP_CUDA(launch_readout(h->y, h->h1, h->head_w, h->head_b, c.pool, batch, k, d, C, d_logits, st));
+    mark(SP_STAGE_READOUT, 1);
+    ++launches;
+    h->last_launches = launches;
+    return SP_OK;
+}
+
+sp_status sp_classify(sp_handle *h, sp_stream stream, int batch, const int *d_seq_ids,
+                      const int *d_seq_lens, const sp_kv_cache *kv, const void *d_rows,
+                      float *d_logits) {
+    return classify_impl(h, (cudaStream_t)stream, batch, d_seq_ids, d_seq_lens, 0, kv, d_rows,
+                         d_logits);
+}
+
+sp_status sp_classify_host(sp_handle *h, sp_stream stream, int batch, const int *h_seq_ids,
+                           const int *h_seq_lens, const sp_kv_cache *kv, const void *h_rows,
+                           float *h_logits) {
+    if (!h) return fail(SP_ERR_INVALID_ARG, "handle is NULL");
+    const sp_config &c = h->cfg;
+    if (batch < 1 || batch > c.max_batch)
+        return fail(SP_ERR_INVALID_ARG, "batch %d outside 1..max_batch (%d)", batch, c.max_batch);
+    if (!h_seq_lens || !h_logits) return fail(SP_ERR_INVALID_ARG, "seq_lens and logits are required");
+    cudaStream_t st = (cudaStream_t)stream;
+    if (h_seq_ids)
+        SP_CUDA(cudaMemcpyAsync(h->stage_ids, h_seq_ids, batch * sizeof(int), cudaMemcpyHostToDevice, st));
+    SP_CUDA(cudaMemcpyAsync(h->stage_lens, h_seq_lens, batch * sizeof(int), cudaMemcpyHostToDevice, st));
+    if (h_rows)
+        SP_CUDA(cudaMemcpyAsync(h->stage_rows, h_rows, (size_t)batch * c.k_rows * c.d_model * h->es,
+                                cudaMemcpyHostToDevice, st));
+    sp_status s = classify_impl(h, st, batch, h_seq_ids ? h->stage_ids : nullptr, h->stage_lens, 1,
+                                kv, h_rows ? h->stage_rows : nullptr, h->stage_logits);
+    if (s != SP_OK) return s;
+    SP_CUDA(cudaMemcpyAsync(h_logits, h->stage_logits, (size_t)batch * c.n_classes * sizeof(float),
+                            cudaMemcpyDeviceToHost, st));
+    int bits = 0;
+    return sp_check_status(h, stream, &bits);
+}
+
+sp_status sp_check_status(sp_handle *h, sp_stream stream, int *bits) {
+    if (!h) return fail(SP_ERR_INVALID_ARG, "handle is NULL");
+    int v = 0;
+    SP_CUDA(cudaStreamSynchronize((cudaStream_t)stream));
+    SP_CUDA(cudaMemcpy(&v, h->status, sizeof(int), cudaMemcpyDeviceToHost));
+    if (bits) *bits = v;
+    if (v) {
+        SP_CUDA(cudaMemset(h->status, 0, sizeof(int)));
+        return fail(SP_ERR_DEVICE_STATUS, "device reported status bits 0x%x%s%s%s", v,
+                    (v & SP_DEV_BAD_SEQ_ID) ? " (sequence id out of range)" : "",
+                    (v & SP_DEV_BAD_LENGTH) ? " (cached length out of range)" : "",
+                    (v & SP_DEV_BAD_PAGE) ? " (page id outside the pool)" : "");
+    }
+    return SP_OK;
+}
+
+size_t sp_attend_workspace_bytes(const sp_attn_dims *dm, int batch) {
+    if (!dm || batch < 1 || dm->n_kv_heads < 1 || dm->n_q_heads % dm->n_kv_heads || dm->k_rows < 1 ||
+        dm->k_rows > 32 || dm->max_seq_len < 0 || (dm->split_tokens % 64) || dm->split_tokens < 0)
+        return 0;
+    int split, ns;
+    plan_attention(batch, dm->n_kv_heads, dm->k_rows, dm->max_seq_len, dm->split_tokens, sm_count(),
+                   &split, &ns);
+    return attention_workspace_bytes(batch, dm->n_kv_heads,
+                                     (dm->n_q_heads / dm->n_kv_heads) * dm->k_rows, dm->head_dim, ns);
+}
+
+sp_status sp_attend(sp_stream stream, const sp_attn_dims *dm, int batch, const int *d_seq_ids,
+                    const int *d_seq_lens, const sp_kv_cache *kv, const float *d_q,
+                    const float *d_k_new, const float *d_v_new, void *d_out, int out_dtype,
+                    void *d_workspace, size_t workspace_bytes, int *d_status,
+                    int *d_gathered_pages) {
+    if (!dm) return fail(SP_ERR_INVALID_ARG, "dims is NULL");
+    if (dm->n_kv_heads < 1 || dm->n_q_heads < 1 || dm->n_q_heads % dm->n_kv_heads)
+        return fail(SP_ERR_INVALID_ARG, "n_q_heads must be a positive multiple of n_kv_heads");
+    if (dm->head_dim != 32 && dm->head_dim != 64 && dm->head_dim != 128)
+        return fail(SP_ERR_UNSUPPORTED, "head_dim %d unsupported", dm->head_dim);
+    if (dm->k_rows < 1 || dm->k_rows > 32) return fail(SP_ERR_INVALID_ARG, "k_rows must be in 1..32");
+    if (dm->kv_dtype != SP_F32 && dm->kv_dtype != SP_BF16) return fail(SP_ERR_INVALID_ARG, "bad kv_dtype");
+    if (out_dtype != SP_F32 && out_dtype != SP_BF16) return fail(SP_ERR_INVALID_ARG, "bad out_dtype");
+    if (dm->split_tokens < 0 || dm->split_tokens % 64)
+        return fail(SP_ERR_INVALID_ARG, "split_tokens must be a multiple of 64");
+    if (batch < 1) return fail(SP_ERR_INVALID_ARG, "batch must be >= 1");
+    if (!d_seq_lens || !d_q || !d_k_new || !d_v_new || !d_out || !d_workspace)
+        return fail(SP_ERR_INVALID_ARG, "a required pointer is NULL");
+    if (((uintptr_t)d_workspace) & 255) return fail(SP_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    sp_status s = check_kv(kv, dm->kv_dtype);
+    if (s != SP_OK) return s;
+    if (!d_seq_ids && batch > kv->n_seqs)
+        return fail(SP_ERR_INVALID_ARG, "batch %d exceeds n_seqs %d with implicit ids", batch, kv->n_seqs);
+    const int G = dm->n_q_heads / dm->n_kv_heads;
+    if (G * dm->k_rows * dm->head_dim > 128 * 128)
+        return fail(SP_ERR_UNSUPPORTED, "query group x k_rows x head_dim too large");
+    AttnArgs a;
+    memset(&a, 0, sizeof a);
+    a.B = batch; a.Hq = dm->n_q_heads; a.Hkv = dm->n_kv_heads; a.dh = dm->head_dim;
+    a.k = dm->k_rows; a.G = G; a.R = G * dm->k_rows;
+    a.kv_bf16 = dm->kv_dtype == SP_BF16;
+    plan_attention(batch, a.Hkv, a.k, dm->max_seq_len, dm->split_tokens, sm_count(), &a.split_tokens,
+                   &a.n_splits);
+    a.max_seq_len = dm->max_seq_len;
+    a.seq_ids = d_seq_ids; a.seq_lens = d_seq_lens; a.lens_by_batch = 0;
+    a.kv = to_dev(kv);
+    a.q = d_q; a.k_new = d_k_new; a.v_new = d_v_new;
+    a.status = d_status;
+    a.gathered = d_gathered_pages;
+    a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)a.dh));
+    a.out = d_out;
+    a.out_bf16 = out_dtype == SP_BF16;
+    int launches = 0;
+    return enqueue_attention(a, d_workspace, workspace_bytes, 0, &launches, (cudaStream_t)stream);
+}
+
+}  // extern "C"

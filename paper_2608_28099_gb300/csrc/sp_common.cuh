@@ -1,0 +1,141 @@
+// Internal declarations shared by the CUDA translation units of libsp.so.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/sp.h"
+
+namespace sp {
+
+typedef __nv_bfloat16 bf16;
+
+__host__ __device__ inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
+__host__ __device__ inline long long ceil_div_ll(long long a, long long b) { return (a + b - 1) / b; }
+
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }
+template <typename T> __device__ __forceinline__ T from_f(float x);
+template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float x) { return __float2bfloat16_rn(x); }
+
+// Cache description as the kernels see it (same fields as sp_kv_cache).
+struct KVDev {
+    int layout;
+    const void *const *k_seq;
+    const void *const *v_seq;
+    const void *k_pool;
+    const void *v_pool;
+    const int *page_table;
+    int page_size;
+    int n_pages;
+    int max_pages;
+    int n_seqs;
+};
+
+// Per-sequence bookkeeping shared by every kernel that reads ids/lengths:
+// out-of-range ids or lengths set a status bit and are clamped so that no
+// access leaves the caller's buffers.
+struct SeqRef {
+    int sid;   // cache sequence id (clamped to a valid id, or -1)
+    int len;   // cached length L_b, clamped to [0, max_seq_len]
+};
+
+// Lengths are indexed by sequence id (lens_by_batch = 0) or by batch entry.
+__device__ __forceinline__ SeqRef resolve_seq(const int *seq_ids, const int *seq_lens,
+                                              int lens_by_batch, int b, int n_seqs,
+                                              int max_seq_len, int *status) {
+    SeqRef r;
+    int sid = seq_ids ? seq_ids[b] : b;
+    if (sid < 0 || sid >= n_seqs) {
+        if (status) atomicOr(status, SP_DEV_BAD_SEQ_ID);
+        r.sid = -1;
+        r.len = 0;
+        return r;
+    }
+    int L = seq_lens[lens_by_batch ? b : sid];
+    if (L < 0 || L > max_seq_len) {
+        if (status) atomicOr(status, SP_DEV_BAD_LENGTH);
+        L = L < 0 ? 0 : max_seq_len;
+    }
+    r.sid = sid;
+    r.len = L;
+    return r;
+}
+
+// ---------------------------------------------------------------------------
+// attention step
+// ---------------------------------------------------------------------------
+struct AttnArgs {
+    int B, Hq, Hkv, dh, k, G, R;  // R = G * k query rows per (sequence, kv head)
+    int kv_bf16;                  // cache element type: 1 bf16, 0 fp32
+    int split_tokens;             // tokens per work unit
+    int n_splits;                 // work units per (sequence, kv head) in the grid
+    int max_seq_len;
+    const int *seq_ids;
+    const int *seq_lens;
+    int lens_by_batch;
+    KVDev kv;
+    const float *q;               // [B][k][Hq][dh], rotated
+    const float *k_new;           // [B][k][Hkv][dh], rotated
+    const float *v_new;           // [B][k][Hkv][dh]
+    float *part_o;                // [B][Hkv][n_splits][R][dh], unnormalised
+    float *part_ml;               // [B][Hkv][n_splits][R][2] (running max in log2 units, sum)
+    int *status;
+    int *gathered;                // [B][max_pages] or NULL
+    float scale_log2;             // log2(e) / sqrt(dh)
+    void *out;                    // merge output [B][k][Hq][dh]
+    int out_bf16;
+};
+
+// Plan: tokens per split-KV work unit and number of units per sequence.
+void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, int n_sm,
+                    int *split_tokens, int *n_splits);
+size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits);
+cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st);
+cudaError_t launch_attention_merge(const AttnArgs &a, cudaStream_t st);
+
+// ---------------------------------------------------------------------------
+// row-wise steps
+// ---------------------------------------------------------------------------
+// out[m] = RMSNorm(x[src(m)]) * gain, src(m) = m or m % row_mod (shared rows)
+cudaError_t launch_rmsnorm_rows(int w_bf16, const void *x, int row_mod, const float *gain, float eps,
+                                int M, int d, void *out, cudaStream_t st);
+
+struct QkvRopeArgs {
+    const float *y;          // projections [rows][(Hq + 2 Hkv) dh]
+    int shared;              // 1: row of m is m % k (shared soft prompt), 0: row m
+    int B, k, Hq, Hkv, dh;
+    const int *seq_ids, *seq_lens;
+    int lens_by_batch;
+    int n_seqs, max_seq_len;
+    const float2 *rope_cs;   // [max_seq_len + k][dh/2] (cos, sin)
+    float *q, *k_new, *v_new;
+    int *status;
+};
+cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st);
+
+// h1 = x + y ; n = RMSNorm(h1) * gain   (x: input rows, w dtype; n: activation dtype)
+cudaError_t launch_residual_norm(int w_bf16, const float *y, const void *x, int row_mod,
+                                 const float *gain, float eps, int M, int d, float *h1, void *n,
+                                 cudaStream_t st);
+
+// a[m][j] = silu(g) * u for gate/up columns laid out in blocks of `blk`
+// (gate block i at columns 2*i*blk.., up block right after it)
+cudaError_t launch_swiglu(int act_bf16, const float *y, int M, int f, int blk, void *a,
+                          cudaStream_t st);
+
+// logits[b] = W_head pool_r(h1 + y) + bias
+cudaError_t launch_readout(const float *y, const float *h1, const float *head_w,
+                           const float *head_b, int pool, int B, int k, int d, int C,
+                           float *logits, cudaStream_t st);
+
+// ---------------------------------------------------------------------------
+// projections
+// ---------------------------------------------------------------------------
+// Y[M][N] (fp32) = X[M][K] * W[N][K]^T on CUDA cores; X and W share w_bf16.
+cudaError_t launch_gemm_simt(int w_bf16, const void *X, const void *W, float *Y, int M, int N,
+                             int K, cudaStream_t st);
+
+}  // namespace sp

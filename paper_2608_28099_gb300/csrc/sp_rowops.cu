@@ -1,0 +1,262 @@
+// Row-wise steps of the decoder layer (Sec. 3.1) and the CUDA-core projection:
+// RMSNorm, rotary embedding of the new queries/keys (positions L_b..L_b+k-1,
+// Sec. 3.3), residual + post-norm, SwiGLU, pooling + linear readout (Sec. 3.2).
+#include "sp_common.cuh"
+
+namespace sp {
+
+namespace {
+
+constexpr int kRowThreads = 256;
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// Block-wide sum for blockDim.x == kRowThreads.
+__device__ __forceinline__ float block_sum(float v, float *red) {
+    v = warp_sum(v);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    __syncthreads();
+    if (l == 0) red[w] = v;
+    __syncthreads();
+    float t = (l < kRowThreads / 32) ? red[l] : 0.f;
+    return warp_sum(t);
+}
+
+template <typename T>
+__global__ void rmsnorm_rows_kernel(const T *__restrict__ x, int row_mod,
+                                    const float *__restrict__ gain, float eps, int d,
+                                    T *__restrict__ out) {
+    __shared__ float red[32];
+    const int m = blockIdx.x;
+    const T *xr = x + (size_t)(row_mod ? m % row_mod : m) * d;
+    float ss = 0.f;
+    for (int j = threadIdx.x; j < d; j += blockDim.x) {
+        float v = to_f(xr[j]);
+        ss += v * v;
+    }
+    ss = block_sum(ss, red);
+    const float inv = rsqrtf(ss / (float)d + eps);
+    T *o = out + (size_t)m * d;
+    for (int j = threadIdx.x; j < d; j += blockDim.x) o[j] = from_f<T>(to_f(xr[j]) * inv * gain[j]);
+}
+
+__global__ void qkv_rope_kernel(QkvRopeArgs a) {
+    const int m = blockIdx.x;
+    const int b = m / a.k, r = m % a.k;
+    SeqRef s = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.n_seqs, a.max_seq_len,
+                           threadIdx.x == 0 ? a.status : nullptr);
+    const int pos = s.len + r;
+    const int dh = a.dh, half = dh >> 1;
+    const int nqkv = (a.Hq + 2 * a.Hkv) * dh;
+    const float *y = a.y + (size_t)(a.shared ? r : m) * nqkv;
+    const float2 *cs = a.rope_cs + (size_t)pos * half;
+    const int nrot = (a.Hq + a.Hkv) * half;  // rotated pairs: all q heads, then k heads
+    for (int idx = threadIdx.x; idx < nrot; idx += blockDim.x) {
+        const int h = idx / half, i = idx - h * half;
+        const float x0 = y[h * dh + i], x1 = y[h * dh + i + half];
+        const float2 c = cs[i];
+        const float r0 = x0 * c.x - x1 * c.y;
+        const float r1 = x1 * c.x + x0 * c.y;
+        float *dst;
+        if (h < a.Hq) {
+            dst = a.q + ((size_t)m * a.Hq + h) * dh;
+        } else {
+            dst = a.k_new + ((size_t)m * a.Hkv + (h - a.Hq)) * dh;
+        }
+        dst[i] = r0;
+        dst[i + half] = r1;
+    }
+    const float *yv = y + (a.Hq + a.Hkv) * dh;
+    float *v = a.v_new + (size_t)m * a.Hkv * dh;
+    for (int j = threadIdx.x; j < a.Hkv * dh; j += blockDim.x) v[j] = yv[j];
+}
+
+template <typename TX, typename TN>
+__global__ void residual_norm_kernel(const float *__restrict__ y, const TX *__restrict__ x,
+                                     int row_mod, const float *__restrict__ gain, float eps, int d,
+                                     float *__restrict__ h1, TN *__restrict__ n) {
+    __shared__ float red[32];
+    const int m = blockIdx.x;
+    const TX *xr = x + (size_t)(row_mod ? m % row_mod : m) * d;
+    const float *yr = y + (size_t)m * d;
+    float *hr = h1 + (size_t)m * d;
+    float ss = 0.f;
+    for (int j = threadIdx.x; j < d; j += blockDim.x) {
+        float v = to_f(xr[j]) + yr[j];
+        hr[j] = v;
+        ss += v * v;
+    }
+    ss = block_sum(ss, red);
+    const float inv = rsqrtf(ss / (float)d + eps);
+    TN *nr = n + (size_t)m * d;
+    for (int j = threadIdx.x; j < d; j += blockDim.x) nr[j] = from_f<TN>(hr[j] * inv * gain[j]);
+}
+
+template <typename TA>
+__global__ void swiglu_kernel(const float *__restrict__ y, int M, int f, int blk,
+                              TA *__restrict__ a) {
+    const long long total = (long long)M * f;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int m = (int)(idx / f), j = (int)(idx - (long long)m * f);
+        const int blkid = j / blk, jj = j - blkid * blk;
+        const float *yr = y + (size_t)m * 2 * f;
+        const float g = yr[2 * blkid * blk + jj];
+        const float u = yr[2 * blkid * blk + blk + jj];
+        const float s = g / (1.f + __expf(-g));
+        a[idx] = from_f<TA>(s * u);
+    }
+}
+
+__global__ void readout_kernel(const float *__restrict__ y, const float *__restrict__ h1,
+                               const float *__restrict__ head_w, const float *__restrict__ head_b,
+                               int pool, int k, int d, int C, float *__restrict__ logits) {
+    extern __shared__ float pooled[];  // [d]
+    __shared__ float red[32];
+    const int b = blockIdx.x;
+    const size_t base = (size_t)b * k * d;
+    const float invk = 1.f / (float)k;
+    for (int j = threadIdx.x; j < d; j += blockDim.x) {
+        float acc;
+        if (pool == SP_POOL_LAST) {
+            const size_t o = base + (size_t)(k - 1) * d + j;
+            acc = h1[o] + y[o];
+        } else {
+            acc = 0.f;
+            for (int r = 0; r < k; ++r) {
+                const size_t o = base + (size_t)r * d + j;
+                acc += h1[o] + y[o];
+            }
+            acc *= invk;
+        }
+        pooled[j] = acc;
+    }
+    __syncthreads();
+    for (int c = 0; c < C; ++c) {
+        float acc = 0.f;
+        const float *wr = head_w + (size_t)c * d;
+        for (int j = threadIdx.x; j < d; j += blockDim.x) acc += wr[j] * pooled[j];
+        acc = block_sum(acc, red);
+        if (threadIdx.x == 0) logits[(size_t)b * C + c] = acc + (head_b ? head_b[c] : 0.f);
+    }
+}
+
+// CUDA-core tiled GEMM: Y[M][N] = X[M][K] W[N][K]^T, fp32 accumulation.
+// 64x64 output tile, 32-deep k slices, 256 threads, 4x4 outputs per thread.
+template <typename T>
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const T *__restrict__ X,
+                                                        const T *__restrict__ W,
+                                                        float *__restrict__ Y, int M, int N,
+                                                        int K) {
+    constexpr int BM = 64, BN = 64, BK = 32;
+    __shared__ float Xs[BK][BM + 4];
+    __shared__ float Ws[BK][BN + 4];
+    const int tid = threadIdx.x;
+    const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+    const int ty = tid >> 4, tx = tid & 15;
+    float acc[4][4] = {};
+    for (int k0 = 0; k0 < K; k0 += BK) {
+        for (int idx = tid; idx < BM * BK; idx += 256) {
+            const int row = idx / BK, kk = idx - row * BK;
+            const int gm = m0 + row, gk = k0 + kk;
+            Xs[kk][row] = (gm < M && gk < K) ? to_f(X[(size_t)gm * K + gk]) : 0.f;
+            const int gn = n0 + row;
+            Ws[kk][row] = (gn < N && gk < K) ? to_f(W[(size_t)gn * K + gk]) : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int kk = 0; kk < BK; ++kk) {
+            float xa[4], wb[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) xa[i] = Xs[kk][ty * 4 + i];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) wb[j] = Ws[kk][tx * 4 + j];
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(xa[i], wb[j], acc[i][j]);
+        }
+        __syncthreads();
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int gm = m0 + ty * 4 + i;
+        if (gm >= M) continue;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int gn = n0 + tx * 4 + j;
+            if (gn < N) Y[(size_t)gm * N + gn] = acc[i][j];
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_rmsnorm_rows(int w_bf16, const void *x, int row_mod, const float *gain,
+                                float eps, int M, int d, void *out, cudaStream_t st) {
+    if (w_bf16)
+        rmsnorm_rows_kernel<bf16><<<M, kRowThreads, 0, st>>>((const bf16 *)x, row_mod, gain, eps, d,
+                                                             (bf16 *)out);
+    else
+        rmsnorm_rows_kernel<float><<<M, kRowThreads, 0, st>>>((const float *)x, row_mod, gain, eps,
+                                                              d, (float *)out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st) {
+    qkv_rope_kernel<<<a.B * a.k, 128, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_residual_norm(int w_bf16, const float *y, const void *x, int row_mod,
+                                 const float *gain, float eps, int M, int d, float *h1, void *n,
+                                 cudaStream_t st) {
+    if (w_bf16)
+        residual_norm_kernel<bf16, bf16><<<M, kRowThreads, 0, st>>>(y, (const bf16 *)x, row_mod,
+                                                                   gain, eps, d, h1, (bf16 *)n);
+    else
+        residual_norm_kernel<float, float><<<M, kRowThreads, 0, st>>>(y, (const float *)x, row_mod,
+                                                                     gain, eps, d, h1, (float *)n);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_swiglu(int act_bf16, const float *y, int M, int f, int blk, void *a,
+                          cudaStream_t st) {
+    const long long total = (long long)M * f;
+    int grid = (int)((total + 255) / 256);
+    if (grid > 152 * 16) grid = 152 * 16;
+    if (act_bf16)
+        swiglu_kernel<bf16><<<grid, 256, 0, st>>>(y, M, f, blk, (bf16 *)a);
+    else
+        swiglu_kernel<float><<<grid, 256, 0, st>>>(y, M, f, blk, (float *)a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_readout(const float *y, const float *h1, const float *head_w,
+                           const float *head_b, int pool, int B, int k, int d, int C,
+                           float *logits, cudaStream_t st) {
+    const size_t smem = (size_t)d * sizeof(float);
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(readout_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    readout_kernel<<<B, kRowThreads, smem, st>>>(y, h1, head_w, head_b, pool, k, d, C, logits);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_simt(int w_bf16, const void *X, const void *W, float *Y, int M, int N,
+                             int K, cudaStream_t st) {
+    dim3 grid(ceil_div(N, 64), ceil_div(M, 64));
+    if (w_bf16)
+        gemm_simt_kernel<bf16><<<grid, 256, 0, st>>>((const bf16 *)X, (const bf16 *)W, Y, M, N, K);
+    else
+        gemm_simt_kernel<float><<<grid, 256, 0, st>>>((const float *)X, (const float *)W, Y, M, N, K);
+    return cudaGetLastError();
+}
+
+}  // namespace sp

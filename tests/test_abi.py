@@ -1,0 +1,90 @@
+"""The C-ABI library builds, loads without a GPU, exports every symbol that
+include/sp.h declares, and rejects bad arguments on the host before touching
+the device."""
+import ctypes as C
+import os
+import re
+
+import numpy as np
+import pytest
+
+import paper_2608_28099_gb300 as sp
+from paper_2608_28099_gb300 import build_lib
+from paper_2608_28099_gb300 import workloads as wl
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_symbols():
+    names = []
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        if h.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", h)).read()
+            names += re.findall(r"^SP_API\s+[\w\s\*]*?\b(sp_\w+)\s*\(", text, flags=re.M)
+    return sorted(set(names))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build_lib.build()
+    return sp.load_library()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_symbols()
+    assert len(names) >= 10
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(sp.EXPORTED) <= set(names)
+
+
+def _cfg(**over):
+    shape = wl.named("tiny").shape
+    c = sp.make_config(shape, 4, 128)
+    for k, v in over.items():
+        setattr(c, k, v)
+    return c
+
+
+@pytest.mark.parametrize("field,value,status", [
+    ("head_dim", 96, sp.SP_ERR_UNSUPPORTED),
+    ("n_q_heads", 3, sp.SP_ERR_INVALID_ARG),
+    ("k_rows", 0, sp.SP_ERR_INVALID_ARG),
+    ("k_rows", 33, sp.SP_ERR_INVALID_ARG),
+    ("d_model", 100, sp.SP_ERR_INVALID_ARG),
+    ("max_batch", 0, sp.SP_ERR_INVALID_ARG),
+    ("pool", 7, sp.SP_ERR_INVALID_ARG),
+    ("kv_dtype", 5, sp.SP_ERR_INVALID_ARG),
+])
+def test_create_rejects_bad_config_on_host(lib, field, value, status):
+    h = C.c_void_p(123)
+    w = sp.sp_weights()
+    st = lib.sp_create(C.byref(_cfg(**{field: value})), C.byref(w), C.byref(h))
+    assert st == status
+    assert h.value is None
+    assert lib.sp_last_error()
+
+
+def test_create_rejects_missing_weights_on_host(lib):
+    h = C.c_void_p()
+    w = sp.sp_weights()
+    assert lib.sp_create(C.byref(_cfg()), C.byref(w), C.byref(h)) == sp.SP_ERR_INVALID_ARG
+    assert b"weight" in lib.sp_last_error()
+
+
+def test_null_handle_calls_fail_cleanly(lib):
+    kv = sp.sp_kv_cache()
+    assert lib.sp_classify(None, None, 1, None, None, C.byref(kv), None, None) == sp.SP_ERR_INVALID_ARG
+    assert lib.sp_set_option(None, 1, 0) == sp.SP_ERR_INVALID_ARG
+    assert lib.sp_destroy(None) == sp.SP_OK
+    assert lib.sp_last_launch_count(None) == -1
+
+
+def test_attend_rejects_bad_dims_on_host(lib):
+    kv = sp.sp_kv_cache()
+    dims = sp.sp_attn_dims(4, 3, 32, 4, sp.SP_F32, 64, 0)    # 4 q heads over 3 kv heads
+    st = lib.sp_attend(None, C.byref(dims), 1, None, None, C.byref(kv), None, None, None, None, 0,
+                       None, 0, None, None)
+    assert st == sp.SP_ERR_INVALID_ARG
+    dims = sp.sp_attn_dims(4, 2, 32, 4, sp.SP_F32, 64, 100)   # split not a multiple of 64
+    assert lib.sp_attend_workspace_bytes(C.byref(dims), 1) == 0

@@ -1,0 +1,249 @@
+"""CUDA path vs the fp64 oracle on seeded inputs (all named workloads, edge
+cases) and invariants of the GPU path.  Every call goes through the C ABI."""
+import hashlib
+
+import numpy as np
+import pytest
+
+import oracle.sp_oracle as so
+import paper_2608_28099_gb300 as sp
+from paper_2608_28099_gb300 import workloads as wl
+from gpu_util import ATOL, RTOL, GpuRun, compare, ensure_built, oracle_logits, torch_dev
+
+pytestmark = pytest.mark.gpu
+
+
+# --------------------------------------------------------------------------- #
+# named workloads
+# --------------------------------------------------------------------------- #
+def test_tiny_fp32_matches_oracle_tightly():
+    w = wl.generate(wl.named("tiny"))
+    run = GpuRun(w)
+    gpu = run.logits()
+    ref = oracle_logits(w)
+    # fp32 weights and cache: a much tighter bound than the bf16 one
+    scale = float(np.max(np.abs(ref)))
+    assert np.max(np.abs(gpu - ref)) <= 1e-5 * scale + 1e-7, (gpu, ref)
+    compare(gpu, ref, label="tiny")
+    run.close()
+
+
+@pytest.mark.parametrize("name", ["4b", "8b_paged", "27b_long"])
+def test_named_workload_matches_oracle(name):
+    w = wl.generate(wl.named(name, rows_per_seq=True))
+    run = GpuRun(w)
+    for use_rows in (True, False):
+        gpu = run.logits(use_rows=use_rows)
+        ref = oracle_logits(w, use_rows=use_rows)
+        assert np.all(np.isfinite(gpu))
+        # logits are O(0.1-1) here, so the bound is not vacuous
+        assert np.max(np.abs(ref)) > 0.05
+        compare(gpu, ref, label=f"{name} rows={use_rows}")
+    run.close()
+
+
+SWEEP_SAMPLE = ["sweep_B1_L512_k1_C2", "sweep_B8_L2048_k4_C16", "sweep_B32_L8192_k16_C2",
+                "sweep_B8_L16384_k32_C16", "sweep_B128_L512_k32_C2", "sweep_B256_L512_k1_C16"]
+
+
+@pytest.mark.parametrize("name", SWEEP_SAMPLE)
+def test_sweep_point_matches_oracle_on_a_subset(name):
+    w = wl.generate(wl.named(name))
+    run = GpuRun(w)
+    gpu = run.logits()
+    sub = np.random.default_rng(0).choice(len(w.seq_ids), size=min(8, len(w.seq_ids)),
+                                          replace=False)
+    ref = oracle_logits(w, ids=np.sort(sub))
+    compare(gpu[np.sort(sub)], ref, label=name)
+    run.close()
+
+
+# --------------------------------------------------------------------------- #
+# edge cases on small shapes (several tiles, ragged tails)
+# --------------------------------------------------------------------------- #
+SMALL_BF16 = wl.Shape(256, 8, 2, 128, 512, 4, 3)
+EDGE_LENS = [0, 1, 15, 16, 17, 63, 64, 65, 127, 300]
+
+
+@pytest.mark.parametrize("layout", [wl.LAYOUT_CONTIGUOUS, wl.LAYOUT_PAGED])
+@pytest.mark.parametrize("rows", [False, True])
+def test_edge_lengths(layout, rows):
+    w = wl.custom(SMALL_BF16, EDGE_LENS, layout, 31, rows_per_seq=rows, head_bias=True)
+    run = GpuRun(w)
+    compare(run.logits(), oracle_logits(w), label="edge")
+    run.close()
+
+
+@pytest.mark.parametrize("shape", [
+    wl.Shape(128, 4, 4, 64, 256, 1, 2),            # MHA (G=1), k=1
+    wl.Shape(256, 8, 1, 32, 256, 32, 5),           # MQA, k=32, head_dim 32
+    wl.Shape(512, 8, 2, 128, 1024, 7, 2, pool=wl.POOL_LAST),
+    wl.Shape(384, 12, 4, 64, 768, 5, 16, w_dtype=wl.F32, kv_dtype=wl.F32),
+])
+def test_shape_variants(shape):
+    w = wl.custom(shape, [5, 40, 129, 257], wl.LAYOUT_PAGED, 41, rows_per_seq=True)
+    run = GpuRun(w)
+    gpu = run.logits()
+    ref = oracle_logits(w)
+    if shape.w_dtype == wl.F32:
+        assert np.max(np.abs(gpu - ref)) <= 1e-4 * max(1.0, np.max(np.abs(ref)))
+    compare(gpu, ref, label=str(shape))
+    run.close()
+
+
+def test_sequence_ids_select_and_permute():
+    w = wl.custom(SMALL_BF16, [10, 200, 33, 0, 90, 64], wl.LAYOUT_PAGED, 51)
+    run = GpuRun(w, max_batch=6)
+    ids = [4, 1, 1, 5]
+    compare(run.logits(ids=ids, use_rows=False), oracle_logits(w, use_rows=False, ids=ids))
+    run.close()
+
+
+# --------------------------------------------------------------------------- #
+# invariants
+# --------------------------------------------------------------------------- #
+def _sha(t):
+    return hashlib.sha256(t.cpu().numpy().tobytes()).hexdigest()
+
+
+def test_cache_is_never_written():
+    w = wl.custom(SMALL_BF16, [100, 257], wl.LAYOUT_PAGED, 61, rows_per_seq=True)
+    run = GpuRun(w)
+    before = (_sha(run.cache.k_pool), _sha(run.cache.v_pool), _sha(run.cache.page_table))
+    run.logits()
+    run.logits(use_rows=False)
+    assert before == (_sha(run.cache.k_pool), _sha(run.cache.v_pool), _sha(run.cache.page_table))
+    run.close()
+
+
+def test_layouts_and_page_permutation_agree_bitwise():
+    base = wl.custom(SMALL_BF16, [70, 300, 1, 128], wl.LAYOUT_CONTIGUOUS, 71, rows_per_seq=True)
+    outs = []
+    for cache in (base.cache, wl.contiguous_to_paged(base.cache, 16, 1),
+                  wl.contiguous_to_paged(base.cache, 16, 2)):
+        w = wl.Workload(base.spec, base.weights, cache, base.seq_ids, base.rows)
+        run = GpuRun(w, options={sp.SP_OPT_SPLIT_TOKENS: 128})
+        outs.append(run.logits())
+        run.close()
+    assert np.array_equal(outs[0], outs[1]) and np.array_equal(outs[1], outs[2])
+
+
+def test_split_plan_does_not_change_results():
+    w = wl.custom(SMALL_BF16, [1000, 2000, 37], wl.LAYOUT_PAGED, 81)
+    res = []
+    for split in (64, 256, 2048 + 64):
+        run = GpuRun(w, options={sp.SP_OPT_SPLIT_TOKENS: split})
+        res.append(run.logits())
+        run.close()
+    for r in res[1:]:
+        np.testing.assert_allclose(r, res[0], rtol=1e-5, atol=1e-6)
+    compare(res[0], oracle_logits(w))
+
+
+def test_repeated_calls_are_bitwise_deterministic():
+    w = wl.custom(SMALL_BF16, [500, 12, 1200], wl.LAYOUT_PAGED, 91, rows_per_seq=True)
+    run = GpuRun(w)
+    a, b = run.logits(), run.logits()
+    assert np.array_equal(a, b)
+    run.close()
+
+
+def test_result_does_not_depend_on_batch_company():
+    w = wl.custom(SMALL_BF16, [40, 700, 129, 5], wl.LAYOUT_PAGED, 101)
+    run = GpuRun(w, max_batch=4)
+    full = run.logits(use_rows=False)
+    for i in range(4):
+        one = run.logits(use_rows=False, ids=[i])
+        np.testing.assert_allclose(one[0], full[i], rtol=1e-4, atol=1e-5)
+    run.close()
+
+
+def test_shared_prompt_equals_rows_holding_the_prompt():
+    w = wl.custom(SMALL_BF16, [33, 90], wl.LAYOUT_PAGED, 111)
+    w.rows = np.stack([w.weights.soft_prompt] * 2)
+    run = GpuRun(w)
+    np.testing.assert_allclose(run.logits(use_rows=True), run.logits(use_rows=False),
+                               rtol=1e-4, atol=1e-5)
+    run.close()
+
+
+def test_host_entry_point_matches_device_entry_point():
+    torch = torch_dev()
+    w = wl.custom(SMALL_BF16, [50, 260, 3], wl.LAYOUT_PAGED, 121, rows_per_seq=True)
+    run = GpuRun(w)
+    dev = run.logits()
+    out = np.zeros((3, SMALL_BF16.n_classes), dtype=np.float32)
+    lens = np.ascontiguousarray(w.cache.seq_lens[w.seq_ids], dtype=np.int32)
+    ids = np.ascontiguousarray(w.seq_ids, dtype=np.int32)
+    sp.sp_classify_host(run.model.handle, torch.cuda.current_stream(), 3, ids, lens,
+                        run.cache.desc, np.ascontiguousarray(w.rows), out)
+    assert np.array_equal(out.astype(np.float64), dev)
+    run.close()
+
+
+# --------------------------------------------------------------------------- #
+# the attention step alone and its page gather
+# --------------------------------------------------------------------------- #
+@pytest.mark.parametrize("kv_dtype", [wl.F32, wl.BF16])
+def test_attention_step_and_gathered_pages(kv_dtype):
+    torch = torch_dev()
+    ensure_built()
+    shape = wl.Shape(256, 8, 2, 64, 256, 5, 2, kv_dtype=kv_dtype)
+    lens = [0, 16, 17, 250, 1000]
+    w = wl.custom(shape, lens, wl.LAYOUT_PAGED, 131)
+    rng = np.random.default_rng(7)
+    B, k = len(lens), shape.k_rows
+    q = rng.standard_normal((B, k, shape.n_q_heads, shape.head_dim)).astype(np.float32)
+    kn = rng.standard_normal((B, k, shape.n_kv_heads, shape.head_dim)).astype(np.float32)
+    vn = rng.standard_normal((B, k, shape.n_kv_heads, shape.head_dim)).astype(np.float32)
+    ref = so.attention_step(shape, w.cache, w.seq_ids, q.astype(np.float64), kn.astype(np.float64),
+                            vn.astype(np.float64))
+    cache = sp.DeviceCache(w.cache)
+    dims = sp.sp_attn_dims(shape.n_q_heads, shape.n_kv_heads, shape.head_dim, k, kv_dtype,
+                           max(lens), 128)
+    ws_bytes = sp.sp_attend_workspace_bytes(dims, B)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    out = torch.empty(q.shape, dtype=torch.float32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    gathered = torch.full((B, w.cache.max_pages), -7, dtype=torch.int32, device="cuda")
+    sp.sp_attend(torch.cuda.current_stream(), dims, B, None, cache.seq_lens, cache.desc,
+                 torch.from_numpy(q).cuda(), torch.from_numpy(kn).cuda(), torch.from_numpy(vn).cuda(),
+                 out, sp.SP_F32, ws, ws_bytes, status, gathered)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    tol = 1e-5 if kv_dtype == wl.F32 else 1e-5
+    np.testing.assert_allclose(out.cpu().numpy(), ref, rtol=tol * 10, atol=tol * 10)
+    g = gathered.cpu().numpy()
+    for b, L in enumerate(lens):
+        npg = (L + 15) // 16
+        assert np.array_equal(g[b, :npg], w.cache.page_table[b, :npg])  # bit-exact ids
+        assert np.all(g[b, npg:] == -7)                                 # nothing else read
+
+
+# --------------------------------------------------------------------------- #
+# device-side status (bad ids, lengths, pages never fault; they are reported)
+# --------------------------------------------------------------------------- #
+def test_device_status_reports_bad_inputs():
+    torch = torch_dev()
+    w = wl.custom(SMALL_BF16, [20, 40], wl.LAYOUT_PAGED, 141)
+    run = GpuRun(w, max_batch=2, max_seq_len=64)
+    h = run.model.handle
+    out = torch.empty((2, SMALL_BF16.n_classes), dtype=torch.float32, device="cuda")
+    st = torch.cuda.current_stream()
+    bad_ids = torch.tensor([0, 9], dtype=torch.int32, device="cuda")
+    sp.sp_classify(h, st, 2, bad_ids, run.cache.seq_lens, run.cache.desc, None, out)
+    assert sp.sp_check_status(h) & sp.SP_DEV_BAD_SEQ_ID
+    bad_lens = torch.tensor([20, 65], dtype=torch.int32, device="cuda")
+    sp.sp_classify(h, st, 2, None, bad_lens, run.cache.desc, None, out)
+    assert sp.sp_check_status(h) & sp.SP_DEV_BAD_LENGTH
+    pt = run.cache.page_table.clone()
+    pt[1, 1] = 10_000
+    desc = sp.sp_kv_cache(sp.SP_KV_PAGED, None, None, run.cache.k_pool.data_ptr(),
+                          run.cache.v_pool.data_ptr(), pt.data_ptr(), 16, w.cache.n_pages,
+                          w.cache.max_pages, 2)
+    sp.sp_classify(h, st, 2, None, run.cache.seq_lens, desc, None, out)
+    assert sp.sp_check_status(h) & sp.SP_DEV_BAD_PAGE
+    # the context is still usable and a clean call reports nothing
+    good = run.logits(use_rows=False)
+    compare(good, oracle_logits(w, use_rows=False))
+    run.close()
