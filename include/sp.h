@@ -71,7 +71,9 @@ enum { SP_KV_CONTIGUOUS = 0, SP_KV_PAGED = 1 };/* cache addressing              
 enum {
     SP_DEV_BAD_SEQ_ID = 1,    /* a sequence id was outside [0, n_seqs)               */
     SP_DEV_BAD_LENGTH = 2,    /* a cached length was < 0 or > max_seq_len            */
-    SP_DEV_BAD_PAGE = 4       /* a page-table entry was outside [0, n_pages)         */
+    SP_DEV_BAD_PAGE = 4,      /* a page-table entry was outside [0, n_pages)         */
+    SP_DEV_TIMEOUT = 8        /* a tensor-core kernel gave up waiting on a copy or an
+                                 MMA (its outputs are invalid; the context is intact) */
 };
 
 /* Shapes of the frozen layer and of the probe (Sec. 3.1, 3.2). */
@@ -250,6 +252,22 @@ SP_API sp_status sp_attend(sp_stream stream, const sp_attn_dims *dims, int batch
                     const float *d_k_new, const float *d_v_new, void *d_out, int out_dtype,
                     void *d_workspace, size_t workspace_bytes, int *d_status,
                     int *d_gathered_pages);
+
+/* ------------------------------------------------------------------------- */
+/* The projection step alone: one of the decoder layer's linear maps (Sec. 3.1)*/
+/* ------------------------------------------------------------------------- */
+/* Bytes of device scratch sp_project needs for an M x N x K product. */
+SP_API size_t sp_project_workspace_bytes(int M, int N, int K);
+
+/* Y[M][N] = X[M][K] W[N][K]^T with X and Y fp32 row-major and W bf16 row-major
+ * [N][K] (raw 16-bit patterns), all DEVICE pointers (X, W 16-byte aligned).
+ * path: 1 = CUDA cores, 2 = tensor cores (needs N % 128 == 0 and K % 64 == 0;
+ * SP_ERR_UNSUPPORTED otherwise), 0 = tensor cores when supported.  The tensor
+ * path splits X into bf16 hi + lo parts and may split K across CTAs; both live
+ * in d_workspace (>= sp_project_workspace_bytes, 256-byte aligned). */
+SP_API sp_status sp_project(sp_stream stream, int M, int N, int K, const float *d_x,
+                            const void *d_w, float *d_y, int path, void *d_workspace,
+                            size_t workspace_bytes);
 
 #ifdef __cplusplus
 }

@@ -25,7 +25,7 @@ STAGES = ["input_norm", "qkv", "rope", "attention", "merge", "o_proj", "post_nor
 
 EXPORTED = ["sp_create", "sp_destroy", "sp_classify", "sp_classify_host", "sp_check_status",
             "sp_last_error", "sp_set_option", "sp_last_launch_count", "sp_attend_workspace_bytes",
-            "sp_attend", "sp_stage_times"]
+            "sp_attend", "sp_stage_times", "sp_project_workspace_bytes", "sp_project"]
 
 
 class sp_config(C.Structure):
@@ -87,10 +87,14 @@ def load_library(path: str | None = None):
     lib.sp_attend_workspace_bytes.argtypes = [C.POINTER(sp_attn_dims), i]
     lib.sp_attend_workspace_bytes.restype = C.c_size_t
     lib.sp_stage_times.argtypes = [vp, C.POINTER(C.c_float), i]
+    lib.sp_project_workspace_bytes.argtypes = [i, i, i]
+    lib.sp_project_workspace_bytes.restype = C.c_size_t
+    lib.sp_project.argtypes = [vp, i, i, i, vp, vp, vp, i, vp, C.c_size_t]
     lib.sp_attend.argtypes = [vp, C.POINTER(sp_attn_dims), i, vp, vp, C.POINTER(sp_kv_cache), vp,
                               vp, vp, vp, i, vp, C.c_size_t, vp, vp]
     for name in EXPORTED:
-        if name not in ("sp_last_error", "sp_last_launch_count", "sp_attend_workspace_bytes"):
+        if name not in ("sp_last_error", "sp_last_launch_count", "sp_attend_workspace_bytes",
+                        "sp_project_workspace_bytes"):
             getattr(lib, name).restype = C.c_int
     if path is None:
         _lib = lib
@@ -167,6 +171,15 @@ def sp_stage_times(handle) -> dict:
     ms = (C.c_float * len(STAGES))()
     _check(load_library().sp_stage_times(handle, ms, len(STAGES)))
     return {name: float(ms[i]) for i, name in enumerate(STAGES) if ms[i] >= 0}
+
+
+def sp_project_workspace_bytes(M, N, K) -> int:
+    return load_library().sp_project_workspace_bytes(int(M), int(N), int(K))
+
+
+def sp_project(stream, M, N, K, x, w, y, path, workspace, workspace_bytes):
+    _check(load_library().sp_project(_stream(stream), int(M), int(N), int(K), _ptr(x), _ptr(w),
+                                     _ptr(y), int(path), _ptr(workspace), int(workspace_bytes)))
 
 
 def sp_last_error() -> str:

@@ -53,26 +53,24 @@ struct Arena {
 struct sp_handle {
     sp_config cfg;
     int device = 0, n_sm = 148;
-    int es = 2;        // bytes per weight/activation element
+    int es = 2;        // bytes per stored weight element
     int nqkv = 0;      // (Hq + 2 Hkv) dh
     int gu_blk = 0;    // gate/up interleave block (columns)
     // weights
-    void *w_qkv = nullptr, *w_o = nullptr, *w_gu = nullptr, *w_down = nullptr;
+    WeightMat w_qkv, w_o, w_gu, w_down;
     float *g_in = nullptr, *g_post = nullptr, *head_w = nullptr, *head_b = nullptr;
     void *soft_prompt = nullptr;
     float *qkv_shared = nullptr;  // [k][nqkv] projections of the shared soft prompt
     float2 *rope_cs = nullptr;    // [max_seq_len + k][dh/2]
     // scratch
     Arena arena;
-    void *xn = nullptr;           // [M][d] activation dtype
-    float *y = nullptr;           // [M][max N] projection output
+    ActBuf xn, o, n, a;           // inputs of the four projections
+    float *y = nullptr;           // projection partials [splits][M][N]
+    size_t y_bytes = 0;
     float *q = nullptr, *k_new = nullptr, *v_new = nullptr;
     void *attn_ws = nullptr;
     size_t attn_ws_bytes = 0;
-    void *o = nullptr;            // [M][Hq dh]
     float *h1 = nullptr;          // [M][d]
-    void *n = nullptr;            // [M][d]
-    void *a = nullptr;            // [M][d_ff]
     int *status = nullptr;
     int *stage_ids = nullptr, *stage_lens = nullptr;
     void *stage_rows = nullptr;
@@ -235,21 +233,27 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     };
 
     // weights: [W_q; W_k; W_v] and [W_gate; W_up] concatenated along the output dim
+    void *p_qkv = nullptr, *p_gu = nullptr, *p_o = nullptr, *p_down = nullptr;
     {
         std::vector<char> buf((size_t)h->nqkv * d * es);
         memcpy(buf.data(), w->w_q, (size_t)hq * dh * d * es);
         memcpy(buf.data() + (size_t)hq * dh * d * es, w->w_k, (size_t)hkv * dh * d * es);
         memcpy(buf.data() + (size_t)(hq + hkv) * dh * d * es, w->w_v, (size_t)hkv * dh * d * es);
-        if ((st = upload(h, &h->w_qkv, buf.data(), buf.size())) != SP_OK) return cleanup(st);
+        if ((st = upload(h, &p_qkv, buf.data(), buf.size())) != SP_OK) return cleanup(st);
     }
     {
         std::vector<char> buf((size_t)2 * f * d * es);
         memcpy(buf.data(), w->w_gate, (size_t)f * d * es);
         memcpy(buf.data() + (size_t)f * d * es, w->w_up, (size_t)f * d * es);
-        if ((st = upload(h, &h->w_gu, buf.data(), buf.size())) != SP_OK) return cleanup(st);
+        if ((st = upload(h, &p_gu, buf.data(), buf.size())) != SP_OK) return cleanup(st);
     }
-    if ((st = upload(h, &h->w_o, w->w_o, (size_t)d * hq * dh * es)) != SP_OK) return cleanup(st);
-    if ((st = upload(h, &h->w_down, w->w_down, (size_t)d * f * es)) != SP_OK) return cleanup(st);
+    if ((st = upload(h, &p_o, w->w_o, (size_t)d * hq * dh * es)) != SP_OK) return cleanup(st);
+    if ((st = upload(h, &p_down, w->w_down, (size_t)d * f * es)) != SP_OK) return cleanup(st);
+    const int wb = c.w_dtype == SP_BF16;
+    init_weight(h->w_qkv, p_qkv, h->nqkv, d, wb);
+    init_weight(h->w_o, p_o, d, hq * dh, wb);
+    init_weight(h->w_gu, p_gu, 2 * f, d, wb);
+    init_weight(h->w_down, p_down, d, f, wb);
     if ((st = upload(h, (void **)&h->g_in, w->g_in, d * sizeof(float))) != SP_OK) return cleanup(st);
     if ((st = upload(h, (void **)&h->g_post, w->g_post, d * sizeof(float))) != SP_OK) return cleanup(st);
     if ((st = upload(h, &h->soft_prompt, w->soft_prompt, (size_t)k * d * es)) != SP_OK) return cleanup(st);
@@ -280,54 +284,63 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     if ((size_t)d > maxN) maxN = d;
     if ((size_t)2 * f > maxN) maxN = 2 * (size_t)f;
     h->attn_ws_bytes = max_attention_ws(c, h->n_sm, 0);
-    h->gemm.init(h->n_sm);
-    const size_t gemm_ws = h->gemm.workspace_bytes(M, maxN);
+    // projection partials: room for up to 4 splits of the widest output, and
+    // for as many splits as one wave of CTAs can use on the narrow outputs
+    h->y_bytes = M * maxN * 4 * 4;
+    const size_t narrow = (size_t)h->n_sm * (M < 128 ? 128 : M) * 128 * 4;
+    if (narrow > h->y_bytes) h->y_bytes = narrow;
+    h->gemm.init(h->n_sm, h->y_bytes);
     size_t total = 0;
-    const size_t sizes[] = {M * d * es,                 // xn
-                            M * maxN * 4 + gemm_ws,     // y (+ split-K partials)
+    const size_t sizes[] = {M * d * 4,                  // xn (fp32, or bf16 hi+lo)
+                            h->y_bytes,                 // y partials
                             M * hq * dh * 4,            // q
                             M * hkv * dh * 4,           // k_new
                             M * hkv * dh * 4,           // v_new
                             h->attn_ws_bytes,           // attention partials
-                            M * hq * dh * es,           // o
+                            M * hq * dh * 4,            // o
                             M * d * 4,                  // h1
-                            M * d * es,                 // n
-                            M * f * es,                 // a
+                            M * d * 4,                  // n
+                            M * f * 4,                  // a
                             256,                        // status
                             (size_t)c.max_batch * 4,    // stage ids
                             (size_t)c.max_batch * 4,    // stage lens
                             M * d * es,                 // stage rows
                             (size_t)c.max_batch * C * 4,  // stage logits
                             (size_t)k * h->nqkv * 4};   // qkv_shared
-    for (size_t s : sizes) total += align256(s);
+    for (size_t sz : sizes) total += align256(sz);
     void *arena = nullptr;
     if ((st = dev_alloc(h, &arena, total)) != SP_OK) return cleanup(st);
     h->arena.base = (char *)arena;
     h->arena.cap = total;
-    h->xn = h->arena.take(sizes[0]);
+    void *p_xn = h->arena.take(sizes[0]);
     h->y = (float *)h->arena.take(sizes[1]);
     h->q = (float *)h->arena.take(sizes[2]);
     h->k_new = (float *)h->arena.take(sizes[3]);
     h->v_new = (float *)h->arena.take(sizes[4]);
     h->attn_ws = h->arena.take(sizes[5]);
-    h->o = h->arena.take(sizes[6]);
+    void *p_o_act = h->arena.take(sizes[6]);
     h->h1 = (float *)h->arena.take(sizes[7]);
-    h->n = h->arena.take(sizes[8]);
-    h->a = h->arena.take(sizes[9]);
+    void *p_n = h->arena.take(sizes[8]);
+    void *p_a = h->arena.take(sizes[9]);
     h->status = (int *)h->arena.take(sizes[10]);
     h->stage_ids = (int *)h->arena.take(sizes[11]);
     h->stage_lens = (int *)h->arena.take(sizes[12]);
     h->stage_rows = h->arena.take(sizes[13]);
     h->stage_logits = (float *)h->arena.take(sizes[14]);
     h->qkv_shared = (float *)h->arena.take(sizes[15]);
+    init_act(h->xn, p_xn, (int)M, d, h->w_qkv.tc);
+    init_act(h->o, p_o_act, (int)M, hq * dh, h->w_o.tc);
+    init_act(h->n, p_n, (int)M, d, h->w_gu.tc);
+    init_act(h->a, p_a, (int)M, f, h->w_down.tc);
     if (cudaMemset(h->status, 0, 256) != cudaSuccess) return cleanup(fail(SP_ERR_CUDA, "memset failed"));
 
-    // projections of the shared soft prompt rows (they do not depend on the sequence)
+    // projections of the shared soft prompt rows (they do not depend on the
+    // sequence), on CUDA cores with fp32 activations
     {
-        const int wb = c.w_dtype == SP_BF16;
-        cudaError_t e = launch_rmsnorm_rows(wb, h->soft_prompt, 0, h->g_in, c.rms_eps, k, d, h->xn, 0);
+        cudaError_t e = launch_rmsnorm_rows(wb, h->soft_prompt, 0, h->g_in, c.rms_eps, k, d,
+                                            h->xn.out(false), 0);
         if (e == cudaSuccess)
-            e = launch_gemm_simt(wb, h->xn, h->w_qkv, h->qkv_shared, k, h->nqkv, d, 0);
+            e = launch_gemm_simt(wb, h->xn.ptr, h->w_qkv.ptr, h->qkv_shared, k, h->nqkv, d, 0);
         if (e == cudaSuccess) e = cudaDeviceSynchronize();
         if (e != cudaSuccess)
             return cleanup(fail(SP_ERR_CUDA, "shared prompt projection failed: %s", cudaGetErrorString(e)));
@@ -418,18 +431,25 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         h->ev_used[stage] = true;
     };
 
+    const size_t stride_qkv = (size_t)M * h->nqkv;
+    const bool tc_qkv = h->gemm.use_tc(h->w_qkv, h->xn, h->opt_gemm);
+    const bool tc_o = h->gemm.use_tc(h->w_o, h->o, h->opt_gemm);
+    const bool tc_gu = h->gemm.use_tc(h->w_gu, h->n, h->opt_gemm);
+    const bool tc_down = h->gemm.use_tc(h->w_down, h->a, h->opt_gemm);
+    int ns = 1;
+
     // a1-a2: pre-norm, Q/K/V projection, rotation at positions L_b + r
-    const float *yqkv = h->qkv_shared;
+    PartIn yqkv = {h->qkv_shared, 1, 0};
     if (d_rows) {
         mark(SP_STAGE_INPUT_NORM, 0);
-        SP_CUDA(launch_rmsnorm_rows(wb, d_rows, 0, h->g_in, c.rms_eps, M, d, h->xn, st));
+        SP_CUDA(launch_rmsnorm_rows(wb, d_rows, 0, h->g_in, c.rms_eps, M, d, h->xn.out(tc_qkv), st));
         mark(SP_STAGE_INPUT_NORM, 1);
         ++launches;
         mark(SP_STAGE_QKV, 0);
-        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->nqkv, d, st, &launches);
+        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns);
         mark(SP_STAGE_QKV, 1);
-        if (s != SP_OK) return s;
-        yqkv = h->y;
+        if (s != SP_OK) return fail(s, "Q/K/V projection launch failed");
+        yqkv = PartIn{h->y, ns, stride_qkv};
     }
     QkvRopeArgs r;
     r.y = yqkv;
@@ -458,8 +478,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     a.status = h->status;
     a.gathered = nullptr;
     a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
-    a.out = h->o;
-    a.out_bf16 = wb;
+    a.out = h->o.out(tc_o);
     s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, &launches, st,
                           h->opt_profile ? h->ev[SP_STAGE_ATTN] : nullptr,
                           h->opt_profile ? h->ev[SP_STAGE_MERGE] : nullptr);
@@ -470,29 +489,31 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     const void *x = d_rows ? d_rows : h->soft_prompt;
     const int row_mod = d_rows ? 0 : k;
     mark(SP_STAGE_O_PROJ, 0);
-    s = h->gemm.run(wb, h->opt_gemm, h->o, h->w_o, h->y, M, d, hq * dh, st, &launches);
+    s = h->gemm.run(wb, h->opt_gemm, h->o, h->w_o, h->y, M, h->status, st, &launches, &ns);
     mark(SP_STAGE_O_PROJ, 1);
-    if (s != SP_OK) return s;
+    if (s != SP_OK) return fail(s, "output projection launch failed");
     mark(SP_STAGE_POST_NORM, 0);
-    SP_CUDA(launch_residual_norm(wb, h->y, x, row_mod, h->g_post, c.rms_eps, M, d, h->h1, h->n, st));
+    SP_CUDA(launch_residual_norm(wb, PartIn{h->y, ns, (size_t)M * d}, x, row_mod, h->g_post,
+                                 c.rms_eps, M, d, h->h1, h->n.out(tc_gu), st));
     mark(SP_STAGE_POST_NORM, 1);
     ++launches;
     // a5: gate/up + SwiGLU
     mark(SP_STAGE_GATE_UP, 0);
-    s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, M, 2 * f, d, st, &launches);
+    s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, M, h->status, st, &launches, &ns);
     mark(SP_STAGE_GATE_UP, 1);
-    if (s != SP_OK) return s;
+    if (s != SP_OK) return fail(s, "gate/up projection launch failed");
     mark(SP_STAGE_SWIGLU, 0);
-    SP_CUDA(launch_swiglu(wb, h->y, M, f, h->gu_blk, h->a, st));
+    SP_CUDA(launch_swiglu(PartIn{h->y, ns, (size_t)M * 2 * f}, M, f, h->gu_blk, h->a.out(tc_down), st));
     mark(SP_STAGE_SWIGLU, 1);
     ++launches;
     // a6-a7: down projection + residual, pooling, linear head
     mark(SP_STAGE_DOWN, 0);
-    s = h->gemm.run(wb, h->opt_gemm, h->a, h->w_down, h->y, M, d, f, st, &launches);
+    s = h->gemm.run(wb, h->opt_gemm, h->a, h->w_down, h->y, M, h->status, st, &launches, &ns);
     mark(SP_STAGE_DOWN, 1);
-    if (s != SP_OK) return s;
+    if (s != SP_OK) return fail(s, "down projection launch failed");
     mark(SP_STAGE_READOUT, 0);
-    SP_CUDA(launch_readout(h->y, h->h1, h->head_w, h->head_b, c.pool, batch, k, d, C, d_logits, st));
+    SP_CUDA(launch_readout(PartIn{h->y, ns, (size_t)M * d}, h->h1, h->head_w, h->head_b, c.pool,
+                           batch, k, d, C, d_logits, st));
     mark(SP_STAGE_READOUT, 1);
     ++launches;
     h->last_launches = launches;
@@ -597,10 +618,50 @@ sp_status sp_attend(sp_stream stream, const sp_attn_dims *dm, int batch, const i
     a.status = d_status;
     a.gathered = d_gathered_pages;
     a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)a.dh));
-    a.out = d_out;
-    a.out_bf16 = out_dtype == SP_BF16;
+    a.out.f32 = out_dtype == SP_F32 ? (float *)d_out : nullptr;
+    a.out.hi = out_dtype == SP_BF16 ? (bf16 *)d_out : nullptr;
+    a.out.lo = nullptr;
     int launches = 0;
     return enqueue_attention(a, d_workspace, workspace_bytes, 0, &launches, (cudaStream_t)stream);
+}
+
+size_t sp_project_workspace_bytes(int M, int N, int K) {
+    if (M < 1 || N < 1 || K < 1) return 0;
+    const size_t planes = align256((size_t)M * K * 2 * sizeof(uint16_t));
+    const int n_sm = sm_count();
+    const TcPlan p = tc_plan(M, N, K, n_sm, (size_t)-1);
+    return planes + align256((size_t)p.splits * M * N * sizeof(float));
+}
+
+sp_status sp_project(sp_stream stream, int M, int N, int K, const float *d_x, const void *d_w,
+                     float *d_y, int path, void *d_workspace, size_t workspace_bytes) {
+    if (M < 1 || N < 1 || K < 1) return fail(SP_ERR_INVALID_ARG, "M, N, K must be >= 1");
+    if (!d_x || !d_w || !d_y) return fail(SP_ERR_INVALID_ARG, "a required pointer is NULL");
+    if (path < 0 || path > 2) return fail(SP_ERR_INVALID_ARG, "bad path");
+    cudaStream_t st = (cudaStream_t)stream;
+    const bool tc_ok = tc_supported(N, K);
+    if (path == 2 && !tc_ok)
+        return fail(SP_ERR_UNSUPPORTED, "tensor path needs N %% 128 == 0 and K %% 64 == 0");
+    if (path == 1 || !tc_ok) {
+        SP_CUDA(launch_gemm_simt(1, d_x, d_w, d_y, M, N, K, st));
+        return SP_OK;
+    }
+    if (!d_workspace || ((uintptr_t)d_workspace & 255))
+        return fail(SP_ERR_INVALID_ARG, "workspace must be non-NULL and 256-byte aligned");
+    const size_t planes = align256((size_t)M * K * 2 * sizeof(uint16_t));
+    if (workspace_bytes < planes + 256) return fail(SP_ERR_INVALID_ARG, "workspace too small");
+    WeightMat w;
+    init_weight(w, d_w, N, K, 1);
+    ActBuf x;
+    init_act(x, d_workspace, M, K, true);
+    if (!w.tc || !x.maps) return fail(SP_ERR_CUDA, "tensor map encoding failed");
+    float *part = (float *)((char *)d_workspace + planes);
+    const TcPlan p = tc_plan(M, N, K, sm_count(), workspace_bytes - planes);
+    SP_CUDA(launch_to_act(d_x, (size_t)M * K, x.out(true), st));
+    const int bi = bn_index(p.bn);
+    SP_CUDA(launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, N, K, part, nullptr, st));
+    SP_CUDA(launch_sum_partials(PartIn{part, p.splits, (size_t)M * N}, (size_t)M * N, d_y, st));
+    return SP_OK;
 }
 
 }  // extern "C"

@@ -174,14 +174,13 @@ __global__ void __launch_bounds__(kThreads) attn_split_simt(AttnArgs a) {
 }
 
 // Merge the split partials of one (sequence, kv head): grid (Hkv, B).
-template <typename TO>
 __global__ void attn_merge_kernel(AttnArgs a) {
     const int g = blockIdx.x, b = blockIdx.y;
     const int R = a.R, dh = a.dh, k = a.k;
-    const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs, a.max_seq_len, nullptr);
+    const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs,
+                                  a.max_seq_len, nullptr);
     const int n_valid = min(a.n_splits, ceil_div(sq.len + k, a.split_tokens));
     const size_t unit0 = ((size_t)b * a.Hkv + g) * a.n_splits;
-    TO *out = (TO *)a.out;
     for (int idx = threadIdx.x; idx < R * dh; idx += blockDim.x) {
         const int rr = idx / dh, c = idx - rr * dh;
         float mmax = -INFINITY;
@@ -196,7 +195,7 @@ __global__ void attn_merge_kernel(AttnArgs a) {
         }
         const int hl = rr / k, r = rr - hl * k;
         const int h = g * a.G + hl;
-        out[(((size_t)b * k + r) * a.Hq + h) * dh + c] = from_f<TO>(l > 0.f ? o / l : 0.f);
+        act_store(a.out, (((size_t)b * k + r) * a.Hq + h) * dh + c, l > 0.f ? o / l : 0.f);
     }
 }
 
@@ -256,10 +255,7 @@ cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st) {
 
 cudaError_t launch_attention_merge(const AttnArgs &a, cudaStream_t st) {
     dim3 grid(a.Hkv, a.B);
-    if (a.out_bf16)
-        attn_merge_kernel<bf16><<<grid, 256, 0, st>>>(a);
-    else
-        attn_merge_kernel<float><<<grid, 256, 0, st>>>(a);
+    attn_merge_kernel<<<grid, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -20,6 +20,37 @@ template <typename T> __device__ __forceinline__ T from_f(float x);
 template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
 template <> __device__ __forceinline__ bf16 from_f<bf16>(float x) { return __float2bfloat16_rn(x); }
 
+// Where a producer writes an activation: fp32 (f32 != null), plain bf16
+// (hi != null, lo == null) or the two-plane form hi = rn(v), lo = rn(v - hi)
+// that the tensor-core projections consume.
+struct ActOut {
+    float *f32;
+    bf16 *hi;
+    bf16 *lo;
+};
+__device__ __forceinline__ void act_store(const ActOut &o, size_t idx, float v) {
+    if (o.f32) {
+        o.f32[idx] = v;
+        return;
+    }
+    const bf16 h = __float2bfloat16_rn(v);
+    o.hi[idx] = h;
+    if (o.lo) o.lo[idx] = __float2bfloat16_rn(v - __bfloat162float(h));
+}
+
+// A projection result held as `n` fp32 partial sums `stride` elements apart
+// (split-K); readers add them.
+struct PartIn {
+    const float *y;
+    int n;
+    size_t stride;
+};
+__device__ __forceinline__ float part_get(const PartIn &p, size_t idx) {
+    float s = p.y[idx];
+    for (int i = 1; i < p.n; ++i) s += p.y[(size_t)i * p.stride + idx];
+    return s;
+}
+
 // Cache description as the kernels see it (same fields as sp_kv_cache).
 struct KVDev {
     int layout;
@@ -85,8 +116,7 @@ struct AttnArgs {
     int *status;
     int *gathered;                // [B][max_pages] or NULL
     float scale_log2;             // log2(e) / sqrt(dh)
-    void *out;                    // merge output [B][k][Hq][dh]
-    int out_bf16;
+    ActOut out;                   // merge output [B][k][Hq][dh]
 };
 
 // Plan: tokens per split-KV work unit and number of units per sequence.
@@ -99,12 +129,13 @@ cudaError_t launch_attention_merge(const AttnArgs &a, cudaStream_t st);
 // ---------------------------------------------------------------------------
 // row-wise steps
 // ---------------------------------------------------------------------------
-// out[m] = RMSNorm(x[src(m)]) * gain, src(m) = m or m % row_mod (shared rows)
-cudaError_t launch_rmsnorm_rows(int w_bf16, const void *x, int row_mod, const float *gain, float eps,
-                                int M, int d, void *out, cudaStream_t st);
+// out[m] = RMSNorm(x[src(m)]) * gain, src(m) = m or m % row_mod (shared rows);
+// x is bf16 (x_bf16) or fp32.
+cudaError_t launch_rmsnorm_rows(int x_bf16, const void *x, int row_mod, const float *gain, float eps,
+                                int M, int d, ActOut out, cudaStream_t st);
 
 struct QkvRopeArgs {
-    const float *y;          // projections [rows][(Hq + 2 Hkv) dh]
+    PartIn y;                // projections [rows][(Hq + 2 Hkv) dh]
     int shared;              // 1: row of m is m % k (shared soft prompt), 0: row m
     int B, k, Hq, Hkv, dh;
     const int *seq_ids, *seq_lens;
@@ -116,25 +147,27 @@ struct QkvRopeArgs {
 };
 cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st);
 
-// h1 = x + y ; n = RMSNorm(h1) * gain   (x: input rows, w dtype; n: activation dtype)
-cudaError_t launch_residual_norm(int w_bf16, const float *y, const void *x, int row_mod,
-                                 const float *gain, float eps, int M, int d, float *h1, void *n,
+// h1 = x + y ; n = RMSNorm(h1) * gain   (x: input rows, bf16 or fp32)
+cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mod,
+                                 const float *gain, float eps, int M, int d, float *h1, ActOut n,
                                  cudaStream_t st);
 
 // a[m][j] = silu(g) * u for gate/up columns laid out in blocks of `blk`
 // (gate block i at columns 2*i*blk.., up block right after it)
-cudaError_t launch_swiglu(int act_bf16, const float *y, int M, int f, int blk, void *a,
-                          cudaStream_t st);
+cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_t st);
 
 // logits[b] = W_head pool_r(h1 + y) + bias
-cudaError_t launch_readout(const float *y, const float *h1, const float *head_w,
-                           const float *head_b, int pool, int B, int k, int d, int C,
-                           float *logits, cudaStream_t st);
+cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
+                           int pool, int B, int k, int d, int C, float *logits, cudaStream_t st);
 
 // ---------------------------------------------------------------------------
 // projections
 // ---------------------------------------------------------------------------
-// Y[M][N] (fp32) = X[M][K] * W[N][K]^T on CUDA cores; X and W share w_bf16.
+// out = x split into ActOut form (n elements); out = sum of the partials.
+cudaError_t launch_to_act(const float *x, size_t n, ActOut out, cudaStream_t st);
+cudaError_t launch_sum_partials(PartIn y, size_t n, float *out, cudaStream_t st);
+
+// Y[M][N] (fp32) = X[M][K] (fp32) * W[N][K]^T (bf16 or fp32) on CUDA cores.
 cudaError_t launch_gemm_simt(int w_bf16, const void *X, const void *W, float *Y, int M, int N,
                              int K, cudaStream_t st);
 

@@ -1,24 +1,108 @@
-// Projection dispatch: chooses the kernel for Y[M][N] = X[M][K] W[N][K]^T.
+// Projection dispatch for Y[M][N] = X[M][K] W[N][K]^T.
+//  - tensor cores (tcgen05, sp_gemm_tc.cu): bf16 weights with N % 128 == 0 and
+//    K % 64 == 0; activations as bf16 hi/lo planes; fp32 split-K partials.
+//  - CUDA cores (sp_rowops.cu): anything else; fp32 activations; one partial.
 #pragma once
+
+#include <cuda.h>
 
 #include "sp_common.cuh"
 
 namespace sp {
 
+struct TcPlan {
+    int bn, m_tiles, n_tiles, n_kb, kb_per_split, splits;
+};
+
+bool encode_kmajor_bf16(CUtensorMap *map, const void *base, int rows, int K, int box_rows);
+bool tc_supported(int N, int K);
+int tc_bn_for(int M);
+TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes);
+cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
+                           const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
+                           float *y, int *status, cudaStream_t st);
+
+constexpr int kNumBn = 4;  // tile widths 16, 32, 64, 128
+inline int bn_index(int bn) { return bn == 16 ? 0 : bn == 32 ? 1 : bn == 64 ? 2 : 3; }
+inline int bn_value(int i) { return 16 << i; }
+
+// A frozen weight matrix on the device, with its TMA map when tensor cores apply.
+struct WeightMat {
+    const void *ptr = nullptr;
+    int N = 0, K = 0;
+    bool tc = false;
+    CUtensorMap map;
+};
+
+// An activation buffer holding up to rows_max rows of K values, either as fp32
+// [rows][K] or as two bf16 planes hi [rows_max][K] then lo [rows_max][K].
+struct ActBuf {
+    void *ptr = nullptr;
+    int K = 0, rows_max = 0;
+    bool maps = false;
+    CUtensorMap hi[kNumBn], lo[kNumBn];
+    ActOut out(bool hilo) const {
+        ActOut o;
+        if (hilo) {
+            o.f32 = nullptr;
+            o.hi = (bf16 *)ptr;
+            o.lo = (bf16 *)ptr + (size_t)rows_max * K;
+        } else {
+            o.f32 = (float *)ptr;
+            o.hi = o.lo = nullptr;
+        }
+        return o;
+    }
+};
+
+inline bool init_weight(WeightMat &w, const void *ptr, int N, int K, int w_bf16) {
+    w.ptr = ptr;
+    w.N = N;
+    w.K = K;
+    w.tc = w_bf16 && tc_supported(N, K) && encode_kmajor_bf16(&w.map, ptr, N, K, 128);
+    return true;
+}
+
+inline void init_act(ActBuf &a, void *ptr, int rows_max, int K, bool want_maps) {
+    a.ptr = ptr;
+    a.K = K;
+    a.rows_max = rows_max;
+    a.maps = false;
+    if (!want_maps || K % 64) return;
+    bool ok = true;
+    const bf16 *hi = (const bf16 *)ptr, *lo = hi + (size_t)rows_max * K;
+    for (int i = 0; i < kNumBn; ++i) {
+        ok = ok && encode_kmajor_bf16(&a.hi[i], hi, rows_max, K, bn_value(i));
+        ok = ok && encode_kmajor_bf16(&a.lo[i], lo, rows_max, K, bn_value(i));
+    }
+    a.maps = ok;
+}
+
 struct GemmPlanner {
     int n_sm = 148;
-    void init(int sms) { n_sm = sms; }
-    // Extra scratch (bytes) the tensor-core path may need for M x N outputs.
-    size_t workspace_bytes(size_t M, size_t N) const {
-        (void)M;
-        (void)N;
-        return 0;
+    size_t y_capacity = 0;  // bytes available for [splits][M][N] partials
+    void init(int sms, size_t cap) {
+        n_sm = sms;
+        y_capacity = cap;
     }
-    // path: 0 automatic, 1 CUDA cores, 2 tensor cores where supported.
-    sp_status run(int w_bf16, int path, const void *X, const void *W, float *Y, int M, int N, int K,
-                  cudaStream_t st, int *launches) const {
-        (void)path;
-        cudaError_t e = launch_gemm_simt(w_bf16, X, W, Y, M, N, K, st);
+    // Does this projection run on tensor cores under path option `path`
+    // (0 automatic, 1 CUDA cores, 2 tensor cores where supported)?
+    bool use_tc(const WeightMat &w, const ActBuf &x, int path) const {
+        return path != 1 && w.tc && x.maps;
+    }
+    // Enqueue the projection; *nsplit receives the number of partials in y.
+    sp_status run(int w_bf16, int path, const ActBuf &x, const WeightMat &w, float *y, int M,
+                  int *status, cudaStream_t st, int *launches, int *nsplit) const {
+        cudaError_t e;
+        if (use_tc(w, x, path)) {
+            const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity);
+            const int bi = bn_index(p.bn);
+            e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st);
+            *nsplit = p.splits;
+        } else {
+            e = launch_gemm_simt(w_bf16, x.ptr, w.ptr, y, M, w.N, w.K, st);
+            *nsplit = 1;
+        }
         if (e != cudaSuccess) return SP_ERR_CUDA;
         ++*launches;
         return SP_OK;

@@ -28,8 +28,7 @@ __device__ __forceinline__ float block_sum(float v, float *red) {
 
 template <typename T>
 __global__ void rmsnorm_rows_kernel(const T *__restrict__ x, int row_mod,
-                                    const float *__restrict__ gain, float eps, int d,
-                                    T *__restrict__ out) {
+                                    const float *__restrict__ gain, float eps, int d, ActOut out) {
     __shared__ float red[32];
     const int m = blockIdx.x;
     const T *xr = x + (size_t)(row_mod ? m % row_mod : m) * d;
@@ -40,8 +39,8 @@ __global__ void rmsnorm_rows_kernel(const T *__restrict__ x, int row_mod,
     }
     ss = block_sum(ss, red);
     const float inv = rsqrtf(ss / (float)d + eps);
-    T *o = out + (size_t)m * d;
-    for (int j = threadIdx.x; j < d; j += blockDim.x) o[j] = from_f<T>(to_f(xr[j]) * inv * gain[j]);
+    for (int j = threadIdx.x; j < d; j += blockDim.x)
+        act_store(out, (size_t)m * d + j, to_f(xr[j]) * inv * gain[j]);
 }
 
 __global__ void qkv_rope_kernel(QkvRopeArgs a) {
@@ -52,12 +51,13 @@ __global__ void qkv_rope_kernel(QkvRopeArgs a) {
     const int pos = s.len + r;
     const int dh = a.dh, half = dh >> 1;
     const int nqkv = (a.Hq + 2 * a.Hkv) * dh;
-    const float *y = a.y + (size_t)(a.shared ? r : m) * nqkv;
+    const size_t row = (size_t)(a.shared ? r : m) * nqkv;
     const float2 *cs = a.rope_cs + (size_t)pos * half;
     const int nrot = (a.Hq + a.Hkv) * half;  // rotated pairs: all q heads, then k heads
     for (int idx = threadIdx.x; idx < nrot; idx += blockDim.x) {
         const int h = idx / half, i = idx - h * half;
-        const float x0 = y[h * dh + i], x1 = y[h * dh + i + half];
+        const float x0 = part_get(a.y, row + h * dh + i);
+        const float x1 = part_get(a.y, row + h * dh + i + half);
         const float2 c = cs[i];
         const float r0 = x0 * c.x - x1 * c.y;
         const float r1 = x1 * c.x + x0 * c.y;
@@ -70,49 +70,46 @@ __global__ void qkv_rope_kernel(QkvRopeArgs a) {
         dst[i] = r0;
         dst[i + half] = r1;
     }
-    const float *yv = y + (a.Hq + a.Hkv) * dh;
+    const size_t vrow = row + (size_t)(a.Hq + a.Hkv) * dh;
     float *v = a.v_new + (size_t)m * a.Hkv * dh;
-    for (int j = threadIdx.x; j < a.Hkv * dh; j += blockDim.x) v[j] = yv[j];
+    for (int j = threadIdx.x; j < a.Hkv * dh; j += blockDim.x) v[j] = part_get(a.y, vrow + j);
 }
 
-template <typename TX, typename TN>
-__global__ void residual_norm_kernel(const float *__restrict__ y, const TX *__restrict__ x,
-                                     int row_mod, const float *__restrict__ gain, float eps, int d,
-                                     float *__restrict__ h1, TN *__restrict__ n) {
+template <typename TX>
+__global__ void residual_norm_kernel(PartIn y, const TX *__restrict__ x, int row_mod,
+                                     const float *__restrict__ gain, float eps, int d,
+                                     float *__restrict__ h1, ActOut n) {
     __shared__ float red[32];
     const int m = blockIdx.x;
     const TX *xr = x + (size_t)(row_mod ? m % row_mod : m) * d;
-    const float *yr = y + (size_t)m * d;
     float *hr = h1 + (size_t)m * d;
     float ss = 0.f;
     for (int j = threadIdx.x; j < d; j += blockDim.x) {
-        float v = to_f(xr[j]) + yr[j];
+        float v = to_f(xr[j]) + part_get(y, (size_t)m * d + j);
         hr[j] = v;
         ss += v * v;
     }
     ss = block_sum(ss, red);
     const float inv = rsqrtf(ss / (float)d + eps);
-    TN *nr = n + (size_t)m * d;
-    for (int j = threadIdx.x; j < d; j += blockDim.x) nr[j] = from_f<TN>(hr[j] * inv * gain[j]);
+    for (int j = threadIdx.x; j < d; j += blockDim.x)
+        act_store(n, (size_t)m * d + j, hr[j] * inv * gain[j]);
 }
 
-template <typename TA>
-__global__ void swiglu_kernel(const float *__restrict__ y, int M, int f, int blk,
-                              TA *__restrict__ a) {
+__global__ void swiglu_kernel(PartIn y, int M, int f, int blk, ActOut a) {
     const long long total = (long long)M * f;
     for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
          idx += (long long)gridDim.x * blockDim.x) {
         const int m = (int)(idx / f), j = (int)(idx - (long long)m * f);
         const int blkid = j / blk, jj = j - blkid * blk;
-        const float *yr = y + (size_t)m * 2 * f;
-        const float g = yr[2 * blkid * blk + jj];
-        const float u = yr[2 * blkid * blk + blk + jj];
+        const size_t row = (size_t)m * 2 * f;
+        const float g = part_get(y, row + 2 * blkid * blk + jj);
+        const float u = part_get(y, row + 2 * blkid * blk + blk + jj);
         const float s = g / (1.f + __expf(-g));
-        a[idx] = from_f<TA>(s * u);
+        act_store(a, (size_t)idx, s * u);
     }
 }
 
-__global__ void readout_kernel(const float *__restrict__ y, const float *__restrict__ h1,
+__global__ void readout_kernel(PartIn y, const float *__restrict__ h1,
                                const float *__restrict__ head_w, const float *__restrict__ head_b,
                                int pool, int k, int d, int C, float *__restrict__ logits) {
     extern __shared__ float pooled[];  // [d]
@@ -124,12 +121,12 @@ __global__ void readout_kernel(const float *__restrict__ y, const float *__restr
         float acc;
         if (pool == SP_POOL_LAST) {
             const size_t o = base + (size_t)(k - 1) * d + j;
-            acc = h1[o] + y[o];
+            acc = h1[o] + part_get(y, o);
         } else {
             acc = 0.f;
             for (int r = 0; r < k; ++r) {
                 const size_t o = base + (size_t)r * d + j;
-                acc += h1[o] + y[o];
+                acc += h1[o] + part_get(y, o);
             }
             acc *= invk;
         }
@@ -145,10 +142,22 @@ __global__ void readout_kernel(const float *__restrict__ y, const float *__restr
     }
 }
 
+__global__ void to_act_kernel(const float *__restrict__ x, size_t n, ActOut out) {
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
+         i += (size_t)gridDim.x * blockDim.x)
+        act_store(out, i, x[i]);
+}
+
+__global__ void sum_partials_kernel(PartIn y, size_t n, float *__restrict__ out) {
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
+         i += (size_t)gridDim.x * blockDim.x)
+        out[i] = part_get(y, i);
+}
+
 // CUDA-core tiled GEMM: Y[M][N] = X[M][K] W[N][K]^T, fp32 accumulation.
 // 64x64 output tile, 32-deep k slices, 256 threads, 4x4 outputs per thread.
 template <typename T>
-__global__ void __launch_bounds__(256) gemm_simt_kernel(const T *__restrict__ X,
+__global__ void __launch_bounds__(256) gemm_simt_kernel(const float *__restrict__ X,
                                                         const T *__restrict__ W,
                                                         float *__restrict__ Y, int M, int N,
                                                         int K) {
@@ -163,7 +172,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T *__restrict__ X,
         for (int idx = tid; idx < BM * BK; idx += 256) {
             const int row = idx / BK, kk = idx - row * BK;
             const int gm = m0 + row, gk = k0 + kk;
-            Xs[kk][row] = (gm < M && gk < K) ? to_f(X[(size_t)gm * K + gk]) : 0.f;
+            Xs[kk][row] = (gm < M && gk < K) ? X[(size_t)gm * K + gk] : 0.f;
             const int gn = n0 + row;
             Ws[kk][row] = (gn < N && gk < K) ? to_f(W[(size_t)gn * K + gk]) : 0.f;
         }
@@ -196,14 +205,14 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T *__restrict__ X,
 
 }  // namespace
 
-cudaError_t launch_rmsnorm_rows(int w_bf16, const void *x, int row_mod, const float *gain,
-                                float eps, int M, int d, void *out, cudaStream_t st) {
-    if (w_bf16)
+cudaError_t launch_rmsnorm_rows(int x_bf16, const void *x, int row_mod, const float *gain,
+                                float eps, int M, int d, ActOut out, cudaStream_t st) {
+    if (x_bf16)
         rmsnorm_rows_kernel<bf16><<<M, kRowThreads, 0, st>>>((const bf16 *)x, row_mod, gain, eps, d,
-                                                             (bf16 *)out);
+                                                             out);
     else
         rmsnorm_rows_kernel<float><<<M, kRowThreads, 0, st>>>((const float *)x, row_mod, gain, eps,
-                                                              d, (float *)out);
+                                                              d, out);
     return cudaGetLastError();
 }
 
@@ -212,33 +221,28 @@ cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_residual_norm(int w_bf16, const float *y, const void *x, int row_mod,
-                                 const float *gain, float eps, int M, int d, float *h1, void *n,
+cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mod,
+                                 const float *gain, float eps, int M, int d, float *h1, ActOut n,
                                  cudaStream_t st) {
-    if (w_bf16)
-        residual_norm_kernel<bf16, bf16><<<M, kRowThreads, 0, st>>>(y, (const bf16 *)x, row_mod,
-                                                                   gain, eps, d, h1, (bf16 *)n);
+    if (x_bf16)
+        residual_norm_kernel<bf16><<<M, kRowThreads, 0, st>>>(y, (const bf16 *)x, row_mod, gain, eps,
+                                                             d, h1, n);
     else
-        residual_norm_kernel<float, float><<<M, kRowThreads, 0, st>>>(y, (const float *)x, row_mod,
-                                                                     gain, eps, d, h1, (float *)n);
+        residual_norm_kernel<float><<<M, kRowThreads, 0, st>>>(y, (const float *)x, row_mod, gain,
+                                                              eps, d, h1, n);
     return cudaGetLastError();
 }
 
-cudaError_t launch_swiglu(int act_bf16, const float *y, int M, int f, int blk, void *a,
-                          cudaStream_t st) {
+cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_t st) {
     const long long total = (long long)M * f;
     int grid = (int)((total + 255) / 256);
     if (grid > 152 * 16) grid = 152 * 16;
-    if (act_bf16)
-        swiglu_kernel<bf16><<<grid, 256, 0, st>>>(y, M, f, blk, (bf16 *)a);
-    else
-        swiglu_kernel<float><<<grid, 256, 0, st>>>(y, M, f, blk, (float *)a);
+    swiglu_kernel<<<grid, 256, 0, st>>>(y, M, f, blk, a);
     return cudaGetLastError();
 }
 
-cudaError_t launch_readout(const float *y, const float *h1, const float *head_w,
-                           const float *head_b, int pool, int B, int k, int d, int C,
-                           float *logits, cudaStream_t st) {
+cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
+                           int pool, int B, int k, int d, int C, float *logits, cudaStream_t st) {
     const size_t smem = (size_t)d * sizeof(float);
     if (smem > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute(readout_kernel,
@@ -249,11 +253,27 @@ cudaError_t launch_readout(const float *y, const float *h1, const float *head_w,
     return cudaGetLastError();
 }
 
+cudaError_t launch_to_act(const float *x, size_t n, ActOut out, cudaStream_t st) {
+    size_t grid = (n + 255) / 256;
+    if (grid > 152 * 16) grid = 152 * 16;
+    if (grid == 0) grid = 1;
+    to_act_kernel<<<(unsigned)grid, 256, 0, st>>>(x, n, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_sum_partials(PartIn y, size_t n, float *out, cudaStream_t st) {
+    size_t grid = (n + 255) / 256;
+    if (grid > 152 * 16) grid = 152 * 16;
+    if (grid == 0) grid = 1;
+    sum_partials_kernel<<<(unsigned)grid, 256, 0, st>>>(y, n, out);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_gemm_simt(int w_bf16, const void *X, const void *W, float *Y, int M, int N,
                              int K, cudaStream_t st) {
     dim3 grid(ceil_div(N, 64), ceil_div(M, 64));
     if (w_bf16)
-        gemm_simt_kernel<bf16><<<grid, 256, 0, st>>>((const bf16 *)X, (const bf16 *)W, Y, M, N, K);
+        gemm_simt_kernel<bf16><<<grid, 256, 0, st>>>((const float *)X, (const bf16 *)W, Y, M, N, K);
     else
         gemm_simt_kernel<float><<<grid, 256, 0, st>>>((const float *)X, (const float *)W, Y, M, N, K);
     return cudaGetLastError();
