@@ -253,6 +253,29 @@ SP_API sp_status sp_attend(sp_stream stream, const sp_attn_dims *dims, int batch
                     void *d_workspace, size_t workspace_bytes, int *d_status,
                     int *d_gathered_pages);
 
+/* sp_attend for callers that cannot allocate device memory; the paper has no
+ * counterpart to this entry point.  A monitor on the decoding hot path must not
+ * call cudaMalloc (it can synchronise the device and stall decoding), and some
+ * serving frameworks give a library no device memory of its own to allocate.
+ * This call takes its split-KV scratch from a 32 MiB array inside the library
+ * (a static device object that every GPU loading the library holds until the
+ * process exits) and allocates nothing; the caller passes the same inputs and
+ * outputs as to sp_attend, without a workspace.
+ *  - A batch whose scratch (sp_attend_workspace_bytes) exceeds 32 MiB is
+ *    rejected with SP_ERR_INVALID_ARG before any launch.
+ *  - The first call on each device looks up the array's device address, with
+ *    that device current, and caches it; make that first call before any
+ *    stream capture.
+ *  - Every call shares the one array and leaves its contents behind: calls
+ *    whose work overlaps on the GPU (other streams, other threads) race on it
+ *    and must be serialised by the caller.  Nothing in it needs clearing: each
+ *    call writes every value it later reads. */
+SP_API sp_status sp_attend_static(sp_stream stream, const sp_attn_dims *dims, int batch,
+                                  const int *d_seq_ids, const int *d_seq_lens,
+                                  const sp_kv_cache *kv, const float *d_q, const float *d_k_new,
+                                  const float *d_v_new, void *d_out, int out_dtype, int *d_status,
+                                  int *d_gathered_pages);
+
 /* ------------------------------------------------------------------------- */
 /* The projection step alone: one of the decoder layer's linear maps (Sec. 3.1)*/
 /* ------------------------------------------------------------------------- */

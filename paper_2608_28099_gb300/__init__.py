@@ -25,7 +25,8 @@ STAGES = ["input_norm", "qkv", "rope", "attention", "merge", "o_proj", "post_nor
 
 EXPORTED = ["sp_create", "sp_destroy", "sp_classify", "sp_classify_host", "sp_check_status",
             "sp_last_error", "sp_set_option", "sp_last_launch_count", "sp_attend_workspace_bytes",
-            "sp_attend", "sp_stage_times", "sp_project_workspace_bytes", "sp_project"]
+            "sp_attend", "sp_stage_times", "sp_project_workspace_bytes", "sp_project",
+            "sp_attend_static"]
 
 
 class sp_config(C.Structure):
@@ -90,6 +91,8 @@ def load_library(path: str | None = None):
     lib.sp_project_workspace_bytes.argtypes = [i, i, i]
     lib.sp_project_workspace_bytes.restype = C.c_size_t
     lib.sp_project.argtypes = [vp, i, i, i, vp, vp, vp, i, vp, C.c_size_t]
+    lib.sp_attend_static.argtypes = [vp, C.POINTER(sp_attn_dims), i, vp, vp,
+                                     C.POINTER(sp_kv_cache), vp, vp, vp, vp, i, vp, vp]
     lib.sp_attend.argtypes = [vp, C.POINTER(sp_attn_dims), i, vp, vp, C.POINTER(sp_kv_cache), vp,
                               vp, vp, vp, i, vp, C.c_size_t, vp, vp]
     for name in EXPORTED:
@@ -171,6 +174,14 @@ def sp_stage_times(handle) -> dict:
     ms = (C.c_float * len(STAGES))()
     _check(load_library().sp_stage_times(handle, ms, len(STAGES)))
     return {name: float(ms[i]) for i, name in enumerate(STAGES) if ms[i] >= 0}
+
+
+def sp_attend_static(stream, dims, batch, seq_ids, seq_lens, kv, q, k_new, v_new, out, out_dtype,
+                     status=None, gathered_pages=None):
+    _check(load_library().sp_attend_static(_stream(stream), C.byref(dims), int(batch),
+                                           _ptr(seq_ids), _ptr(seq_lens), C.byref(kv), _ptr(q),
+                                           _ptr(k_new), _ptr(v_new), _ptr(out), int(out_dtype),
+                                           _ptr(status), _ptr(gathered_pages)))
 
 
 def sp_project_workspace_bytes(M, N, K) -> int:

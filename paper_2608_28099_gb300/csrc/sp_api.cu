@@ -50,6 +50,8 @@ struct Arena {
 
 }  // namespace
 
+void sp::set_error_text(const char *msg) { g_err = msg; }
+
 struct sp_handle {
     sp_config cfg;
     int device = 0, n_sm = 148;

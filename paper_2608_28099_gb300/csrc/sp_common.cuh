@@ -171,4 +171,7 @@ cudaError_t launch_sum_partials(PartIn y, size_t n, float *out, cudaStream_t st)
 cudaError_t launch_gemm_simt(int w_bf16, const void *X, const void *W, float *Y, int M, int N,
                              int K, cudaStream_t st);
 
+// Replace the text sp_last_error() returns on this thread.
+void set_error_text(const char *msg);
+
 }  // namespace sp
