@@ -230,6 +230,10 @@ typedef struct sp_attn_dims {
     int max_seq_len;                     /* bound on the cached lengths             */
     int split_tokens;                    /* tokens per split-KV work unit (multiple
                                             of 64), 0 = automatic plan              */
+    int path;                            /* 0 = automatic, 1 = CUDA-core kernel,
+                                            2 = tensor-core kernel (head_dim 128,
+                                            bf16 cache, G * k <= 128; else
+                                            SP_ERR_UNSUPPORTED)                     */
 } sp_attn_dims;
 
 /* Bytes of device scratch sp_attend needs for `batch` sequences (256-byte

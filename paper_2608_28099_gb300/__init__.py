@@ -52,7 +52,7 @@ class sp_kv_cache(C.Structure):
 class sp_attn_dims(C.Structure):
     _fields_ = [("n_q_heads", C.c_int), ("n_kv_heads", C.c_int), ("head_dim", C.c_int),
                 ("k_rows", C.c_int), ("kv_dtype", C.c_int), ("max_seq_len", C.c_int),
-                ("split_tokens", C.c_int)]
+                ("split_tokens", C.c_int), ("path", C.c_int)]
 
 
 class SpError(RuntimeError):

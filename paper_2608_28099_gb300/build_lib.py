@@ -11,7 +11,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libsp.so")
-SOURCES = ["sp_api.cu", "sp_rowops.cu", "sp_attn_simt.cu", "sp_gemm_tc.cu", "sp_attend_static.cu"]
+SOURCES = ["sp_api.cu", "sp_rowops.cu", "sp_attn_simt.cu", "sp_gemm_tc.cu", "sp_attend_static.cu",
+           "sp_attn_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-Xcompiler", "-fvisibility=hidden"]

@@ -192,9 +192,25 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
     if (ws_bytes < need) return fail(SP_ERR_INVALID_ARG, "attention workspace too small (%zu < %zu)", ws_bytes, need);
     a.part_o = (float *)ws;
     a.part_ml = (float *)((char *)ws + align256((size_t)a.B * a.Hkv * a.n_splits * a.R * a.dh * sizeof(float)));
-    (void)attn_path;
+    bool tc = attn_path != 1 && attention_tc_supported(a);
+    CUtensorMap mk, mv;
+    const CUtensorMap *pk = nullptr, *pv = nullptr;
+    if (tc && a.kv.layout == SP_KV_PAGED) {
+        const long long rows = (long long)a.kv.n_pages * a.Hkv * a.kv.page_size;
+        tc = rows <= 0x7fffffffLL &&
+             encode_kmajor_bf16(&mk, a.kv.k_pool, (int)rows, a.dh, a.kv.page_size) &&
+             encode_kmajor_bf16(&mv, a.kv.v_pool, (int)rows, a.dh, a.kv.page_size);
+        pk = &mk;
+        pv = &mv;
+    }
+    if (attn_path == 2 && !tc)
+        return fail(SP_ERR_UNSUPPORTED, "tensor-core attention needs head_dim 128, a bf16 cache "
+                                        "and at most 128 query rows per kv head");
     if (ev_attn) cudaEventRecord(ev_attn[0], st);
-    SP_CUDA(launch_attention_simt(a, st));
+    if (tc)
+        SP_CUDA(launch_attention_tc(a, pk, pv, st));
+    else
+        SP_CUDA(launch_attention_simt(a, st));
     if (ev_attn) cudaEventRecord(ev_attn[1], st);
     if (ev_merge) cudaEventRecord(ev_merge[0], st);
     SP_CUDA(launch_attention_merge(a, st));
@@ -623,8 +639,10 @@ sp_status sp_attend(sp_stream stream, const sp_attn_dims *dm, int batch, const i
     a.out.f32 = out_dtype == SP_F32 ? (float *)d_out : nullptr;
     a.out.hi = out_dtype == SP_BF16 ? (bf16 *)d_out : nullptr;
     a.out.lo = nullptr;
+    if (dm->path < 0 || dm->path > 2) return fail(SP_ERR_INVALID_ARG, "bad attention path");
     int launches = 0;
-    return enqueue_attention(a, d_workspace, workspace_bytes, 0, &launches, (cudaStream_t)stream);
+    return enqueue_attention(a, d_workspace, workspace_bytes, dm->path, &launches,
+                             (cudaStream_t)stream);
 }
 
 size_t sp_project_workspace_bytes(int M, int N, int K) {

@@ -1,6 +1,7 @@
 // Internal declarations shared by the CUDA translation units of libsp.so.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -124,6 +125,11 @@ void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, in
                     int *split_tokens, int *n_splits);
 size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits);
 cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st);
+// tcgen05 kernel: head_dim 128, bf16 cache, R <= 128; paged caches need TMA
+// maps of the K and V pools viewed as [n_pages * Hkv * page_size][128].
+bool attention_tc_supported(const AttnArgs &a);
+cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
+                                const CUtensorMap *map_v, cudaStream_t st);
 cudaError_t launch_attention_merge(const AttnArgs &a, cudaStream_t st);
 
 // ---------------------------------------------------------------------------

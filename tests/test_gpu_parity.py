@@ -128,15 +128,19 @@ def test_layouts_and_page_permutation_agree_bitwise():
     assert np.array_equal(outs[0], outs[1]) and np.array_equal(outs[1], outs[2])
 
 
-def test_split_plan_does_not_change_results():
+@pytest.mark.parametrize("attn_path", [1, 2])
+def test_split_plan_does_not_change_results(attn_path):
     w = wl.custom(SMALL_BF16, [1000, 2000, 37], wl.LAYOUT_PAGED, 81)
     res = []
     for split in (64, 256, 2048 + 64):
-        run = GpuRun(w, options={sp.SP_OPT_SPLIT_TOKENS: split})
+        run = GpuRun(w, options={sp.SP_OPT_SPLIT_TOKENS: split, sp.SP_OPT_ATTN_PATH: attn_path})
         res.append(run.logits())
         run.close()
+    # fp32 attention: only the merge order changes.  Tensor-core attention: the
+    # split also moves where P is rounded to bf16.
+    tol = 1e-5 if attn_path == 1 else 2e-3
     for r in res[1:]:
-        np.testing.assert_allclose(r, res[0], rtol=1e-5, atol=1e-6)
+        np.testing.assert_allclose(r, res[0], rtol=tol, atol=tol)
     compare(res[0], oracle_logits(w))
 
 
@@ -154,7 +158,8 @@ def test_result_does_not_depend_on_batch_company():
     full = run.logits(use_rows=False)
     for i in range(4):
         one = run.logits(use_rows=False, ids=[i])
-        np.testing.assert_allclose(one[0], full[i], rtol=1e-4, atol=1e-5)
+        # the batch size changes the split plans (rounding points), nothing else
+        np.testing.assert_allclose(one[0], full[i], rtol=2e-3, atol=2e-3)
     run.close()
 
 
@@ -162,8 +167,9 @@ def test_shared_prompt_equals_rows_holding_the_prompt():
     w = wl.custom(SMALL_BF16, [33, 90], wl.LAYOUT_PAGED, 111)
     w.rows = np.stack([w.weights.soft_prompt] * 2)
     run = GpuRun(w)
+    # fp32 projections of the shared prompt vs tensor-core projections of rows
     np.testing.assert_allclose(run.logits(use_rows=True), run.logits(use_rows=False),
-                               rtol=1e-4, atol=1e-5)
+                               rtol=2e-3, atol=2e-3)
     run.close()
 
 
@@ -184,40 +190,82 @@ def test_host_entry_point_matches_device_entry_point():
 # --------------------------------------------------------------------------- #
 # the attention step alone and its page gather
 # --------------------------------------------------------------------------- #
-@pytest.mark.parametrize("kv_dtype", [wl.F32, wl.BF16])
-def test_attention_step_and_gathered_pages(kv_dtype):
+def _attend(shape, w, q, kn, vn, path, split=128):
     torch = torch_dev()
-    ensure_built()
-    shape = wl.Shape(256, 8, 2, 64, 256, 5, 2, kv_dtype=kv_dtype)
-    lens = [0, 16, 17, 250, 1000]
-    w = wl.custom(shape, lens, wl.LAYOUT_PAGED, 131)
-    rng = np.random.default_rng(7)
+    lens = [int(x) for x in w.cache.seq_lens]
     B, k = len(lens), shape.k_rows
-    q = rng.standard_normal((B, k, shape.n_q_heads, shape.head_dim)).astype(np.float32)
-    kn = rng.standard_normal((B, k, shape.n_kv_heads, shape.head_dim)).astype(np.float32)
-    vn = rng.standard_normal((B, k, shape.n_kv_heads, shape.head_dim)).astype(np.float32)
-    ref = so.attention_step(shape, w.cache, w.seq_ids, q.astype(np.float64), kn.astype(np.float64),
-                            vn.astype(np.float64))
     cache = sp.DeviceCache(w.cache)
-    dims = sp.sp_attn_dims(shape.n_q_heads, shape.n_kv_heads, shape.head_dim, k, kv_dtype,
-                           max(lens), 128)
+    dims = sp.sp_attn_dims(shape.n_q_heads, shape.n_kv_heads, shape.head_dim, k, shape.kv_dtype,
+                           max(lens), split, path)
     ws_bytes = sp.sp_attend_workspace_bytes(dims, B)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
-    out = torch.empty(q.shape, dtype=torch.float32, device="cuda")
+    out = torch.full(q.shape, float("nan"), dtype=torch.float32, device="cuda")
     status = torch.zeros(1, dtype=torch.int32, device="cuda")
-    gathered = torch.full((B, w.cache.max_pages), -7, dtype=torch.int32, device="cuda")
+    gathered = None
+    if w.cache.layout == wl.LAYOUT_PAGED:
+        gathered = torch.full((B, w.cache.max_pages), -7, dtype=torch.int32, device="cuda")
     sp.sp_attend(torch.cuda.current_stream(), dims, B, None, cache.seq_lens, cache.desc,
                  torch.from_numpy(q).cuda(), torch.from_numpy(kn).cuda(), torch.from_numpy(vn).cuda(),
                  out, sp.SP_F32, ws, ws_bytes, status, gathered)
     torch.cuda.synchronize()
     assert int(status.item()) == 0
-    tol = 1e-5 if kv_dtype == wl.F32 else 1e-5
-    np.testing.assert_allclose(out.cpu().numpy(), ref, rtol=tol * 10, atol=tol * 10)
-    g = gathered.cpu().numpy()
-    for b, L in enumerate(lens):
-        npg = (L + 15) // 16
-        assert np.array_equal(g[b, :npg], w.cache.page_table[b, :npg])  # bit-exact ids
-        assert np.all(g[b, npg:] == -7)                                 # nothing else read
+    return out.cpu().numpy(), (None if gathered is None else gathered.cpu().numpy())
+
+
+ATTN_CASES = [
+    # kv dtype, head_dim, layout, q heads, kv heads, k rows, page size, path
+    (wl.F32, 64, wl.LAYOUT_PAGED, 8, 2, 5, 16, 1),
+    (wl.BF16, 64, wl.LAYOUT_PAGED, 8, 2, 5, 16, 1),
+    (wl.BF16, 128, wl.LAYOUT_PAGED, 8, 2, 5, 16, 2),
+    (wl.BF16, 128, wl.LAYOUT_CONTIGUOUS, 8, 2, 5, 16, 2),
+    (wl.BF16, 128, wl.LAYOUT_PAGED, 8, 2, 32, 16, 2),     # 128 query rows per kv head
+    (wl.BF16, 128, wl.LAYOUT_PAGED, 10, 2, 16, 32, 2),    # G=5 as in the 27B shape, 32-token pages
+    (wl.BF16, 128, wl.LAYOUT_PAGED, 4, 4, 1, 64, 2),      # MHA, k=1, 64-token pages
+    (wl.BF16, 128, wl.LAYOUT_CONTIGUOUS, 16, 2, 9, 16, 2),
+]
+
+
+@pytest.mark.parametrize("case", ATTN_CASES, ids=lambda c: "-".join(map(str, c)))
+def test_attention_step_and_gathered_pages(case):
+    ensure_built()
+    kv_dtype, dh, layout, hq, hkv, k, P, path = case
+    shape = wl.Shape(256, hq, hkv, dh, 256, k, 2, kv_dtype=kv_dtype, page_size=P)
+    lens = [0, 16, 17, 250, 1000, 64, 127]
+    w = wl.custom(shape, lens, layout, 131)
+    rng = np.random.default_rng(7)
+    B = len(lens)
+    q = rng.standard_normal((B, k, hq, dh)).astype(np.float32)
+    kn = rng.standard_normal((B, k, hkv, dh)).astype(np.float32)
+    vn = rng.standard_normal((B, k, hkv, dh)).astype(np.float32)
+    ref = so.attention_step(shape, w.cache, w.seq_ids, q.astype(np.float64), kn.astype(np.float64),
+                            vn.astype(np.float64))
+    out, g = _attend(shape, w, q, kn, vn, path)
+    # CUDA cores: fp32 throughout.  Tensor cores: Q as bf16 hi+lo, P and the new
+    # keys/values as bf16, fp32 accumulation.
+    tol = 1e-4 if path == 1 else 1e-2
+    np.testing.assert_allclose(out, ref, rtol=tol, atol=tol)
+    if g is not None:
+        for b, L in enumerate(lens):
+            npg = (L + P - 1) // P
+            assert np.array_equal(g[b, :npg], w.cache.page_table[b, :npg])  # bit-exact ids
+            assert np.all(g[b, npg:] == -7)                                 # nothing else read
+
+
+@pytest.mark.parametrize("layout", [wl.LAYOUT_PAGED, wl.LAYOUT_CONTIGUOUS])
+def test_attention_tensor_and_cuda_core_kernels_agree(layout):
+    ensure_built()
+    shape = wl.Shape(256, 32, 8, 128, 256, 8, 2)
+    lens = [3000, 70, 1025, 0, 4096]
+    w = wl.custom(shape, lens, layout, 137)
+    rng = np.random.default_rng(8)
+    B = len(lens)
+    q = (rng.standard_normal((B, 8, 32, 128))).astype(np.float32)
+    kn = rng.standard_normal((B, 8, 8, 128)).astype(np.float32)
+    vn = rng.standard_normal((B, 8, 8, 128)).astype(np.float32)
+    tc, _ = _attend(shape, w, q, kn, vn, 2, split=0)
+    ref, _ = _attend(shape, w, q, kn, vn, 1, split=0)
+    np.testing.assert_allclose(tc, ref, rtol=1e-2, atol=1e-2)
+    assert np.sqrt(np.mean((tc - ref) ** 2)) < 2e-3
 
 
 # --------------------------------------------------------------------------- #
