@@ -185,13 +185,17 @@ SP_API const char *sp_last_error(void);
  * key or value. */
 enum {
     SP_OPT_SPLIT_TOKENS = 1,  /* attention tokens per split-KV work unit (multiple
-                                 of 64), 0 = automatic plan                      */
+                                 of 64), 0 = automatic plan; a finer plan than
+                                 sp_create sized for grows the handle's scratch
+                                 here (the only allocation after sp_create)      */
     SP_OPT_GEMM_PATH = 2,     /* 0 = automatic, 1 = CUDA-core kernels only,
                                  2 = tensor-core kernels wherever supported       */
     SP_OPT_ATTN_PATH = 3,     /* 0 = automatic, 1 = CUDA-core kernel only,
                                  2 = tensor-core kernel wherever supported        */
     SP_OPT_PROFILE = 4        /* 1 = record CUDA events around every stage of
-                                 sp_classify on its stream, 0 = off (default)    */
+                                 sp_classify on its stream (as external event
+                                 nodes when the call is captured in a graph),
+                                 0 = off (default)                              */
 };
 
 /* Stages of sp_classify, in launch order. */

@@ -77,6 +77,7 @@ struct sp_handle {
     int *stage_ids = nullptr, *stage_lens = nullptr;
     void *stage_rows = nullptr;
     float *stage_logits = nullptr;
+    float *readout_part = nullptr;  // [B][chunks][C] partial head dot products
     GemmPlanner gemm;
     // options
     int opt_split = 0, opt_gemm = 0, opt_attn = 0, opt_profile = 0;
@@ -206,15 +207,15 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
     if (attn_path == 2 && !tc)
         return fail(SP_ERR_UNSUPPORTED, "tensor-core attention needs head_dim 128, a bf16 cache "
                                         "and at most 128 query rows per kv head");
-    if (ev_attn) cudaEventRecord(ev_attn[0], st);
+    if (ev_attn) cudaEventRecordWithFlags(ev_attn[0], st, cudaEventRecordExternal);
     if (tc)
         SP_CUDA(launch_attention_tc(a, pk, pv, st));
     else
         SP_CUDA(launch_attention_simt(a, st));
-    if (ev_attn) cudaEventRecord(ev_attn[1], st);
-    if (ev_merge) cudaEventRecord(ev_merge[0], st);
+    if (ev_attn) cudaEventRecordWithFlags(ev_attn[1], st, cudaEventRecordExternal);
+    if (ev_merge) cudaEventRecordWithFlags(ev_merge[0], st, cudaEventRecordExternal);
     SP_CUDA(launch_attention_merge(a, st));
-    if (ev_merge) cudaEventRecord(ev_merge[1], st);
+    if (ev_merge) cudaEventRecordWithFlags(ev_merge[1], st, cudaEventRecordExternal);
     *launches += 2;
     return SP_OK;
 }
@@ -324,7 +325,8 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
                             (size_t)c.max_batch * 4,    // stage lens
                             M * d * es,                 // stage rows
                             (size_t)c.max_batch * C * 4,  // stage logits
-                            (size_t)k * h->nqkv * 4};   // qkv_shared
+                            (size_t)k * h->nqkv * 4,    // qkv_shared
+                            readout_scratch_bytes(c.max_batch, d, C)};  // readout partials
     for (size_t sz : sizes) total += align256(sz);
     void *arena = nullptr;
     if ((st = dev_alloc(h, &arena, total)) != SP_OK) return cleanup(st);
@@ -346,6 +348,7 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     h->stage_rows = h->arena.take(sizes[13]);
     h->stage_logits = (float *)h->arena.take(sizes[14]);
     h->qkv_shared = (float *)h->arena.take(sizes[15]);
+    h->readout_part = (float *)h->arena.take(sizes[16]);
     init_act(h->xn, p_xn, (int)M, d, h->w_qkv.tc);
     init_act(h->o, p_o_act, (int)M, hq * dh, h->w_o.tc);
     init_act(h->n, p_n, (int)M, d, h->w_gu.tc);
@@ -384,8 +387,14 @@ sp_status sp_set_option(sp_handle *h, int key, int value) {
     case SP_OPT_SPLIT_TOKENS: {
         if (value < 0 || value % 64) return fail(SP_ERR_INVALID_ARG, "split tokens must be a multiple of 64");
         const size_t need = max_attention_ws(h->cfg, h->n_sm, value);
-        if (need > h->attn_ws_bytes)
-            return fail(SP_ERR_INVALID_ARG, "split of %d tokens needs more scratch than sp_create sized", value);
+        if (need > h->attn_ws_bytes) {
+            // a finer forced plan: grow the attention scratch now, never in classify
+            void *p = nullptr;
+            sp_status st = dev_alloc(h, &p, need);
+            if (st != SP_OK) return st;
+            h->attn_ws = p;
+            h->attn_ws_bytes = need;
+        }
         h->opt_split = value;
         return SP_OK;
     }
@@ -445,7 +454,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     for (bool &u : h->ev_used) u = false;
     auto mark = [&](int stage, int end) {
         if (!h->opt_profile) return;
-        cudaEventRecord(h->ev[stage][end], st);
+        cudaEventRecordWithFlags(h->ev[stage][end], st, cudaEventRecordExternal);
         h->ev_used[stage] = true;
     };
 
@@ -531,9 +540,9 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     if (s != SP_OK) return fail(s, "down projection launch failed");
     mark(SP_STAGE_READOUT, 0);
     SP_CUDA(launch_readout(PartIn{h->y, ns, (size_t)M * d}, h->h1, h->head_w, h->head_b, c.pool,
-                           batch, k, d, C, d_logits, st));
+                           batch, k, d, C, h->readout_part, d_logits, st));
     mark(SP_STAGE_READOUT, 1);
-    ++launches;
+    launches += 2;
     h->last_launches = launches;
     return SP_OK;
 }

@@ -173,7 +173,10 @@ __global__ void __launch_bounds__(kThreads) attn_split_simt(AttnArgs a) {
     }
 }
 
-// Merge the split partials of one (sequence, kv head): grid (Hkv, B).
+// Merge the split partials: block (kv head g, sequence b, row group) combines
+// up to 8 query rows; thread c handles output column c (head_dim threads).
+constexpr int kMergeRows = 8;
+
 __global__ void attn_merge_kernel(AttnArgs a) {
     const int g = blockIdx.x, b = blockIdx.y;
     const int R = a.R, dh = a.dh, k = a.k;
@@ -181,8 +184,8 @@ __global__ void attn_merge_kernel(AttnArgs a) {
                                   a.max_seq_len, nullptr);
     const int n_valid = min(a.n_splits, ceil_div(sq.len + k, a.split_tokens));
     const size_t unit0 = ((size_t)b * a.Hkv + g) * a.n_splits;
-    for (int idx = threadIdx.x; idx < R * dh; idx += blockDim.x) {
-        const int rr = idx / dh, c = idx - rr * dh;
+    const int c = threadIdx.x;
+    for (int rr = blockIdx.z * kMergeRows; rr < min(R, (blockIdx.z + 1) * kMergeRows); ++rr) {
         float mmax = -INFINITY;
         for (int s = 0; s < n_valid; ++s) mmax = fmaxf(mmax, a.part_ml[((unit0 + s) * R + rr) * 2]);
         float l = 0.f, o = 0.f;
@@ -223,11 +226,20 @@ void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, in
     if (forced_split > 0) {
         chunk = forced_split;
     } else {
-        const int units = B * Hkv;
-        const int target = 2 * n_sm;
-        const int s = units >= target ? 1 : ceil_div(target, units);
-        chunk = ceil_div(ceil_div(total, s), 64) * 64;
-        if (chunk < 64) chunk = 64;
+        // Aim for about four waves of one-CTA-per-SM work units over the
+        // longest sequence, with splits long enough to amortise a unit's
+        // start-up (>= 512 tokens unless the sequence is shorter) and short
+        // enough that one split's page ids fit in shared memory (<= 16384).
+        const long long units = (long long)B * Hkv;
+        const long long want = 4LL * n_sm;
+        long long s = (want + units - 1) / units;
+        if (s < 1) s = 1;
+        chunk = (int)((total + s - 1) / s);
+        chunk = ((chunk + 63) / 64) * 64;
+        if (chunk < 512) chunk = 512;
+        if (chunk > 16384) chunk = 16384;
+        const int whole = ((total + 63) / 64) * 64;
+        if (chunk > whole) chunk = whole;
     }
     *split_tokens = chunk;
     *n_splits = ceil_div(total, chunk);
@@ -254,8 +266,8 @@ cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st) {
 }
 
 cudaError_t launch_attention_merge(const AttnArgs &a, cudaStream_t st) {
-    dim3 grid(a.Hkv, a.B);
-    attn_merge_kernel<<<grid, 256, 0, st>>>(a);
+    dim3 grid(a.Hkv, a.B, ceil_div(a.R, kMergeRows));
+    attn_merge_kernel<<<grid, a.dh, 0, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -46,7 +46,9 @@ constexpr int OFF_QHI = 0;
 constexpr int OFF_QLO = OFF_QHI + 2 * QSUB;
 constexpr int OFF_KV = OFF_QLO + 2 * QSUB;
 constexpr int OFF_P = OFF_KV + STG * KV_STAGE;
-constexpr int OFF_BAR = OFF_P + 2 * QSUB;
+constexpr int MAX_SPLIT_PAGES = 1024;          // page ids of one split staged in smem
+constexpr int OFF_PAGES = OFF_P + 2 * QSUB;
+constexpr int OFF_BAR = OFF_PAGES + MAX_SPLIT_PAGES * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
 constexpr int THREADS = 192;
 constexpr float RESCALE_LOG2 = 8.f;            // tolerate p <= 2^8 before rescaling O
@@ -155,6 +157,14 @@ __global__ void __launch_bounds__(THREADS, 1)
         int bad = 0;
         const int P = a.kv.page_size;
         const int *ptab = paged ? a.kv.page_table + (size_t)max(sq.sid, 0) * a.kv.max_pages : nullptr;
+        // this split's page ids, read once (coalesced) into shared memory;
+        // entries past the page-table row read as -1
+        int *spages = (int *)(smem + OFF_PAGES);
+        const int lp0 = paged ? t_begin / P : 0;
+        const int n_lp = paged ? min(MAX_SPLIT_PAGES, ceil_div(min(t_end, L) - t_begin, P)) : 0;
+        for (int j = lane; j < n_lp; j += 32)
+            spages[j] = (lp0 + j < a.kv.max_pages) ? ptab[lp0 + j] : -1;
+        __syncwarp();
         for (int i = 0; i < n_tiles; ++i) {
             const int st = i % STG;
             if (!mbar_wait(&bars->kv_empty[st], ((i / STG) & 1) ^ 1, abort)) break;
@@ -165,9 +175,11 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (pure && paged) {
                 const int npg = TT / P;
                 bool ok = true;
+                const int jl = (t0 - t_begin) / P;  // index into spages
                 if (lane < npg) {
                     const int lp = t0 / P + lane;
-                    const int page = lp < a.kv.max_pages ? ptab[lp] : -1;
+                    const int page = jl + lane < n_lp ? spages[jl + lane]
+                                                      : (lp < a.kv.max_pages ? ptab[lp] : -1);
                     ok = page >= 0 && page < a.kv.n_pages;
                     if (ok && a.gathered) a.gathered[(size_t)b * a.kv.max_pages + lp] = page;
                 }
@@ -176,7 +188,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     if (lane == 0) {
                         mbar_arrive_expect_tx(&bars->kv_full[st], KV_STAGE);
                         for (int j = 0; j < npg; ++j) {
-                            const int page = ptab[t0 / P + j];
+                            const int page = jl + j < n_lp ? spages[jl + j] : ptab[t0 / P + j];
                             const int row = (page * a.Hkv + g) * P;
                             const uint32_t off = (uint32_t)(j * P * 128);
                             tma_load_2d(K + off, &map_k, &bars->kv_full[st], 0, row);

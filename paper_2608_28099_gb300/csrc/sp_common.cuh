@@ -162,9 +162,12 @@ cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mo
 // (gate block i at columns 2*i*blk.., up block right after it)
 cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_t st);
 
-// logits[b] = W_head pool_r(h1 + y) + bias
+// logits[b] = W_head pool_r(h1 + y) + bias, via per-chunk partial dot
+// products in `scratch` (readout_scratch_bytes); two launches.
+size_t readout_scratch_bytes(int B, int d, int C);
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
-                           int pool, int B, int k, int d, int C, float *logits, cudaStream_t st);
+                           int pool, int B, int k, int d, int C, float *scratch, float *logits,
+                           cudaStream_t st);
 
 // ---------------------------------------------------------------------------
 // projections

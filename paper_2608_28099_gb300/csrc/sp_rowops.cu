@@ -8,6 +8,7 @@ namespace sp {
 namespace {
 
 constexpr int kRowThreads = 256;
+constexpr int kWideThreads = 1024;
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -15,14 +16,14 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
-// Block-wide sum for blockDim.x == kRowThreads.
+// Block-wide sum (any multiple of 32 threads up to 1024).
 __device__ __forceinline__ float block_sum(float v, float *red) {
     v = warp_sum(v);
     const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
     __syncthreads();
     if (l == 0) red[w] = v;
     __syncthreads();
-    float t = (l < kRowThreads / 32) ? red[l] : 0.f;
+    float t = (l < (int)(blockDim.x >> 5)) ? red[l] : 0.f;
     return warp_sum(t);
 }
 
@@ -43,36 +44,34 @@ __global__ void rmsnorm_rows_kernel(const T *__restrict__ x, int row_mod,
         act_store(out, (size_t)m * d + j, to_f(xr[j]) * inv * gain[j]);
 }
 
+// One thread per rotated pair (query heads, then key heads) or value element
+// of one row: grid (ceil(per_row / 256), B * k).
 __global__ void qkv_rope_kernel(QkvRopeArgs a) {
-    const int m = blockIdx.x;
+    const int m = blockIdx.y;
     const int b = m / a.k, r = m % a.k;
-    SeqRef s = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.n_seqs, a.max_seq_len,
-                           threadIdx.x == 0 ? a.status : nullptr);
-    const int pos = s.len + r;
     const int dh = a.dh, half = dh >> 1;
+    const int nrot = (a.Hq + a.Hkv) * half;
+    const int nval = a.Hkv * dh;
+    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= nrot + nval) return;
+    SeqRef s = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.n_seqs, a.max_seq_len,
+                           idx == 0 ? a.status : nullptr);
     const int nqkv = (a.Hq + 2 * a.Hkv) * dh;
     const size_t row = (size_t)(a.shared ? r : m) * nqkv;
-    const float2 *cs = a.rope_cs + (size_t)pos * half;
-    const int nrot = (a.Hq + a.Hkv) * half;  // rotated pairs: all q heads, then k heads
-    for (int idx = threadIdx.x; idx < nrot; idx += blockDim.x) {
+    if (idx < nrot) {
+        const int pos = s.len + r;
         const int h = idx / half, i = idx - h * half;
         const float x0 = part_get(a.y, row + h * dh + i);
         const float x1 = part_get(a.y, row + h * dh + i + half);
-        const float2 c = cs[i];
-        const float r0 = x0 * c.x - x1 * c.y;
-        const float r1 = x1 * c.x + x0 * c.y;
-        float *dst;
-        if (h < a.Hq) {
-            dst = a.q + ((size_t)m * a.Hq + h) * dh;
-        } else {
-            dst = a.k_new + ((size_t)m * a.Hkv + (h - a.Hq)) * dh;
-        }
-        dst[i] = r0;
-        dst[i + half] = r1;
+        const float2 c = a.rope_cs[(size_t)pos * half + i];
+        float *dst = h < a.Hq ? a.q + ((size_t)m * a.Hq + h) * dh
+                              : a.k_new + ((size_t)m * a.Hkv + (h - a.Hq)) * dh;
+        dst[i] = x0 * c.x - x1 * c.y;
+        dst[i + half] = x1 * c.x + x0 * c.y;
+    } else {
+        const int j = idx - nrot;
+        a.v_new[(size_t)m * nval + j] = part_get(a.y, row + (size_t)(a.Hq + a.Hkv) * dh + j);
     }
-    const size_t vrow = row + (size_t)(a.Hq + a.Hkv) * dh;
-    float *v = a.v_new + (size_t)m * a.Hkv * dh;
-    for (int j = threadIdx.x; j < a.Hkv * dh; j += blockDim.x) v[j] = part_get(a.y, vrow + j);
 }
 
 template <typename TX>
@@ -109,36 +108,55 @@ __global__ void swiglu_kernel(PartIn y, int M, int f, int blk, ActOut a) {
     }
 }
 
-__global__ void readout_kernel(PartIn y, const float *__restrict__ h1,
-                               const float *__restrict__ head_w, const float *__restrict__ head_b,
-                               int pool, int k, int d, int C, float *__restrict__ logits) {
-    extern __shared__ float pooled[];  // [d]
+// Pooling and the linear head, column-parallel: block (chunk, b) pools 512
+// hidden columns of sequence b (h2 = h1 + y over the k rows, mean or last) and
+// writes its partial dot products with every head row to part[b][chunk][C].
+constexpr int kReadoutCols = 512;
+
+__global__ void readout_partial_kernel(PartIn y, const float *__restrict__ h1,
+                                       const float *__restrict__ head_w, int pool, int k, int d,
+                                       int C, float *__restrict__ part) {
     __shared__ float red[32];
-    const int b = blockIdx.x;
+    const int chunk = blockIdx.x, b = blockIdx.y;
     const size_t base = (size_t)b * k * d;
     const float invk = 1.f / (float)k;
-    for (int j = threadIdx.x; j < d; j += blockDim.x) {
-        float acc;
-        if (pool == SP_POOL_LAST) {
-            const size_t o = base + (size_t)(k - 1) * d + j;
-            acc = h1[o] + part_get(y, o);
-        } else {
-            acc = 0.f;
-            for (int r = 0; r < k; ++r) {
-                const size_t o = base + (size_t)r * d + j;
-                acc += h1[o] + part_get(y, o);
+    float pv[2];
+    int col[2];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+        col[e] = chunk * kReadoutCols + threadIdx.x + e * 256;
+        float acc = 0.f;
+        if (col[e] < d) {
+            if (pool == SP_POOL_LAST) {
+                const size_t o = base + (size_t)(k - 1) * d + col[e];
+                acc = h1[o] + part_get(y, o);
+            } else {
+                for (int r = 0; r < k; ++r) {
+                    const size_t o = base + (size_t)r * d + col[e];
+                    acc += h1[o] + part_get(y, o);
+                }
+                acc *= invk;
             }
-            acc *= invk;
         }
-        pooled[j] = acc;
+        pv[e] = acc;
     }
-    __syncthreads();
     for (int c = 0; c < C; ++c) {
         float acc = 0.f;
-        const float *wr = head_w + (size_t)c * d;
-        for (int j = threadIdx.x; j < d; j += blockDim.x) acc += wr[j] * pooled[j];
+#pragma unroll
+        for (int e = 0; e < 2; ++e)
+            if (col[e] < d) acc += head_w[(size_t)c * d + col[e]] * pv[e];
         acc = block_sum(acc, red);
-        if (threadIdx.x == 0) logits[(size_t)b * C + c] = acc + (head_b ? head_b[c] : 0.f);
+        if (threadIdx.x == 0) part[((size_t)b * gridDim.x + chunk) * C + c] = acc;
+    }
+}
+
+__global__ void readout_finish_kernel(const float *__restrict__ part, int n_chunks, int C,
+                                      const float *__restrict__ head_b, float *__restrict__ logits) {
+    const int b = blockIdx.x;
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        float acc = head_b ? head_b[c] : 0.f;
+        for (int j = 0; j < n_chunks; ++j) acc += part[((size_t)b * n_chunks + j) * C + c];
+        logits[(size_t)b * C + c] = acc;
     }
 }
 
@@ -217,7 +235,9 @@ cudaError_t launch_rmsnorm_rows(int x_bf16, const void *x, int row_mod, const fl
 }
 
 cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st) {
-    qkv_rope_kernel<<<a.B * a.k, 128, 0, st>>>(a);
+    const int per_row = (a.Hq + a.Hkv) * (a.dh / 2) + a.Hkv * a.dh;
+    dim3 grid(ceil_div(per_row, 256), a.B * a.k);
+    qkv_rope_kernel<<<grid, 256, 0, st>>>(a);
     return cudaGetLastError();
 }
 
@@ -225,11 +245,11 @@ cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mo
                                  const float *gain, float eps, int M, int d, float *h1, ActOut n,
                                  cudaStream_t st) {
     if (x_bf16)
-        residual_norm_kernel<bf16><<<M, kRowThreads, 0, st>>>(y, (const bf16 *)x, row_mod, gain, eps,
-                                                             d, h1, n);
-    else
-        residual_norm_kernel<float><<<M, kRowThreads, 0, st>>>(y, (const float *)x, row_mod, gain,
+        residual_norm_kernel<bf16><<<M, kWideThreads, 0, st>>>(y, (const bf16 *)x, row_mod, gain,
                                                               eps, d, h1, n);
+    else
+        residual_norm_kernel<float><<<M, kWideThreads, 0, st>>>(y, (const float *)x, row_mod, gain,
+                                                               eps, d, h1, n);
     return cudaGetLastError();
 }
 
@@ -241,15 +261,18 @@ cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_
     return cudaGetLastError();
 }
 
+size_t readout_scratch_bytes(int B, int d, int C) {
+    return (size_t)B * ceil_div(d, kReadoutCols) * C * sizeof(float);
+}
+
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
-                           int pool, int B, int k, int d, int C, float *logits, cudaStream_t st) {
-    const size_t smem = (size_t)d * sizeof(float);
-    if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(readout_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-    }
-    readout_kernel<<<B, kRowThreads, smem, st>>>(y, h1, head_w, head_b, pool, k, d, C, logits);
+                           int pool, int B, int k, int d, int C, float *scratch, float *logits,
+                           cudaStream_t st) {
+    const int chunks = ceil_div(d, kReadoutCols);
+    readout_partial_kernel<<<dim3(chunks, B), 256, 0, st>>>(y, h1, head_w, pool, k, d, C, scratch);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    readout_finish_kernel<<<B, 64, 0, st>>>(scratch, chunks, C, head_b, logits);
     return cudaGetLastError();
 }
 
