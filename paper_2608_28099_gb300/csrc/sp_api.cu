@@ -192,7 +192,8 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
     const size_t need = attention_workspace_bytes(a.B, a.Hkv, a.R, a.dh, a.n_splits);
     if (ws_bytes < need) return fail(SP_ERR_INVALID_ARG, "attention workspace too small (%zu < %zu)", ws_bytes, need);
     a.part_o = (float *)ws;
-    a.part_ml = (float *)((char *)ws + align256((size_t)a.B * a.Hkv * a.n_splits * a.R * a.dh * sizeof(float)));
+    a.part_ml = (float *)((char *)ws + align256((size_t)a.B * a.Hkv * a.n_splits * 2 * a.R * a.dh *
+                                                 sizeof(float)));
     bool tc = attn_path != 1 && attention_tc_supported(a);
     CUtensorMap mk, mv;
     const CUtensorMap *pk = nullptr, *pv = nullptr;
@@ -207,6 +208,7 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
     if (attn_path == 2 && !tc)
         return fail(SP_ERR_UNSUPPORTED, "tensor-core attention needs head_dim 128, a bf16 cache "
                                         "and at most 128 query rows per kv head");
+    a.subs = tc ? 2 : 1;
     if (ev_attn) cudaEventRecordWithFlags(ev_attn[0], st, cudaEventRecordExternal);
     if (tc)
         SP_CUDA(launch_attention_tc(a, pk, pv, st));

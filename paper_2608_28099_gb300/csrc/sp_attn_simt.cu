@@ -182,8 +182,8 @@ __global__ void attn_merge_kernel(AttnArgs a) {
     const int R = a.R, dh = a.dh, k = a.k;
     const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs,
                                   a.max_seq_len, nullptr);
-    const int n_valid = min(a.n_splits, ceil_div(sq.len + k, a.split_tokens));
-    const size_t unit0 = ((size_t)b * a.Hkv + g) * a.n_splits;
+    const int n_valid = min(a.n_splits, ceil_div(sq.len + k, a.split_tokens)) * a.subs;
+    const size_t unit0 = ((size_t)b * a.Hkv + g) * a.n_splits * a.subs;
     const int c = threadIdx.x;
     for (int rr = blockIdx.z * kMergeRows; rr < min(R, (blockIdx.z + 1) * kMergeRows); ++rr) {
         float mmax = -INFINITY;
@@ -246,7 +246,7 @@ void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, in
 }
 
 size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits) {
-    const size_t units = (size_t)B * Hkv * n_splits;
+    const size_t units = (size_t)B * Hkv * n_splits * 2;  // up to two partials per unit
     size_t o = units * R * dh * sizeof(float);
     o = (o + 255) & ~(size_t)255;
     return o + ((units * R * 2 * sizeof(float) + 255) & ~(size_t)255);

@@ -7,22 +7,28 @@
 // R = G * k query rows of the KV head's group share every K/V tile: the GQA
 // group and the k soft-prompt rows together form the M side of the MMA.
 //
-// Per 64-token tile i:
-//   S_i  = Q K_i^T            M = 128 query rows, N = 64 tokens, K = 128 dims,
-//                             Q split into bf16 hi + lo (two MMAs per step),
-//                             S double-buffered in TMEM
-//   softmax                   4 warps, one query row per thread; the running
-//                             max only moves when a row's max grows by more
-//                             than 2^8, and O is rescaled in TMEM then
-//   O   += P_i V_i            P written to shared memory as bf16 (K-major A),
-//                             V read in place as an MN-major B operand
-// Tiles come from a 3-stage ring filled by one producer warp: TMA for whole
+// Per 64-token tile i (w = i & 1):
+//   S_i   = Q K_i^T           M = 128 query rows, N = 64 tokens, K = 128 dims,
+//                             Q split into bf16 hi + lo held in TMEM (the
+//                             MMA's A operand, two MMAs per step), into TMEM
+//                             buffer S_w
+//   softmax                   warpgroup w (tiles alternate between two
+//                             warpgroups), one query row per thread; a row's
+//                             running max only moves when its max grows by
+//                             more than 2^8, and O_w is rescaled in TMEM then
+//   O_w  += P_i V_i           P written as bf16 over the first half of S_w (A
+//                             operand from TMEM), V read in place from shared
+//                             memory as an MN-major B operand
+// Each warpgroup keeps its own (max, sum, O_w) and writes its own partial, so
+// a work unit yields two partials that the merge combines like splits.
+// Tiles come from a 6-stage ring filled by one producer warp: TMA for whole
 // cache tiles of a paged pool, cp.async for contiguous caches, plain loads for
 // the tile holding the sequence end and the new keys (and for pages that fail
 // the bounds check, which are zero-filled and reported).
 //
-// Warps 0-3: softmax + epilogue; warp 4: producer; warp 5: TMEM owner and MMA
-// issuer (lane 0).  Every wait is time-limited (SP_DEV_TIMEOUT).
+// Warps 0-3 and 4-7: the two softmax warpgroups (+ epilogue); warp 8:
+// producer; warp 9: TMEM owner and MMA issuer (lane 0).  Every wait is
+// time-limited (SP_DEV_TIMEOUT).
 #include <cudaTypedefs.h>
 #include <string.h>
 
@@ -37,22 +43,27 @@ using namespace sm100;
 
 constexpr int DH = 128;
 constexpr int TT = 64;                         // tokens per tile
-constexpr int STG = 3;                         // K/V ring depth
-constexpr int DEFER = STG - 2;                 // cp.async tiles in flight beyond the current
-constexpr int QSUB = 128 * 64 * 2;             // one [128 rows][64] bf16 swizzled sub-tile
-constexpr int KVSUB = TT * 64 * 2;             // one [64 tokens][64] sub-tile
+constexpr int STG = 6;                         // K/V ring depth
+// cp.async tiles in flight beyond the current one.  Tile j is published at
+// producer iteration j + DEFER, which first waits for stage j + DEFER - STG to
+// be released; the MMA warp needs tiles 0 and 1 before its first PV and tile
+// i + 2 before it releases stage i + 1, so DEFER <= STG - 2 (else deadlock).
+constexpr int DEFER = STG - 2;
+static_assert(DEFER >= 0 && DEFER <= STG - 2, "cp.async publication depth");
+constexpr int KVSUB = TT * 64 * 2;             // one [64 tokens][64] swizzled sub-tile
 constexpr int KV_STAGE = 4 * KVSUB;            // K (2 subs) + V (2 subs)
-constexpr int OFF_QHI = 0;
-constexpr int OFF_QLO = OFF_QHI + 2 * QSUB;
-constexpr int OFF_KV = OFF_QLO + 2 * QSUB;
-constexpr int OFF_P = OFF_KV + STG * KV_STAGE;
+constexpr int OFF_KV = 0;
 constexpr int MAX_SPLIT_PAGES = 1024;          // page ids of one split staged in smem
-constexpr int OFF_PAGES = OFF_P + 2 * QSUB;
+constexpr int OFF_PAGES = OFF_KV + STG * KV_STAGE;
 constexpr int OFF_BAR = OFF_PAGES + MAX_SPLIT_PAGES * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
-constexpr int THREADS = 192;
+constexpr int THREADS = 320;                   // 2 softmax warpgroups, producer, MMA
+constexpr int PRODUCER_WARP = 8, MMA_WARP = 9;
 constexpr float RESCALE_LOG2 = 8.f;            // tolerate p <= 2^8 before rescaling O
-constexpr uint32_t TMEM_COLS = 256;            // S0 [0,64), S1 [64,128), O [128,256)
+// TMEM columns: S0 [0,64) S1 [64,128) O0 [128,256) O1 [256,384) Qhi [384,448) Qlo [448,512);
+// P_w (64 bf16 per row) overwrites the first 32 columns of S_w once S_w is read.
+constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t O_COL = 128, QHI_COL = 384, QLO_COL = 448;
 
 // byte offset of 16-byte chunk `ch` (0..7) of row `row` in a swizzled sub-tile
 __device__ __forceinline__ uint32_t swz(int row, int ch) {
@@ -111,60 +122,66 @@ __global__ void __launch_bounds__(THREADS, 1)
             prefetch_tmap(&map_v);
         }
     }
-    if (warp == 5) {
+    if (warp == MMA_WARP) {
         tmem_alloc(&bars->tmem, TMEM_COLS);
         tmem_relinquish();
     }
-    // Q -> bf16 hi/lo, scaled to log2 units, rows rr = hl*k + r, zero past R
-    if (warp < 4) {
-        for (int idx = threadIdx.x; idx < 128 * 16; idx += 128) {
-            const int row = idx >> 4, c16 = idx & 15;
-            const int sub = c16 >> 3, ch = c16 & 7;
-            uint32_t hi[4] = {0, 0, 0, 0}, lo[4] = {0, 0, 0, 0};
-            if (row < R) {
-                const int hl = row / k, r = row - hl * k;
-                const float4 *src = (const float4 *)(a.q + (((size_t)b * k + r) * a.Hq +
-                                                             g * a.G + hl) * DH + c16 * 8);
-                const float4 x0 = src[0], x1 = src[1];
-                const float v[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-                float h[8], l8[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float x = v[e] * a.scale_log2;
-                    h[e] = __bfloat162float(__float2bfloat16_rn(x));
-                    l8[e] = x - h[e];
-                }
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    hi[e] = pack_bf16(h[2 * e], h[2 * e + 1]);
-                    lo[e] = pack_bf16(l8[2 * e], l8[2 * e + 1]);
-                }
-            }
-            st_shared_v4(smem + OFF_QHI + sub * QSUB + swz(row, ch), hi[0], hi[1], hi[2], hi[3]);
-            st_shared_v4(smem + OFF_QLO + sub * QSUB + swz(row, ch), lo[0], lo[1], lo[2], lo[3]);
-        }
-        fence_proxy_async();
+    // the producer stages this split's page ids while warpgroup 0 writes Q
+    const int P = a.kv.page_size;
+    const int *ptab = paged ? a.kv.page_table + (size_t)max(sq.sid, 0) * a.kv.max_pages : nullptr;
+    int *spages = (int *)(smem + OFF_PAGES);
+    const int lp0 = paged ? t_begin / P : 0;
+    const int n_lp = paged ? min(MAX_SPLIT_PAGES, max(0, ceil_div(min(t_end, L) - t_begin, P))) : 0;
+    if (warp == PRODUCER_WARP) {
+        for (int j = lane; j < n_lp; j += 32)
+            spages[j] = (lp0 + j < a.kv.max_pages) ? ptab[lp0 + j] : -1;
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = bars->tmem;
+    // Q -> bf16 hi/lo in TMEM (row rr = hl*k + r on lane rr; zero past R),
+    // scaled to log2 units: 64 columns of packed pairs for hi, 64 for lo
+    if (warp < 4) {
+        const int row = threadIdx.x;
+        const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+        const float4 *src = nullptr;
+        if (row < R) {
+            const int hl = row / k, r = row - hl * k;
+            src = (const float4 *)(a.q + (((size_t)b * k + r) * a.Hq + g * a.G + hl) * DH);
+        }
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            uint32_t hi[32], lo[32];
+#pragma unroll
+            for (int c4 = 0; c4 < 16; ++c4) {
+                const float4 x = src ? src[half * 16 + c4] : make_float4(0.f, 0.f, 0.f, 0.f);
+                const float v[4] = {x.x * a.scale_log2, x.y * a.scale_log2, x.z * a.scale_log2,
+                                    x.w * a.scale_log2};
+                float h[4], l4[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    h[e] = __bfloat162float(__float2bfloat16_rn(v[e]));
+                    l4[e] = v[e] - h[e];
+                }
+                hi[2 * c4] = pack_bf16(h[0], h[1]);
+                hi[2 * c4 + 1] = pack_bf16(h[2], h[3]);
+                lo[2 * c4] = pack_bf16(l4[0], l4[1]);
+                lo[2 * c4 + 1] = pack_bf16(l4[2], l4[3]);
+            }
+            tmem_st32u(lane_base + QHI_COL + half * 32, hi);
+            tmem_st32u(lane_base + QLO_COL + half * 32, lo);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
 
-    if (warp == 4) {
+    if (warp == PRODUCER_WARP) {
         // ------------------------------------------------------------ producer
         int issued = 0;
         bool deferred[STG] = {false, false, false};  // contiguous tiles awaiting cp.async
         int bad = 0;
-        const int P = a.kv.page_size;
-        const int *ptab = paged ? a.kv.page_table + (size_t)max(sq.sid, 0) * a.kv.max_pages : nullptr;
-        // this split's page ids, read once (coalesced) into shared memory;
-        // entries past the page-table row read as -1
-        int *spages = (int *)(smem + OFF_PAGES);
-        const int lp0 = paged ? t_begin / P : 0;
-        const int n_lp = paged ? min(MAX_SPLIT_PAGES, ceil_div(min(t_end, L) - t_begin, P)) : 0;
-        for (int j = lane; j < n_lp; j += 32)
-            spages[j] = (lp0 + j < a.kv.max_pages) ? ptab[lp0 + j] : -1;
-        __syncwarp();
         for (int i = 0; i < n_tiles; ++i) {
             const int st = i % STG;
             if (!mbar_wait(&bars->kv_empty[st], ((i / STG) & 1) ^ 1, abort)) break;
@@ -185,20 +202,19 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
                 pure = __all_sync(0xffffffffu, ok);
                 if (pure) {
-                    if (lane == 0) {
-                        mbar_arrive_expect_tx(&bars->kv_full[st], KV_STAGE);
-                        for (int j = 0; j < npg; ++j) {
-                            const int page = jl + j < n_lp ? spages[jl + j] : ptab[t0 / P + j];
-                            const int row = (page * a.Hkv + g) * P;
-                            const uint32_t off = (uint32_t)(j * P * 128);
-                            tma_load_2d(K + off, &map_k, &bars->kv_full[st], 0, row);
-                            tma_load_2d(K + KVSUB + off, &map_k, &bars->kv_full[st], 64, row);
-                            tma_load_2d(V + off, &map_v, &bars->kv_full[st], 0, row);
-                            tma_load_2d(V + KVSUB + off, &map_v, &bars->kv_full[st], 64, row);
-                        }
-                    } else {
-                        mbar_arrive(&bars->kv_full[st]);
+                    // one TMA box per lane: lane = 4 * page + (K lo, K hi, V lo, V hi);
+                    // lane 0 registers the stage's bytes before any box is issued
+                    if (lane == 0) mbar_arrive_expect_tx(&bars->kv_full[st], KV_STAGE);
+                    __syncwarp();
+                    if (lane < 4 * npg) {
+                        const int j = lane >> 2, part = lane & 3;
+                        const int page = jl + j < n_lp ? spages[jl + j] : ptab[t0 / P + j];
+                        const int row = (page * a.Hkv + g) * P;
+                        const uint32_t off = (uint32_t)(j * P * 128) + (part & 1) * KVSUB;
+                        tma_load_2d((part < 2 ? K : V) + off, part < 2 ? &map_k : &map_v,
+                                    &bars->kv_full[st], (part & 1) * 64, row);
                     }
+                    if (lane != 0) mbar_arrive(&bars->kv_full[st]);
                 }
             } else if (pure) {
                 // contiguous: token-major rows of 256 B, 16-byte cp.async per chunk
@@ -261,10 +277,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             cp_async_commit();  // one (possibly empty) group per tile
             issued = i + 1;
-            // A contiguous tile is published once its copies have landed, DEFER
-            // tiles later.  The MMA warp frees tile i-STG only after tile
-            // i-STG+1 is published, and this loop waits for that before issuing
-            // tile i+1, so DEFER must stay below STG - 1.
+            // a contiguous tile is published once its copies have landed, DEFER
+            // tiles later (see DEFER)
             cp_async_wait<DEFER>();
             const int j = i - DEFER;
             if (j >= 0 && deferred[j % STG]) {
@@ -288,12 +302,15 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         bad = __any_sync(0xffffffffu, bad);
         if (bad && lane == 0 && a.status) atomicOr(a.status, SP_DEV_BAD_PAGE);
-    } else if (warp == 5) {
+    } else if (warp == MMA_WARP) {
         // ------------------------------------------------------------ MMA issuer
+        // Order on the tensor pipe: S_0, S_1, then per tile i: PV_i (after
+        // softmax i) and S_{i+2} (reusing S buffer i & 1).  PV_i does not wait
+        // for any later tile's data, so stage i is released as soon as its
+        // softmax is done.
         if (lane == 0) {
             constexpr uint32_t idesc_s = idesc_bf16_f32(128, TT);
             constexpr uint32_t idesc_o = idesc_bf16_f32_bmn(128, DH);
-            const uint32_t o_tmem = tmem + 128;
             auto issue_s = [&](int i) {
                 const uint8_t *K = smem + OFF_KV + (i % STG) * KV_STAGE;
                 const uint32_t s_tmem = tmem + (uint32_t)((i & 1) * TT);
@@ -302,53 +319,59 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const int sub = kk >> 2;
                     const uint32_t off = (uint32_t)((kk & 3) * 2);  // 32 B steps along dh
                     const uint64_t bk = sw128_kmajor_desc(K + sub * KVSUB) + off;
-                    mma_bf16(s_tmem, sw128_kmajor_desc(smem + OFF_QHI + sub * QSUB) + off, bk,
-                             idesc_s, kk > 0 ? 1u : 0u);
-                    mma_bf16(s_tmem, sw128_kmajor_desc(smem + OFF_QLO + sub * QSUB) + off, bk,
-                             idesc_s, 1u);
+                    // 16 dims of Q = 8 TMEM columns
+                    mma_bf16_ts(s_tmem, tmem + QHI_COL + (uint32_t)(kk * 8), bk, idesc_s,
+                                kk > 0 ? 1u : 0u);
+                    mma_bf16_ts(s_tmem, tmem + QLO_COL + (uint32_t)(kk * 8), bk, idesc_s, 1u);
                 }
                 mma_commit(&bars->s_full[i & 1]);
             };
-            bool ok = mbar_wait(&bars->kv_full[0], 0, abort);
-            if (ok) {
-                tc_fence_after();
-                issue_s(0);
+            bool ok = true;
+            for (int i = 0; ok && i < 2 && i < n_tiles; ++i) {
+                ok = mbar_wait(&bars->kv_full[i % STG], (i / STG) & 1, abort);
+                if (ok) {
+                    tc_fence_after();
+                    issue_s(i);
+                }
             }
             for (int i = 0; ok && i < n_tiles; ++i) {
-                if (i + 1 < n_tiles) {
-                    ok = mbar_wait(&bars->kv_full[(i + 1) % STG], ((i + 1) / STG) & 1, abort);
-                    // S buffer (i+1)&1 was last read by the softmax of tile i-1
-                    if (ok && i >= 1) ok = mbar_wait(&bars->p_full[(i + 1) & 1], ((i - 1) >> 1) & 1, abort);
-                    if (!ok) break;
-                    tc_fence_after();
-                    issue_s(i + 1);
-                }
                 if (!mbar_wait(&bars->p_full[i & 1], (i >> 1) & 1, abort)) break;
                 tc_fence_after();
                 const uint8_t *V = smem + OFF_KV + (i % STG) * KV_STAGE + 2 * KVSUB;
-                const uint8_t *Pt = smem + OFF_P + (i & 1) * QSUB;
+                const uint32_t p_tmem = tmem + (uint32_t)((i & 1) * TT);  // P_i over S_i
+                const uint32_t o_tmem = tmem + O_COL + (uint32_t)((i & 1) * DH);
 #pragma unroll
                 for (int kk = 0; kk < TT / 16; ++kk) {
-                    mma_bf16(o_tmem, sw128_kmajor_desc(Pt) + (uint32_t)(kk * 2),
-                             sw128_mnmajor_desc(V + kk * 2048, KVSUB), idesc_o,
-                             (i > 0 || kk > 0) ? 1u : 0u);
+                    // 16 tokens of P = 8 TMEM columns; 16 token rows of V = 2 KB
+                    mma_bf16_ts(o_tmem, p_tmem + (uint32_t)(kk * 8),
+                                sw128_mnmajor_desc(V + kk * 2048, KVSUB), idesc_o,
+                                (i >= 2 || kk > 0) ? 1u : 0u);
                 }
                 mma_commit(&bars->kv_empty[i % STG]);
                 mma_commit(&bars->pv_done[i & 1]);
+                if (i + 2 < n_tiles) {
+                    // S buffer i & 1 is free: softmax i has read it (p_full above)
+                    if (!mbar_wait(&bars->kv_full[(i + 2) % STG], ((i + 2) / STG) & 1, abort)) break;
+                    tc_fence_after();
+                    issue_s(i + 2);
+                }
             }
             mma_commit(&bars->fin);  // completes when every MMA above is done
         }
         __syncwarp();
-    } else if (warp < act_warps) {
+    } else if ((warp & 3) < act_warps) {
         // ------------------------------------------------------------ softmax
-        const int row = threadIdx.x;  // == TMEM lane
+        const int wg = warp >> 2;       // warpgroup: tiles i with (i & 1) == wg
+        const int row = threadIdx.x & 127;  // == TMEM lane
         const bool active = row < R;
         const int r_soft = row % k;
-        const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+        const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+        const uint32_t s_col = (uint32_t)(wg * TT), o_col = O_COL + (uint32_t)(wg * DH);
         float m = -INFINITY, l = 0.f;
         bool ok = true;
-        for (int i = 0; i < n_tiles; ++i) {
-            if (!mbar_wait(&bars->s_full[i & 1], (i >> 1) & 1, abort)) {
+        for (int i = wg; i < n_tiles; i += 2) {
+            const uint32_t ph = (i >> 1) & 1;
+            if (!mbar_wait(&bars->s_full[wg], ph, abort)) {
                 ok = false;
                 break;
             }
@@ -356,10 +379,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             float sv[TT];
             {
                 float t32[32];
-                tmem_ld32(lane_base + (uint32_t)((i & 1) * TT), t32);
+                tmem_ld32(lane_base + s_col, t32);
 #pragma unroll
                 for (int j = 0; j < 32; ++j) sv[j] = t32[j];
-                tmem_ld32(lane_base + (uint32_t)((i & 1) * TT + 32), t32);
+                tmem_ld32(lane_base + s_col + 32, t32);
 #pragma unroll
                 for (int j = 0; j < 32; ++j) sv[32 + j] = t32[j];
             }
@@ -370,64 +393,71 @@ __global__ void __launch_bounds__(THREADS, 1)
                 for (int j = 0; j < TT; ++j)
                     if (t0 + j >= lim) sv[j] = -INFINITY;
             }
-            float mt = -INFINITY;
+            // tile max as an 8-way tree
+            float mx[8];
 #pragma unroll
-            for (int j = 0; j < TT; ++j) mt = fmaxf(mt, sv[j]);
-            if (!active) mt = -INFINITY;
-            const bool grow = mt > m + RESCALE_LOG2 || (m == -INFINITY && mt != -INFINITY);
+            for (int e = 0; e < 8; ++e) mx[e] = fmaxf(sv[e], sv[e + 8]);
+#pragma unroll
+            for (int j = 16; j < TT; j += 8)
+#pragma unroll
+                for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], sv[j + e]);
+            const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                   fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+            const bool grow = active && (mt > m + RESCALE_LOG2 || (m == -INFINITY && mt != -INFINITY));
             const float m_new = grow ? mt : m;
-            const float alpha = (grow && m != -INFINITY) ? exp2f(m - m_new) : (grow ? 0.f : 1.f);
-            if (i > 0 && __any_sync(0xffffffffu, grow)) {
-                // O holds tiles < i: wait for PV_{i-1}, then rescale the rows that moved
-                if (!mbar_wait(&bars->pv_done[(i - 1) & 1], ((i - 1) >> 1) & 1, abort)) {
+            const float alpha = grow ? (m == -INFINITY ? 0.f : fast_exp2(m - m_new)) : 1.f;
+            // O_wg and P_wg were last used by PV_{i-2}
+            if (i >= 2) {
+                if (!mbar_wait(&bars->pv_done[wg], ((i - 2) >> 1) & 1, abort)) {
                     ok = false;
                     break;
                 }
-                tc_fence_after();
+                if (__any_sync(0xffffffffu, grow)) {
+                    tc_fence_after();
 #pragma unroll 1
-                for (int c0 = 0; c0 < DH; c0 += 32) {
-                    float o32[32];
-                    tmem_ld32(lane_base + 128 + c0, o32);
+                    for (int c0 = 0; c0 < DH; c0 += 32) {
+                        float o32[32];
+                        tmem_ld32(lane_base + o_col + c0, o32);
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) o32[j] *= alpha;
-                    tmem_st32(lane_base + 128 + c0, o32);
+                        for (int j = 0; j < 32; ++j) o32[j] *= alpha;
+                        tmem_st32(lane_base + o_col + c0, o32);
+                    }
                 }
             }
             l *= alpha;
             m = m_new;
-            float p[TT];
-            float psum = 0.f;
+            const float mu = (m == -INFINITY) ? 0.f : m;  // a fully masked row gives p = 0
+            float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            uint32_t pk[TT / 2];
 #pragma unroll
-            for (int j = 0; j < TT; ++j) {
-                p[j] = (active && sv[j] != -INFINITY) ? exp2f(sv[j] - m) : 0.f;
-                psum += p[j];
+            for (int j = 0; j < TT; j += 2) {
+                const float p0 = fast_exp2(sv[j] - mu);
+                const float p1 = fast_exp2(sv[j + 1] - mu);
+                ps[(j >> 1) & 7] += p0 + p1;
+                pk[j >> 1] = pack_bf16(p0, p1);
             }
-            l += psum;
-            // P buffer i&1 was last read by PV_{i-2}
-            if (i >= 2 && !mbar_wait(&bars->pv_done[i & 1], ((i - 2) >> 1) & 1, abort)) {
-                ok = false;
-                break;
-            }
-            uint8_t *Pt = smem + OFF_P + (i & 1) * QSUB;
-#pragma unroll
-            for (int ch = 0; ch < 8; ++ch)
-                st_shared_v4(Pt + swz(row, ch), pack_bf16(p[8 * ch], p[8 * ch + 1]),
-                             pack_bf16(p[8 * ch + 2], p[8 * ch + 3]),
-                             pack_bf16(p[8 * ch + 4], p[8 * ch + 5]),
-                             pack_bf16(p[8 * ch + 6], p[8 * ch + 7]));
-            fence_proxy_async();
+            l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+            tmem_st32u(lane_base + s_col, pk);  // P_i over the first half of S_i
             tc_fence_before();
-            mbar_arrive(&bars->p_full[i & 1]);
+            mbar_arrive(&bars->p_full[wg]);
         }
-        // epilogue: the unnormalised partial of this unit
-        if (ok && mbar_wait(&bars->pv_done[(n_tiles - 1) & 1], ((n_tiles - 1) >> 1) & 1, abort)) {
+        // epilogue: this warpgroup's unnormalised partial of the unit
+        const int my_last = (n_tiles - 1 - wg) >= 0 ? n_tiles - 1 - ((n_tiles - 1 - wg) & 1) : -1;
+        const size_t unit = (((size_t)b * a.Hkv + g) * a.n_splits + s_idx) * 2 + wg;
+        float *po = a.part_o + (unit * R + row) * DH;
+        if (my_last < 0) {
+            // no tile for this warpgroup: an empty partial
+            if (active) {
+                for (int c = 0; c < DH; c += 4) *(float4 *)(po + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+                a.part_ml[(unit * R + row) * 2] = -INFINITY;
+                a.part_ml[(unit * R + row) * 2 + 1] = 0.f;
+            }
+        } else if (ok && mbar_wait(&bars->pv_done[wg], (my_last >> 1) & 1, abort)) {
             tc_fence_after();
-            const size_t unit = ((size_t)b * a.Hkv + g) * a.n_splits + s_idx;
-            float *po = a.part_o + (unit * R + row) * DH;
 #pragma unroll 1
             for (int c0 = 0; c0 < DH; c0 += 32) {
                 float o32[32];
-                tmem_ld32(lane_base + 128 + c0, o32);
+                tmem_ld32(lane_base + o_col + c0, o32);
                 if (active) {
 #pragma unroll
                     for (int j = 0; j < 32; j += 4)
@@ -445,7 +475,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     tc_fence_before();
     __syncthreads();
     if (threadIdx.x == 0 && *abort && a.status) atomicOr(a.status, SP_DEV_TIMEOUT);
-    if (warp == 5) tmem_dealloc(tmem, TMEM_COLS);
+    if (warp == MMA_WARP) tmem_dealloc(tmem, TMEM_COLS);
 }
 
 }  // namespace

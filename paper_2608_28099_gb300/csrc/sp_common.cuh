@@ -112,8 +112,9 @@ struct AttnArgs {
     const float *q;               // [B][k][Hq][dh], rotated
     const float *k_new;           // [B][k][Hkv][dh], rotated
     const float *v_new;           // [B][k][Hkv][dh]
-    float *part_o;                // [B][Hkv][n_splits][R][dh], unnormalised
-    float *part_ml;               // [B][Hkv][n_splits][R][2] (running max in log2 units, sum)
+    int subs;                     // partials per work unit (1 CUDA-core, 2 tensor-core)
+    float *part_o;                // [B][Hkv][n_splits][subs][R][dh], unnormalised
+    float *part_ml;               // [B][Hkv][n_splits][subs][R][2] (max in log2 units, sum)
     int *status;
     int *gathered;                // [B][max_pages] or NULL
     float scale_log2;             // log2(e) / sqrt(dh)
