@@ -205,13 +205,15 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
         pk = &mk;
         pv = &mv;
     }
+    CUtensorMap mq;
+    if (tc) tc = encode_q_group_f32(&mq, a.q, a.B * a.k, a.Hq, a.G, a.k);
     if (attn_path == 2 && !tc)
         return fail(SP_ERR_UNSUPPORTED, "tensor-core attention needs head_dim 128, a bf16 cache "
                                         "and at most 128 query rows per kv head");
     a.subs = tc ? 2 : 1;
     if (ev_attn) cudaEventRecordWithFlags(ev_attn[0], st, cudaEventRecordExternal);
     if (tc)
-        SP_CUDA(launch_attention_tc(a, pk, pv, st));
+        SP_CUDA(launch_attention_tc(a, pk, pv, mq, st));
     else
         SP_CUDA(launch_attention_simt(a, st));
     if (ev_attn) cudaEventRecordWithFlags(ev_attn[1], st, cudaEventRecordExternal);

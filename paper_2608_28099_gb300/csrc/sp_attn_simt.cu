@@ -222,24 +222,28 @@ cudaError_t launch_simt_t(const AttnArgs &a, cudaStream_t st) {
 void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, int n_sm,
                     int *split_tokens, int *n_splits) {
     const int total = max_seq_len + k;
+    const int tiles = (total + 63) / 64;
     int chunk;
     if (forced_split > 0) {
         chunk = forced_split;
     } else {
-        // Aim for about four waves of one-CTA-per-SM work units over the
-        // longest sequence, with splits long enough to amortise a unit's
-        // start-up (>= 512 tokens unless the sequence is shorter) and short
-        // enough that one split's page ids fit in shared memory (<= 16384).
+        // Choose the number of splits s of the longest sequence that minimises
+        // waves(s) * (tiles per unit + start-up), for one work unit per SM at a
+        // time: waves = ceil(B * Hkv * s / n_sm), start-up ~ 6 tiles of work.
+        // Splits stay <= 16384 tokens (one split's page ids fit in shared memory).
         const long long units = (long long)B * Hkv;
-        const long long want = 4LL * n_sm;
-        long long s = (want + units - 1) / units;
-        if (s < 1) s = 1;
-        chunk = (int)((total + s - 1) / s);
-        chunk = ((chunk + 63) / 64) * 64;
-        if (chunk < 512) chunk = 512;
-        if (chunk > 16384) chunk = 16384;
-        const int whole = ((total + 63) / 64) * 64;
-        if (chunk > whole) chunk = whole;
+        const int s_min = (tiles + 255) / 256;
+        long long best_cost = -1;
+        int best_s = s_min;
+        for (int s = s_min; s <= tiles && s <= 64; ++s) {
+            const long long waves = (units * s + n_sm - 1) / n_sm;
+            const long long cost = waves * ((tiles + s - 1) / s + 6);
+            if (best_cost < 0 || cost < best_cost) {
+                best_cost = cost;
+                best_s = s;
+            }
+        }
+        chunk = ((tiles + best_s - 1) / best_s) * 64;
     }
     *split_tokens = chunk;
     *n_splits = ceil_div(total, chunk);

@@ -76,14 +76,15 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 }
 
 struct Bars {
-    uint64_t kv_full[STG], kv_empty[STG], s_full[2], p_full[2], pv_done[2], fin;
+    uint64_t kv_full[STG], kv_empty[STG], s_full[2], p_full[2], pv_done[2], fin, q_full;
     uint32_t tmem;
     int abort;
 };
 
 __global__ void __launch_bounds__(THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap map_k,
-                   const __grid_constant__ CUtensorMap map_v, AttnArgs a) {
+                   const __grid_constant__ CUtensorMap map_v,
+                   const __grid_constant__ CUtensorMap map_q, AttnArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     Bars *bars = (Bars *)(smem + OFF_BAR);
@@ -115,8 +116,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             mbar_init(&bars->pv_done[i], 1);
         }
         mbar_init(&bars->fin, 1);
+        mbar_init(&bars->q_full, 1);
         bars->abort = 0;
         fence_mbar_init();
+        prefetch_tmap(&map_q);
         if (paged) {
             prefetch_tmap(&map_k);
             prefetch_tmap(&map_v);
@@ -132,23 +135,31 @@ __global__ void __launch_bounds__(THREADS, 1)
     int *spages = (int *)(smem + OFF_PAGES);
     const int lp0 = paged ? t_begin / P : 0;
     const int n_lp = paged ? min(MAX_SPLIT_PAGES, max(0, ceil_div(min(t_end, L) - t_begin, P))) : 0;
-    if (warp == PRODUCER_WARP) {
-        for (int j = lane; j < n_lp; j += 32)
-            spages[j] = (lp0 + j < a.kv.max_pages) ? ptab[lp0 + j] : -1;
-    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = bars->tmem;
+    // one TMA brings this group's queries [k][G][128] fp32 into the first ring
+    // stages (free until the pipeline starts)
+    float *qs = (float *)(smem + OFF_KV);
+    if (warp == PRODUCER_WARP) {
+        if (lane == 0) {
+            mbar_arrive_expect_tx(&bars->q_full, (uint32_t)(R * DH * 4));
+            tma_load_3d(qs, &map_q, &bars->q_full, 0, g * a.G, b * k);
+        }
+        for (int j = lane; j < n_lp; j += 32)
+            spages[j] = (lp0 + j < a.kv.max_pages) ? ptab[lp0 + j] : -1;
+    }
     // Q -> bf16 hi/lo in TMEM (row rr = hl*k + r on lane rr; zero past R),
     // scaled to log2 units: 64 columns of packed pairs for hi, 64 for lo
     if (warp < 4) {
         const int row = threadIdx.x;
         const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
+        const bool have_q = mbar_wait_drain(&bars->q_full, 0);
         const float4 *src = nullptr;
-        if (row < R) {
+        if (row < R && have_q) {
             const int hl = row / k, r = row - hl * k;
-            src = (const float4 *)(a.q + (((size_t)b * k + r) * a.Hq + g * a.G + hl) * DH);
+            src = (const float4 *)(qs + (r * a.G + hl) * DH);
         }
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
@@ -487,7 +498,8 @@ bool attention_tc_supported(const AttnArgs &a) {
 }
 
 cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
-                                const CUtensorMap *map_v, cudaStream_t st) {
+                                const CUtensorMap *map_v, const CUtensorMap &map_q,
+                                cudaStream_t st) {
     static bool attr = false;
     if (!attr) {
         cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel,
@@ -499,7 +511,7 @@ cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
     memset(&dummy, 0, sizeof dummy);
     dim3 grid(a.n_splits, a.Hkv, a.B);
     attn_tc_kernel<<<grid, THREADS, SMEM_BYTES, st>>>(map_k ? *map_k : dummy,
-                                                      map_v ? *map_v : dummy, a);
+                                                      map_v ? *map_v : dummy, map_q, a);
     return cudaGetLastError();
 }
 

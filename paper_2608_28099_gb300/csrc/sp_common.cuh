@@ -130,7 +130,8 @@ cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st);
 // maps of the K and V pools viewed as [n_pages * Hkv * page_size][128].
 bool attention_tc_supported(const AttnArgs &a);
 cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
-                                const CUtensorMap *map_v, cudaStream_t st);
+                                const CUtensorMap *map_v, const CUtensorMap &map_q,
+                                cudaStream_t st);
 cudaError_t launch_attention_merge(const AttnArgs &a, cudaStream_t st);
 
 // ---------------------------------------------------------------------------

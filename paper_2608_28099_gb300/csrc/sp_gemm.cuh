@@ -15,6 +15,8 @@ struct TcPlan {
 };
 
 bool encode_kmajor_bf16(CUtensorMap *map, const void *base, int rows, int K, int box_rows);
+// TMA map of rotated queries [rows][Hq][128] fp32 by (k rows x G heads) boxes.
+bool encode_q_group_f32(CUtensorMap *map, const float *q, int rows, int Hq, int G, int k);
 bool tc_supported(int N, int K);
 int tc_bn_for(int M);
 TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes);

@@ -216,6 +216,21 @@ bool encode_kmajor_bf16(CUtensorMap *map, const void *base, int rows, int K, int
     return r == CUDA_SUCCESS;
 }
 
+bool encode_q_group_f32(CUtensorMap *map, const float *q, int rows, int Hq, int G, int k) {
+    // q [rows = B*k][Hq][128] fp32; one box = the G heads of one kv group for
+    // the k rows of one sequence: [k][G][128], unswizzled
+    PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+    if (!fn || ((uintptr_t)q & 15) || G > 256 || k > 256) return false;
+    cuuint64_t dims[3] = {128, (cuuint64_t)Hq, (cuuint64_t)rows};
+    cuuint64_t strides[2] = {128 * 4, (cuuint64_t)Hq * 128 * 4};
+    cuuint32_t box[3] = {128, (cuuint32_t)G, (cuuint32_t)k};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<float *>(q), dims, strides,
+                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 int tc_bn_for(int M) {
     if (M <= 16) return 16;
     if (M <= 32) return 32;
