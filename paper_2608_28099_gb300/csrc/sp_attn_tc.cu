@@ -103,11 +103,16 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int t_end = min(total, t_begin + a.split_tokens);
     const int n_tiles = (t_end - t_begin + TT - 1) / TT;
     const int act_warps = (R + 31) / 32;  // softmax warps that own real query rows
+    // producers: warp 8, plus the softmax warps that own no rows (they help
+    // with the cp.async and plain-load tiles; only warp 8 issues TMA)
+    const int n_prod = 1 + 2 * (4 - act_warps);
+    const bool is_producer = warp == PRODUCER_WARP || (warp < 8 && (warp & 3) >= act_warps);
+    const int pidx = warp == PRODUCER_WARP ? 0 : 1 + (warp >> 2) * (4 - act_warps) + ((warp & 3) - act_warps);
     const bool paged = a.kv.layout == SP_KV_PAGED;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STG; ++i) {
-            mbar_init(&bars->kv_full[i], 32);
+            mbar_init(&bars->kv_full[i], 32 * n_prod);
             mbar_init(&bars->kv_empty[i], 1);
         }
         for (int i = 0; i < 2; ++i) {
@@ -188,8 +193,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
     tc_fence_after();
 
-    if (warp == PRODUCER_WARP) {
-        // ------------------------------------------------------------ producer
+    if (is_producer) {
+        // ------------------------------------------------------------ producers
+        const int ptid = pidx * 32 + lane, pstride = 32 * n_prod;
+        const bool lead = pidx == 0;  // warp 8: TMA issue and drain
         int issued = 0;
         bool deferred[STG] = {false, false, false};  // contiguous tiles awaiting cp.async
         int bad = 0;
@@ -211,8 +218,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                     ok = page >= 0 && page < a.kv.n_pages;
                     if (ok && a.gathered) a.gathered[(size_t)b * a.kv.max_pages + lp] = page;
                 }
-                pure = __all_sync(0xffffffffu, ok);
-                if (pure) {
+                pure = __all_sync(0xffffffffu, ok);  // every producer warp reaches the same verdict
+                if (pure && !lead) {
+                    mbar_arrive(&bars->kv_full[st]);
+                } else if (pure) {
                     // one TMA box per lane: lane = 4 * page + (K lo, K hi, V lo, V hi);
                     // lane 0 registers the stage's bytes before any box is issued
                     if (lane == 0) mbar_arrive_expect_tx(&bars->kv_full[st], KV_STAGE);
@@ -231,7 +240,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 // contiguous: token-major rows of 256 B, 16-byte cp.async per chunk
                 const bf16 *kb = (const bf16 *)a.kv.k_seq[sq.sid];
                 const bf16 *vb = (const bf16 *)a.kv.v_seq[sq.sid];
-                for (int idx = lane; idx < TT * 16; idx += 32) {
+                for (int idx = ptid; idx < TT * 16; idx += pstride) {
                     const int row = idx >> 4, c16 = idx & 15;
                     const size_t src = ((size_t)(t0 + row) * a.Hkv + g) * DH + c16 * 8;
                     const uint32_t dst = (c16 >> 3) * KVSUB + swz(row, c16 & 7);
@@ -242,7 +251,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             if (!pure) {
                 // the sequence end / new keys / a bad page: plain loads, zero fill
-                for (int idx = lane; idx < TT * 16; idx += 32) {
+                for (int idx = ptid; idx < TT * 16; idx += pstride) {
                     const int row = idx >> 4, c16 = idx & 15;
                     const int t = t0 + row;
                     const uint32_t dst = (c16 >> 3) * KVSUB + swz(row, c16 & 7);
@@ -306,7 +315,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 deferred[j % STG] = false;
             }
         }
-        if (lane == 0) {
+        if (lead && lane == 0) {
             // drain TMA writes still in flight (only possible after an abort)
             for (int j = issued > STG ? issued - STG : 0; j < issued; ++j)
                 mbar_wait_drain(&bars->kv_full[j % STG], (j / STG) & 1);
@@ -370,7 +379,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             mma_commit(&bars->fin);  // completes when every MMA above is done
         }
         __syncwarp();
-    } else if ((warp & 3) < act_warps) {
+    } else if (warp < 8 && (warp & 3) < act_warps) {
         // ------------------------------------------------------------ softmax
         const int wg = warp >> 2;       // warpgroup: tiles i with (i & 1) == wg
         const int row = threadIdx.x & 127;  // == TMEM lane
