@@ -155,7 +155,8 @@ SP_API sp_status sp_destroy(sp_handle *h);
  *   kv         the cache (see sp_kv_cache); kv_dtype must match the handle.
  *   d_rows     [batch][k][d] device, w_dtype: the per-sequence input rows of
  *              the layer (e.g. an MTP head's fused inputs), or NULL: every
- *              sequence uses the handle's shared soft prompt rows.
+ *              sequence uses the handle's shared soft prompt rows.  Must be
+ *              16-byte aligned (SP_ERR_INVALID_ARG otherwise).
  *   d_logits   [batch][C] float device, caller-owned: raw class logits.
  * 1 <= batch <= max_batch.  Device-side range problems are reported through
  * sp_check_status(). */

@@ -449,6 +449,8 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     if (s != SP_OK) return s;
     if (!d_seq_ids && batch > kv->n_seqs)
         return fail(SP_ERR_INVALID_ARG, "batch %d exceeds n_seqs %d with implicit ids", batch, kv->n_seqs);
+    if (d_rows && ((uintptr_t)d_rows & 15))
+        return fail(SP_ERR_INVALID_ARG, "d_rows must be 16-byte aligned");
 
     const int d = c.d_model, hq = c.n_q_heads, hkv = c.n_kv_heads, dh = c.head_dim, f = c.d_ff;
     const int k = c.k_rows, C = c.n_classes, G = hq / hkv;

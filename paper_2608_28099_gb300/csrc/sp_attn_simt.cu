@@ -54,6 +54,8 @@ __device__ __forceinline__ const T *cache_row(const KVDev &kv, const void *pool_
 
 template <typename TKV, int DH>
 __global__ void __launch_bounds__(kThreads) attn_split_simt(AttnArgs a) {
+    pdl_trigger();
+    pdl_wait();
     extern __shared__ float smem[];
     const int s = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
     const int R = a.R, k = a.k;
@@ -173,33 +175,50 @@ __global__ void __launch_bounds__(kThreads) attn_split_simt(AttnArgs a) {
     }
 }
 
-// Merge the split partials: block (kv head g, sequence b, row group) combines
-// up to 8 query rows; thread c handles output column c (head_dim threads).
-constexpr int kMergeRows = 8;
-
+// Merge the partials of one query row: block (kv head g, sequence b, row rr),
+// thread c = output column c (head_dim threads).  Each pass issues the loads
+// of up to eight partials before combining them.
 __global__ void attn_merge_kernel(AttnArgs a) {
-    const int g = blockIdx.x, b = blockIdx.y;
+    pdl_trigger();
+    pdl_wait();
+    const int g = blockIdx.x, b = blockIdx.y, rr = blockIdx.z;
     const int R = a.R, dh = a.dh, k = a.k;
     const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs,
                                   a.max_seq_len, nullptr);
     const int n_valid = min(a.n_splits, ceil_div(sq.len + k, a.split_tokens)) * a.subs;
     const size_t unit0 = ((size_t)b * a.Hkv + g) * a.n_splits * a.subs;
     const int c = threadIdx.x;
-    for (int rr = blockIdx.z * kMergeRows; rr < min(R, (blockIdx.z + 1) * kMergeRows); ++rr) {
-        float mmax = -INFINITY;
-        for (int s = 0; s < n_valid; ++s) mmax = fmaxf(mmax, a.part_ml[((unit0 + s) * R + rr) * 2]);
-        float l = 0.f, o = 0.f;
-        for (int s = 0; s < n_valid; ++s) {
-            const float ms = a.part_ml[((unit0 + s) * R + rr) * 2];
-            if (ms == -INFINITY) continue;
-            const float wgt = exp2f(ms - mmax);
-            l += a.part_ml[((unit0 + s) * R + rr) * 2 + 1] * wgt;
-            o += a.part_o[((unit0 + s) * R + rr) * dh + c] * wgt;
-        }
-        const int hl = rr / k, r = rr - hl * k;
-        const int h = g * a.G + hl;
-        act_store(a.out, (((size_t)b * k + r) * a.Hq + h) * dh + c, l > 0.f ? o / l : 0.f);
+    float mmax = -INFINITY;
+    for (int s0 = 0; s0 < n_valid; s0 += 8) {
+        float mv[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+            mv[j] = s0 + j < n_valid ? a.part_ml[((unit0 + s0 + j) * R + rr) * 2] : -INFINITY;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) mmax = fmaxf(mmax, mv[j]);
     }
+    float l = 0.f, o = 0.f;
+    for (int s0 = 0; s0 < n_valid; s0 += 8) {
+        float ms[8], ls[8], os[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const bool in = s0 + j < n_valid;
+            const size_t u = unit0 + s0 + j;
+            ms[j] = in ? a.part_ml[(u * R + rr) * 2] : -INFINITY;
+            ls[j] = in ? a.part_ml[(u * R + rr) * 2 + 1] : 0.f;
+            os[j] = in ? a.part_o[(u * R + rr) * dh + c] : 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            if (ms[j] == -INFINITY) continue;
+            const float wgt = exp2f(ms[j] - mmax);
+            l += ls[j] * wgt;
+            o += os[j] * wgt;
+        }
+    }
+    const int hl = rr / k, r = rr - hl * k;
+    const int h = g * a.G + hl;
+    act_store(a.out, (((size_t)b * k + r) * a.Hq + h) * dh + c, l > 0.f ? o / l : 0.f);
 }
 
 template <typename TKV, int DH>
@@ -213,8 +232,7 @@ cudaError_t launch_simt_t(const AttnArgs &a, cudaStream_t st) {
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     dim3 grid(a.n_splits, a.Hkv, a.B);
-    attn_split_simt<TKV, DH><<<grid, kThreads, smem, st>>>(a);
-    return cudaGetLastError();
+    return launch_k(attn_split_simt<TKV, DH>, grid, dim3(kThreads), smem, st, a);
 }
 
 }  // namespace
@@ -270,9 +288,8 @@ cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st) {
 }
 
 cudaError_t launch_attention_merge(const AttnArgs &a, cudaStream_t st) {
-    dim3 grid(a.Hkv, a.B, ceil_div(a.R, kMergeRows));
-    attn_merge_kernel<<<grid, a.dh, 0, st>>>(a);
-    return cudaGetLastError();
+    dim3 grid(a.Hkv, a.B, a.R);
+    return launch_k(attn_merge_kernel, grid, dim3(a.dh), 0, st, a);
 }
 
 }  // namespace sp

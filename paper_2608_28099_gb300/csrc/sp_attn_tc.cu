@@ -92,6 +92,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int s_idx = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int R = a.R, k = a.k;
+    pdl_trigger();
 
     const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs,
                                   a.max_seq_len,
@@ -140,6 +141,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     int *spages = (int *)(smem + OFF_PAGES);
     const int lp0 = paged ? t_begin / P : 0;
     const int n_lp = paged ? min(MAX_SPLIT_PAGES, max(0, ceil_div(min(t_end, L) - t_begin, P))) : 0;
+    pdl_wait();  // the rotated queries and new keys come from the previous kernel
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -519,9 +521,8 @@ cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
     CUtensorMap dummy;
     memset(&dummy, 0, sizeof dummy);
     dim3 grid(a.n_splits, a.Hkv, a.B);
-    attn_tc_kernel<<<grid, THREADS, SMEM_BYTES, st>>>(map_k ? *map_k : dummy,
-                                                      map_v ? *map_v : dummy, map_q, a);
-    return cudaGetLastError();
+    return launch_k(attn_tc_kernel, grid, dim3(THREADS), SMEM_BYTES, st, map_k ? *map_k : dummy,
+                    map_v ? *map_v : dummy, map_q, a);
 }
 
 }  // namespace sp

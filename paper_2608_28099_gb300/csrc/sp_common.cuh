@@ -21,6 +21,34 @@ template <typename T> __device__ __forceinline__ T from_f(float x);
 template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
 template <> __device__ __forceinline__ bf16 from_f<bf16>(float x) { return __float2bfloat16_rn(x); }
 
+// Programmatic dependent launch.  Every kernel of the path is launched with
+// programmatic stream serialisation (launch_k), so its CTAs may start -- and do
+// their independent set-up -- while the previous kernel on the stream drains.
+// pdl_wait() returns once the previous kernel has completed and its writes are
+// visible; every kernel calls it before touching data an earlier kernel
+// writes, and before writing scratch an earlier kernel may still read.
+// pdl_trigger() allows the next kernel to launch (it still waits in pdl_wait).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename Kern, typename... Args>
+inline cudaError_t launch_k(Kern kernel, dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                            Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = st ? 1 : 0;  // the legacy default stream keeps plain serialisation
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // Where a producer writes an activation: fp32 (f32 != null), plain bf16
 // (hi != null, lo == null) or the two-plane form hi = rn(v), lo = rn(v - hi)
 // that the tensor-core projections consume.
@@ -46,10 +74,72 @@ struct PartIn {
     int n;
     size_t stride;
 };
+// Loads of up to eight partials are issued together before they are added
+// (the adds would otherwise serialise one memory latency per partial).
 __device__ __forceinline__ float part_get(const PartIn &p, size_t idx) {
-    float s = p.y[idx];
-    for (int i = 1; i < p.n; ++i) s += p.y[(size_t)i * p.stride + idx];
+    float s = 0.f;
+    for (int i0 = 0; i0 < p.n; i0 += 8) {
+        float v[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[j] = (i0 + j < p.n) ? p.y[(size_t)(i0 + j) * p.stride + idx] : 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) s += v[j];
+    }
     return s;
+}
+// Four consecutive values (idx and stride multiples of 4).
+__device__ __forceinline__ float4 part_get4(const PartIn &p, size_t idx) {
+    float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int i0 = 0; i0 < p.n; i0 += 4) {
+        float4 v[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            v[j] = (i0 + j < p.n) ? *(const float4 *)(p.y + (size_t)(i0 + j) * p.stride + idx)
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            s.x += v[j].x;
+            s.y += v[j].y;
+            s.z += v[j].z;
+            s.w += v[j].w;
+        }
+    }
+    return s;
+}
+
+// Vector helpers for 8 consecutive elements (16-byte aligned bf16, 32-byte fp32).
+__device__ __forceinline__ void load8(const float *p, float (&v)[8]) {
+    const float4 a = *(const float4 *)p, b = *(const float4 *)(p + 4);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void load8(const bf16 *p, float (&v)[8]) {
+    const uint4 u = *(const uint4 *)p;
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        v[2 * i] = __uint_as_float(w[i] << 16);
+        v[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
+}
+__device__ __forceinline__ uint32_t pack2_bf16(float a, float b) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t *>(&h);
+}
+// act_store of 4 consecutive values (idx multiple of 4)
+__device__ __forceinline__ void act_store4(const ActOut &o, size_t idx, float4 v) {
+    if (o.f32) {
+        *(float4 *)(o.f32 + idx) = v;
+        return;
+    }
+    const float x[4] = {v.x, v.y, v.z, v.w};
+    float h[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) h[i] = __bfloat162float(__float2bfloat16_rn(x[i]));
+    *(uint2 *)(o.hi + idx) = make_uint2(pack2_bf16(h[0], h[1]), pack2_bf16(h[2], h[3]));
+    if (o.lo)
+        *(uint2 *)(o.lo + idx) = make_uint2(pack2_bf16(x[0] - h[0], x[1] - h[1]),
+                                            pack2_bf16(x[2] - h[2], x[3] - h[3]));
 }
 
 // Cache description as the kernels see it (same fields as sp_kv_cache).

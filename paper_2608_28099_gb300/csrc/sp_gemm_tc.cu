@@ -68,6 +68,7 @@ __global__ void __launch_bounds__(128, 1)
     const int m0 = blockIdx.x * BN, n0 = blockIdx.y * 128;
     const int kb0 = blockIdx.z * g.kb_per_split;
     const int nkb = min(g.kb_per_split, g.n_kb - kb0);
+    pdl_trigger();
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < Cfg::STAGES; ++s) {
@@ -92,20 +93,31 @@ __global__ void __launch_bounds__(128, 1)
 
     int issued = 0;
     if (warp == 0 && lane == 0) {
-        // producer: weights streamed once (evict-first), activations reused (evict-last)
+        // producer: weights streamed once (evict-first), activations reused (evict-last).
+        // The weights are constant, so the first ring of weight tiles is requested
+        // before waiting for the previous kernel; the activations it writes after.
         const uint64_t pol_w = policy_evict_first();
         const uint64_t pol_x = policy_evict_last();
+        const int pre = nkb < Cfg::STAGES ? nkb : Cfg::STAGES;
+        for (int i = 0; i < pre; ++i) {
+            mbar_arrive_expect_tx(&full[i], Cfg::STAGE);
+            tma_load_2d_hint(smem + i * Cfg::STAGE, &map_w, &full[i], (kb0 + i) * BK, n0, pol_w);
+        }
+        issued = pre;
+        pdl_wait();
         for (int i = 0; i < nkb; ++i) {
             const int s = i % Cfg::STAGES;
             const uint32_t ph = (i / Cfg::STAGES) & 1;
-            if (!mbar_wait(&empty[s], ph ^ 1, abort)) break;
             uint8_t *st = smem + s * Cfg::STAGE;
-            mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
             const int kc = (kb0 + i) * BK;
-            tma_load_2d_hint(st, &map_w, &full[s], kc, n0, pol_w);
+            if (i >= pre) {
+                if (!mbar_wait(&empty[s], ph ^ 1, abort)) break;
+                mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
+                tma_load_2d_hint(st, &map_w, &full[s], kc, n0, pol_w);
+                issued = i + 1;
+            }
             tma_load_2d_hint(st + A_BYTES, &map_xhi, &full[s], kc, m0, pol_x);
             tma_load_2d_hint(st + A_BYTES + Cfg::B_BYTES, &map_xlo, &full[s], kc, m0, pol_x);
-            issued = i + 1;
         }
     } else if (warp == 1 && lane == 0) {
         // MMA issuer
@@ -130,6 +142,7 @@ __global__ void __launch_bounds__(128, 1)
         mma_commit(done);  // completes once every MMA issued above has finished
     }
     __syncwarp();
+    pdl_wait();  // before writing partials a previous kernel may still be reading
 
     // epilogue: TMEM -> registers -> fp32 partial tile
     const bool have = mbar_wait_drain(done, 0) && !*abort;
@@ -181,8 +194,7 @@ cudaError_t launch_bn(const CUtensorMap &mw, const CUtensorMap &mh, const CUtens
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    gemm_tc_kernel<BN><<<grid, 128, smem, st>>>(mw, mh, ml, g);
-    return cudaGetLastError();
+    return launch_k(gemm_tc_kernel<BN>, grid, dim3(128), (size_t)smem, st, mw, mh, ml, g);
 }
 
 }  // namespace

@@ -27,26 +27,46 @@ __device__ __forceinline__ float block_sum(float v, float *red) {
     return warp_sum(t);
 }
 
+// One block per row, d % 8 == 0: 8-element vector loads, four chunks in
+// flight per thread.
 template <typename T>
-__global__ void rmsnorm_rows_kernel(const T *__restrict__ x, int row_mod,
-                                    const float *__restrict__ gain, float eps, int d, ActOut out) {
+__global__ void __launch_bounds__(256) rmsnorm_rows_kernel(const T *__restrict__ x, int row_mod,
+                                                           const float *__restrict__ gain, float eps,
+                                                           int d, ActOut out) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float red[32];
     const int m = blockIdx.x;
     const T *xr = x + (size_t)(row_mod ? m % row_mod : m) * d;
+    const int nch = d >> 3;
     float ss = 0.f;
-    for (int j = threadIdx.x; j < d; j += blockDim.x) {
-        float v = to_f(xr[j]);
-        ss += v * v;
+#pragma unroll 4
+    for (int c = threadIdx.x; c < nch; c += blockDim.x) {
+        float v[8];
+        load8(xr + c * 8, v);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) ss += v[e] * v[e];
     }
     ss = block_sum(ss, red);
     const float inv = rsqrtf(ss / (float)d + eps);
-    for (int j = threadIdx.x; j < d; j += blockDim.x)
-        act_store(out, (size_t)m * d + j, to_f(xr[j]) * inv * gain[j]);
+#pragma unroll 4
+    for (int c = threadIdx.x; c < nch; c += blockDim.x) {
+        float v[8], gv[8];
+        load8(xr + c * 8, v);
+        load8(gain + c * 8, gv);
+        const size_t o = (size_t)m * d + c * 8;
+        act_store4(out, o, make_float4(v[0] * inv * gv[0], v[1] * inv * gv[1], v[2] * inv * gv[2],
+                                       v[3] * inv * gv[3]));
+        act_store4(out, o + 4, make_float4(v[4] * inv * gv[4], v[5] * inv * gv[5],
+                                           v[6] * inv * gv[6], v[7] * inv * gv[7]));
+    }
 }
 
 // One thread per rotated pair (query heads, then key heads) or value element
 // of one row: grid (ceil(per_row / 256), B * k).
 __global__ void qkv_rope_kernel(QkvRopeArgs a) {
+    pdl_trigger();
+    pdl_wait();
     const int m = blockIdx.y;
     const int b = m / a.k, r = m % a.k;
     const int dh = a.dh, half = dh >> 1;
@@ -74,84 +94,121 @@ __global__ void qkv_rope_kernel(QkvRopeArgs a) {
     }
 }
 
+// h1 = x + y, n = RMSNorm(h1): one block per row, 4-element vectors.
 template <typename TX>
-__global__ void residual_norm_kernel(PartIn y, const TX *__restrict__ x, int row_mod,
-                                     const float *__restrict__ gain, float eps, int d,
-                                     float *__restrict__ h1, ActOut n) {
+__global__ void __launch_bounds__(1024) residual_norm_kernel(PartIn y, const TX *__restrict__ x,
+                                                             int row_mod,
+                                                             const float *__restrict__ gain,
+                                                             float eps, int d,
+                                                             float *__restrict__ h1, ActOut n) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float red[32];
     const int m = blockIdx.x;
     const TX *xr = x + (size_t)(row_mod ? m % row_mod : m) * d;
     float *hr = h1 + (size_t)m * d;
+    const int nch = d >> 2;
     float ss = 0.f;
-    for (int j = threadIdx.x; j < d; j += blockDim.x) {
-        float v = to_f(xr[j]) + part_get(y, (size_t)m * d + j);
-        hr[j] = v;
-        ss += v * v;
+#pragma unroll 2
+    for (int c = threadIdx.x; c < nch; c += blockDim.x) {
+        const float4 yv = part_get4(y, (size_t)m * d + c * 4);
+        float4 v = make_float4(to_f(xr[c * 4]) + yv.x, to_f(xr[c * 4 + 1]) + yv.y,
+                               to_f(xr[c * 4 + 2]) + yv.z, to_f(xr[c * 4 + 3]) + yv.w);
+        *(float4 *)(hr + c * 4) = v;
+        ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
     }
     ss = block_sum(ss, red);
     const float inv = rsqrtf(ss / (float)d + eps);
-    for (int j = threadIdx.x; j < d; j += blockDim.x)
-        act_store(n, (size_t)m * d + j, hr[j] * inv * gain[j]);
+    __syncthreads();  // h1 row written by this block is re-read below
+#pragma unroll 2
+    for (int c = threadIdx.x; c < nch; c += blockDim.x) {
+        const float4 v = *(const float4 *)(hr + c * 4);
+        const float4 gv = *(const float4 *)(gain + c * 4);
+        act_store4(n, (size_t)m * d + c * 4,
+                   make_float4(v.x * inv * gv.x, v.y * inv * gv.y, v.z * inv * gv.z, v.w * inv * gv.w));
+    }
 }
 
+// a = silu(g) * u over 4-element vectors (f and blk multiples of 4).
 __global__ void swiglu_kernel(PartIn y, int M, int f, int blk, ActOut a) {
-    const long long total = (long long)M * f;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
-         idx += (long long)gridDim.x * blockDim.x) {
+    pdl_trigger();
+    pdl_wait();
+    const long long total4 = (long long)M * f / 4;
+    for (long long i4 = blockIdx.x * (long long)blockDim.x + threadIdx.x; i4 < total4;
+         i4 += (long long)gridDim.x * blockDim.x) {
+        const long long idx = i4 * 4;
         const int m = (int)(idx / f), j = (int)(idx - (long long)m * f);
         const int blkid = j / blk, jj = j - blkid * blk;
         const size_t row = (size_t)m * 2 * f;
-        const float g = part_get(y, row + 2 * blkid * blk + jj);
-        const float u = part_get(y, row + 2 * blkid * blk + blk + jj);
-        const float s = g / (1.f + __expf(-g));
-        act_store(a, (size_t)idx, s * u);
+        const float4 g = part_get4(y, row + 2 * blkid * blk + jj);
+        const float4 u = part_get4(y, row + 2 * blkid * blk + blk + jj);
+        const float gx[4] = {g.x, g.y, g.z, g.w}, ux[4] = {u.x, u.y, u.z, u.w};
+        float r[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) r[e] = gx[e] / (1.f + __expf(-gx[e])) * ux[e];
+        act_store4(a, (size_t)idx, make_float4(r[0], r[1], r[2], r[3]));
     }
 }
 
-// Pooling and the linear head, column-parallel: block (chunk, b) pools 512
-// hidden columns of sequence b (h2 = h1 + y over the k rows, mean or last) and
-// writes its partial dot products with every head row to part[b][chunk][C].
-constexpr int kReadoutCols = 512;
+// Pooling and the linear head, column-parallel: block (chunk, b) pools 64
+// hidden columns of sequence b (h2 = h1 + y summed over the k rows by four
+// row groups, then mean or last) and writes its partial dot products with
+// every head row to part[b][chunk][C]; four classes are reduced at a time.
+constexpr int kReadoutCols = 64;
 
-__global__ void readout_partial_kernel(PartIn y, const float *__restrict__ h1,
+__global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const float *__restrict__ h1,
                                        const float *__restrict__ head_w, int pool, int k, int d,
                                        int C, float *__restrict__ part) {
-    __shared__ float red[32];
+    pdl_trigger();
+    pdl_wait();
+    __shared__ float acc_s[4][kReadoutCols];
+    __shared__ float pooled[kReadoutCols];
+    __shared__ float red[4][8];
     const int chunk = blockIdx.x, b = blockIdx.y;
+    const int c = threadIdx.x & (kReadoutCols - 1), rg = threadIdx.x / kReadoutCols;
+    const int col = chunk * kReadoutCols + c;
     const size_t base = (size_t)b * k * d;
-    const float invk = 1.f / (float)k;
-    float pv[2];
-    int col[2];
-#pragma unroll
-    for (int e = 0; e < 2; ++e) {
-        col[e] = chunk * kReadoutCols + threadIdx.x + e * 256;
-        float acc = 0.f;
-        if (col[e] < d) {
-            if (pool == SP_POOL_LAST) {
-                const size_t o = base + (size_t)(k - 1) * d + col[e];
+    float acc = 0.f;
+    if (col < d) {
+        if (pool == SP_POOL_LAST) {
+            if (rg == 0) {
+                const size_t o = base + (size_t)(k - 1) * d + col;
                 acc = h1[o] + part_get(y, o);
-            } else {
-                for (int r = 0; r < k; ++r) {
-                    const size_t o = base + (size_t)r * d + col[e];
-                    acc += h1[o] + part_get(y, o);
-                }
-                acc *= invk;
+            }
+        } else {
+            for (int r = rg; r < k; r += 4) {
+                const size_t o = base + (size_t)r * d + col;
+                acc += h1[o] + part_get(y, o);
             }
         }
-        pv[e] = acc;
     }
-    for (int c = 0; c < C; ++c) {
-        float acc = 0.f;
+    acc_s[rg][c] = acc;
+    __syncthreads();
+    if (threadIdx.x < kReadoutCols) {
+        const float sum = (acc_s[0][c] + acc_s[1][c]) + (acc_s[2][c] + acc_s[3][c]);
+        pooled[c] = pool == SP_POOL_LAST ? sum : sum / (float)k;
+    }
+    __syncthreads();
+    // thread (group cg = tid / 64, column c): class c0 + cg
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int c0 = 0; c0 < C; c0 += 4) {
+        const int cls = c0 + rg;
+        float v = (cls < C && col < d) ? head_w[(size_t)cls * d + col] * pooled[c] : 0.f;
 #pragma unroll
-        for (int e = 0; e < 2; ++e)
-            if (col[e] < d) acc += head_w[(size_t)c * d + col[e]] * pv[e];
-        acc = block_sum(acc, red);
-        if (threadIdx.x == 0) part[((size_t)b * gridDim.x + chunk) * C + c] = acc;
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0) red[w >> 1][w & 1] = v;
+        __syncthreads();
+        if (threadIdx.x < 4 && c0 + (int)threadIdx.x < C)
+            part[((size_t)b * gridDim.x + chunk) * C + c0 + threadIdx.x] =
+                red[threadIdx.x][0] + red[threadIdx.x][1];
+        __syncthreads();
     }
 }
 
 __global__ void readout_finish_kernel(const float *__restrict__ part, int n_chunks, int C,
                                       const float *__restrict__ head_b, float *__restrict__ logits) {
+    pdl_trigger();
+    pdl_wait();
     const int b = blockIdx.x;
     for (int c = threadIdx.x; c < C; c += blockDim.x) {
         float acc = head_b ? head_b[c] : 0.f;
@@ -161,12 +218,16 @@ __global__ void readout_finish_kernel(const float *__restrict__ part, int n_chun
 }
 
 __global__ void to_act_kernel(const float *__restrict__ x, size_t n, ActOut out) {
+    pdl_trigger();
+    pdl_wait();
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
          i += (size_t)gridDim.x * blockDim.x)
         act_store(out, i, x[i]);
 }
 
 __global__ void sum_partials_kernel(PartIn y, size_t n, float *__restrict__ out) {
+    pdl_trigger();
+    pdl_wait();
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
          i += (size_t)gridDim.x * blockDim.x)
         out[i] = part_get(y, i);
@@ -179,6 +240,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const float *__restrict_
                                                         const T *__restrict__ W,
                                                         float *__restrict__ Y, int M, int N,
                                                         int K) {
+    pdl_trigger();
+    pdl_wait();
     constexpr int BM = 64, BN = 64, BK = 32;
     __shared__ float Xs[BK][BM + 4];
     __shared__ float Ws[BK][BN + 4];
@@ -226,39 +289,35 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const float *__restrict_
 cudaError_t launch_rmsnorm_rows(int x_bf16, const void *x, int row_mod, const float *gain,
                                 float eps, int M, int d, ActOut out, cudaStream_t st) {
     if (x_bf16)
-        rmsnorm_rows_kernel<bf16><<<M, kRowThreads, 0, st>>>((const bf16 *)x, row_mod, gain, eps, d,
-                                                             out);
+        return launch_k(rmsnorm_rows_kernel<bf16>, dim3(M), dim3(kRowThreads), 0, st, (const bf16 *)x,
+                        row_mod, gain, eps, d, out);
     else
-        rmsnorm_rows_kernel<float><<<M, kRowThreads, 0, st>>>((const float *)x, row_mod, gain, eps,
-                                                              d, out);
-    return cudaGetLastError();
+        return launch_k(rmsnorm_rows_kernel<float>, dim3(M), dim3(kRowThreads), 0, st, (const float *)x,
+                        row_mod, gain, eps, d, out);
 }
 
 cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st) {
     const int per_row = (a.Hq + a.Hkv) * (a.dh / 2) + a.Hkv * a.dh;
     dim3 grid(ceil_div(per_row, 256), a.B * a.k);
-    qkv_rope_kernel<<<grid, 256, 0, st>>>(a);
-    return cudaGetLastError();
+    return launch_k(qkv_rope_kernel, grid, dim3(256), 0, st, a);
 }
 
 cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mod,
                                  const float *gain, float eps, int M, int d, float *h1, ActOut n,
                                  cudaStream_t st) {
     if (x_bf16)
-        residual_norm_kernel<bf16><<<M, kWideThreads, 0, st>>>(y, (const bf16 *)x, row_mod, gain,
-                                                              eps, d, h1, n);
+        return launch_k(residual_norm_kernel<bf16>, dim3(M), dim3(kWideThreads), 0, st, y,
+                        (const bf16 *)x, row_mod, gain, eps, d, h1, n);
     else
-        residual_norm_kernel<float><<<M, kWideThreads, 0, st>>>(y, (const float *)x, row_mod, gain,
-                                                               eps, d, h1, n);
-    return cudaGetLastError();
+        return launch_k(residual_norm_kernel<float>, dim3(M), dim3(kWideThreads), 0, st, y,
+                        (const float *)x, row_mod, gain, eps, d, h1, n);
 }
 
 cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_t st) {
-    const long long total = (long long)M * f;
+    const long long total = (long long)M * f / 4;
     int grid = (int)((total + 255) / 256);
     if (grid > 152 * 16) grid = 152 * 16;
-    swiglu_kernel<<<grid, 256, 0, st>>>(y, M, f, blk, a);
-    return cudaGetLastError();
+    return launch_k(swiglu_kernel, dim3(grid), dim3(256), 0, st, y, M, f, blk, a);
 }
 
 size_t readout_scratch_bytes(int B, int d, int C) {
@@ -269,37 +328,36 @@ cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const
                            int pool, int B, int k, int d, int C, float *scratch, float *logits,
                            cudaStream_t st) {
     const int chunks = ceil_div(d, kReadoutCols);
-    readout_partial_kernel<<<dim3(chunks, B), 256, 0, st>>>(y, h1, head_w, pool, k, d, C, scratch);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_k(readout_partial_kernel, dim3(chunks, B), dim3(256), 0, st, y, h1,
+                             head_w, pool, k, d, C, scratch);
     if (e != cudaSuccess) return e;
-    readout_finish_kernel<<<B, 64, 0, st>>>(scratch, chunks, C, head_b, logits);
-    return cudaGetLastError();
+    return launch_k(readout_finish_kernel, dim3(B), dim3(64), 0, st, (const float *)scratch, chunks,
+                    C, head_b, logits);
 }
 
 cudaError_t launch_to_act(const float *x, size_t n, ActOut out, cudaStream_t st) {
     size_t grid = (n + 255) / 256;
     if (grid > 152 * 16) grid = 152 * 16;
     if (grid == 0) grid = 1;
-    to_act_kernel<<<(unsigned)grid, 256, 0, st>>>(x, n, out);
-    return cudaGetLastError();
+    return launch_k(to_act_kernel, dim3((unsigned)grid), dim3(256), 0, st, x, n, out);
 }
 
 cudaError_t launch_sum_partials(PartIn y, size_t n, float *out, cudaStream_t st) {
     size_t grid = (n + 255) / 256;
     if (grid > 152 * 16) grid = 152 * 16;
     if (grid == 0) grid = 1;
-    sum_partials_kernel<<<(unsigned)grid, 256, 0, st>>>(y, n, out);
-    return cudaGetLastError();
+    return launch_k(sum_partials_kernel, dim3((unsigned)grid), dim3(256), 0, st, y, n, out);
 }
 
 cudaError_t launch_gemm_simt(int w_bf16, const void *X, const void *W, float *Y, int M, int N,
                              int K, cudaStream_t st) {
     dim3 grid(ceil_div(N, 64), ceil_div(M, 64));
     if (w_bf16)
-        gemm_simt_kernel<bf16><<<grid, 256, 0, st>>>((const float *)X, (const bf16 *)W, Y, M, N, K);
+        return launch_k(gemm_simt_kernel<bf16>, grid, dim3(256), 0, st, (const float *)X, (const bf16 *)W,
+                        Y, M, N, K);
     else
-        gemm_simt_kernel<float><<<grid, 256, 0, st>>>((const float *)X, (const float *)W, Y, M, N, K);
-    return cudaGetLastError();
+        return launch_k(gemm_simt_kernel<float>, grid, dim3(256), 0, st, (const float *)X,
+                        (const float *)W, Y, M, N, K);
 }
 
 }  // namespace sp
