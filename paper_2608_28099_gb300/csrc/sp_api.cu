@@ -198,10 +198,9 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
     CUtensorMap mk, mv;
     const CUtensorMap *pk = nullptr, *pv = nullptr;
     if (tc && a.kv.layout == SP_KV_PAGED) {
-        const long long rows = (long long)a.kv.n_pages * a.Hkv * a.kv.page_size;
-        tc = rows <= 0x7fffffffLL &&
-             encode_kmajor_bf16(&mk, a.kv.k_pool, (int)rows, a.dh, a.kv.page_size) &&
-             encode_kmajor_bf16(&mv, a.kv.v_pool, (int)rows, a.dh, a.kv.page_size);
+        const long long blocks = (long long)a.kv.n_pages * a.Hkv;
+        tc = encode_kv_pages_bf16(&mk, a.kv.k_pool, blocks, a.kv.page_size) &&
+             encode_kv_pages_bf16(&mv, a.kv.v_pool, blocks, a.kv.page_size);
         pk = &mk;
         pv = &mv;
     }

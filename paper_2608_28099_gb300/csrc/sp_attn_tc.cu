@@ -20,15 +20,24 @@
 //                             operand from TMEM), V read in place from shared
 //                             memory as an MN-major B operand
 // Each warpgroup keeps its own (max, sum, O_w) and writes its own partial, so
-// a work unit yields two partials that the merge combines like splits.
-// Tiles come from a 6-stage ring filled by one producer warp: TMA for whole
-// cache tiles of a paged pool, cp.async for contiguous caches, plain loads for
-// the tile holding the sequence end and the new keys (and for pages that fail
-// the bounds check, which are zero-filled and reported).
+// a work unit yields two partials that the merge combines like splits.  The
+// even and odd tiles form two independent pipelines, each with its own MMA
+// issuing warp: one thread issuing small-N MMAs back to back leaves the tensor
+// pipe idle between them, two keep it busy.
+// Tiles come from a 6-stage ring: TMA for whole cache tiles of a paged pool
+// (one box per (page, kv head) block of K and of V, issued by two lead warps
+// taking alternate tiles), cp.async for contiguous caches, plain loads for the
+// tile holding the sequence end and the new keys (and for pages that fail the
+// bounds check, which are zero-filled and reported).
 //
-// Warps 0-3 and 4-7: the two softmax warpgroups (+ epilogue); warp 8:
-// producer; warp 9: TMEM owner and MMA issuer (lane 0).  Every wait is
-// time-limited (SP_DEV_TIMEOUT).
+// Tile layout in shared memory (K and V alike, 64 tokens x 128 dims bf16):
+// [8-token group][dim half][8 tokens][64 dims], 128-byte swizzle, so that a
+// (page, head) block of 16/32/64 tokens is one TMA box and both MMAs read the
+// tile with uniform strides (8-token groups 2048 B apart, dim halves 1024 B).
+//
+// Warps 0-3 and 4-7: the two softmax warpgroups (+ epilogue); warps 8 and 11:
+// producers; warp 9: TMEM owner and MMA issuer of even tiles; warp 10: MMA
+// issuer of odd tiles.  Every wait is time-limited (SP_DEV_TIMEOUT).
 #include <cudaTypedefs.h>
 #include <string.h>
 
@@ -50,24 +59,28 @@ constexpr int STG = 6;                         // K/V ring depth
 // i + 2 before it releases stage i + 1, so DEFER <= STG - 2 (else deadlock).
 constexpr int DEFER = STG - 2;
 static_assert(DEFER >= 0 && DEFER <= STG - 2, "cp.async publication depth");
-constexpr int KVSUB = TT * 64 * 2;             // one [64 tokens][64] swizzled sub-tile
-constexpr int KV_STAGE = 4 * KVSUB;            // K (2 subs) + V (2 subs)
+constexpr int KV_TILE = TT * DH * 2;           // K or V of one tile, 16 KB
+constexpr int KV_STAGE = 2 * KV_TILE;          // K then V
+constexpr uint32_t GROUP_STRIDE = 2048;        // 8-token groups
+constexpr uint32_t HALF_STRIDE = 1024;         // 64-dim halves within a group
 constexpr int OFF_KV = 0;
 constexpr int MAX_SPLIT_PAGES = 1024;          // page ids of one split staged in smem
 constexpr int OFF_PAGES = OFF_KV + STG * KV_STAGE;
 constexpr int OFF_BAR = OFF_PAGES + MAX_SPLIT_PAGES * 4;
 constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
-constexpr int THREADS = 320;                   // 2 softmax warpgroups, producer, MMA
-constexpr int PRODUCER_WARP = 8, MMA_WARP = 9;
+constexpr int THREADS = 384;                   // 2 softmax warpgroups, 2 producers, 2 MMA
+constexpr int PRODUCER_WARP = 8, MMA_WARP = 9, MMA_WARP1 = 10, PRODUCER_WARP1 = 11;
 constexpr float RESCALE_LOG2 = 8.f;            // tolerate p <= 2^8 before rescaling O
 // TMEM columns: S0 [0,64) S1 [64,128) O0 [128,256) O1 [256,384) Qhi [384,448) Qlo [448,512);
 // P_w (64 bf16 per row) overwrites the first 32 columns of S_w once S_w is read.
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t O_COL = 128, QHI_COL = 384, QLO_COL = 448;
 
-// byte offset of 16-byte chunk `ch` (0..7) of row `row` in a swizzled sub-tile
-__device__ __forceinline__ uint32_t swz(int row, int ch) {
-    return (uint32_t)(row * 128 + ((ch ^ (row & 7)) << 4));
+// byte offset of 16-byte chunk c16 (0..15, 8 dims each) of token row `row`
+// (0..63) in a K or V tile
+__device__ __forceinline__ uint32_t kv_off(int row, int c16) {
+    return (uint32_t)((row >> 3) * GROUP_STRIDE + (c16 >> 3) * HALF_STRIDE + (row & 7) * 128 +
+                      (((c16 & 7) ^ (row & 7)) << 4));
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
@@ -76,7 +89,7 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 }
 
 struct Bars {
-    uint64_t kv_full[STG], kv_empty[STG], s_full[2], p_full[2], pv_done[2], fin, q_full;
+    uint64_t kv_full[STG], kv_empty[STG], s_full[2], p_full[2], pv_done[2], fin, q_full;  // fin: 2 arrivals
     uint32_t tmem;
     int abort;
 };
@@ -104,11 +117,14 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int t_end = min(total, t_begin + a.split_tokens);
     const int n_tiles = (t_end - t_begin + TT - 1) / TT;
     const int act_warps = (R + 31) / 32;  // softmax warps that own real query rows
-    // producers: warp 8, plus the softmax warps that own no rows (they help
-    // with the cp.async and plain-load tiles; only warp 8 issues TMA)
-    const int n_prod = 1 + 2 * (4 - act_warps);
-    const bool is_producer = warp == PRODUCER_WARP || (warp < 8 && (warp & 3) >= act_warps);
-    const int pidx = warp == PRODUCER_WARP ? 0 : 1 + (warp >> 2) * (4 - act_warps) + ((warp & 3) - act_warps);
+    // producers: warps 8 and 11, plus the softmax warps that own no rows (they
+    // help with the cp.async and plain-load tiles; warps 8 and 11 issue TMA)
+    const int n_prod = 2 + 2 * (4 - act_warps);
+    const bool is_producer = warp == PRODUCER_WARP || warp == PRODUCER_WARP1 ||
+                             (warp < 8 && (warp & 3) >= act_warps);
+    const int pidx = warp == PRODUCER_WARP    ? 0
+                     : warp == PRODUCER_WARP1 ? 1
+                                              : 2 + (warp >> 2) * (4 - act_warps) + ((warp & 3) - act_warps);
     const bool paged = a.kv.layout == SP_KV_PAGED;
 
     if (threadIdx.x == 0) {
@@ -121,7 +137,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             mbar_init(&bars->p_full[i], 32 * act_warps);
             mbar_init(&bars->pv_done[i], 1);
         }
-        mbar_init(&bars->fin, 1);
+        mbar_init(&bars->fin, 2);
         mbar_init(&bars->q_full, 1);
         bars->abort = 0;
         fence_mbar_init();
@@ -198,7 +214,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (is_producer) {
         // ------------------------------------------------------------ producers
         const int ptid = pidx * 32 + lane, pstride = 32 * n_prod;
-        const bool lead = pidx == 0;  // warp 8: TMA issue and drain
+        const bool tma_warp = pidx < 2;  // warps 8 and 11 issue TMA for even and odd tiles
         int issued = 0;
         bool deferred[STG] = {false, false, false};  // contiguous tiles awaiting cp.async
         int bad = 0;
@@ -207,7 +223,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (!mbar_wait(&bars->kv_empty[st], ((i / STG) & 1) ^ 1, abort)) break;
             const int t0 = t_begin + i * TT;
             uint8_t *K = smem + OFF_KV + st * KV_STAGE;
-            uint8_t *V = K + 2 * KVSUB;
+            uint8_t *V = K + KV_TILE;
+            const bool lead = pidx == (i & 1);
             bool pure = (t0 + TT <= L);
             if (pure && paged) {
                 const int npg = TT / P;
@@ -224,17 +241,17 @@ __global__ void __launch_bounds__(THREADS, 1)
                 if (pure && !lead) {
                     mbar_arrive(&bars->kv_full[st]);
                 } else if (pure) {
-                    // one TMA box per lane: lane = 4 * page + (K lo, K hi, V lo, V hi);
-                    // lane 0 registers the stage's bytes before any box is issued
+                    // one TMA box per lane: lane = 2 * page + (K, V), each the
+                    // (page, head) block of P tokens; lane 0 registers the
+                    // stage's bytes before any box is issued
                     if (lane == 0) mbar_arrive_expect_tx(&bars->kv_full[st], KV_STAGE);
                     __syncwarp();
-                    if (lane < 4 * npg) {
-                        const int j = lane >> 2, part = lane & 3;
+                    if (lane < 2 * npg) {
+                        const int j = lane >> 1, part = lane & 1;
                         const int page = jl + j < n_lp ? spages[jl + j] : ptab[t0 / P + j];
-                        const int row = (page * a.Hkv + g) * P;
-                        const uint32_t off = (uint32_t)(j * P * 128) + (part & 1) * KVSUB;
-                        tma_load_2d((part < 2 ? K : V) + off, part < 2 ? &map_k : &map_v,
-                                    &bars->kv_full[st], (part & 1) * 64, row);
+                        const int grp = (page * a.Hkv + g) * (P / 8);
+                        tma_load_4d((part ? V : K) + j * P * 256, part ? &map_v : &map_k,
+                                    &bars->kv_full[st], 0, 0, 0, grp);
                     }
                     if (lane != 0) mbar_arrive(&bars->kv_full[st]);
                 }
@@ -245,7 +262,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 for (int idx = ptid; idx < TT * 16; idx += pstride) {
                     const int row = idx >> 4, c16 = idx & 15;
                     const size_t src = ((size_t)(t0 + row) * a.Hkv + g) * DH + c16 * 8;
-                    const uint32_t dst = (c16 >> 3) * KVSUB + swz(row, c16 & 7);
+                    const uint32_t dst = kv_off(row, c16);
                     cp_async16(K + dst, kb + src);
                     cp_async16(V + dst, vb + src);
                 }
@@ -256,7 +273,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 for (int idx = ptid; idx < TT * 16; idx += pstride) {
                     const int row = idx >> 4, c16 = idx & 15;
                     const int t = t0 + row;
-                    const uint32_t dst = (c16 >> 3) * KVSUB + swz(row, c16 & 7);
+                    const uint32_t dst = kv_off(row, c16);
                     uint4 kv4 = make_uint4(0, 0, 0, 0), vv4 = make_uint4(0, 0, 0, 0);
                     if (t < L) {
                         const bf16 *ks = nullptr, *vs = nullptr;
@@ -317,68 +334,69 @@ __global__ void __launch_bounds__(THREADS, 1)
                 deferred[j % STG] = false;
             }
         }
-        if (lead && lane == 0) {
+        if (tma_warp && lane == 0) {
             // drain TMA writes still in flight (only possible after an abort)
             for (int j = issued > STG ? issued - STG : 0; j < issued; ++j)
-                mbar_wait_drain(&bars->kv_full[j % STG], (j / STG) & 1);
+                if ((j & 1) == pidx) mbar_wait_drain(&bars->kv_full[j % STG], (j / STG) & 1);
         }
         bad = __any_sync(0xffffffffu, bad);
         if (bad && lane == 0 && a.status) atomicOr(a.status, SP_DEV_BAD_PAGE);
-    } else if (warp == MMA_WARP) {
-        // ------------------------------------------------------------ MMA issuer
-        // Order on the tensor pipe: S_0, S_1, then per tile i: PV_i (after
-        // softmax i) and S_{i+2} (reusing S buffer i & 1).  PV_i does not wait
-        // for any later tile's data, so stage i is released as soon as its
-        // softmax is done.
+    } else if (warp == MMA_WARP || warp == MMA_WARP1) {
+        // ------------------------------------------------------------ MMA issuers
+        // Pipeline w = warp - MMA_WARP takes tiles i = w, w + 2, ...: S_w, then
+        // per tile i: PV_i (after softmax i) and S_{i+2} (reusing S buffer w).
+        // PV_i does not wait for any later tile's data, so stage i is released
+        // as soon as its softmax is done.
+        const int w = warp - MMA_WARP;
         if (lane == 0) {
             constexpr uint32_t idesc_s = idesc_bf16_f32(128, TT);
             constexpr uint32_t idesc_o = idesc_bf16_f32_bmn(128, DH);
+            const uint32_t s_tmem = tmem + (uint32_t)(w * TT);  // S_w; P_w over its first half
+            const uint32_t o_tmem = tmem + O_COL + (uint32_t)(w * DH);
             auto issue_s = [&](int i) {
                 const uint8_t *K = smem + OFF_KV + (i % STG) * KV_STAGE;
-                const uint32_t s_tmem = tmem + (uint32_t)((i & 1) * TT);
 #pragma unroll
                 for (int kk = 0; kk < DH / 16; ++kk) {
-                    const int sub = kk >> 2;
-                    const uint32_t off = (uint32_t)((kk & 3) * 2);  // 32 B steps along dh
-                    const uint64_t bk = sw128_kmajor_desc(K + sub * KVSUB) + off;
+                    // 16 dims = 32 B along a 128-byte row of dim half kk / 4
+                    const uint64_t bk =
+                        sw128_kmajor_desc_sbo(K + (kk >> 2) * HALF_STRIDE, GROUP_STRIDE) +
+                        (uint64_t)((kk & 3) * 2);
                     // 16 dims of Q = 8 TMEM columns
                     mma_bf16_ts(s_tmem, tmem + QHI_COL + (uint32_t)(kk * 8), bk, idesc_s,
                                 kk > 0 ? 1u : 0u);
                     mma_bf16_ts(s_tmem, tmem + QLO_COL + (uint32_t)(kk * 8), bk, idesc_s, 1u);
                 }
-                mma_commit(&bars->s_full[i & 1]);
+                mma_commit(&bars->s_full[w]);
             };
             bool ok = true;
-            for (int i = 0; ok && i < 2 && i < n_tiles; ++i) {
-                ok = mbar_wait(&bars->kv_full[i % STG], (i / STG) & 1, abort);
+            if (w < n_tiles) {
+                ok = mbar_wait(&bars->kv_full[w % STG], (w / STG) & 1, abort);
                 if (ok) {
                     tc_fence_after();
-                    issue_s(i);
+                    issue_s(w);
                 }
             }
-            for (int i = 0; ok && i < n_tiles; ++i) {
-                if (!mbar_wait(&bars->p_full[i & 1], (i >> 1) & 1, abort)) break;
+            for (int i = w; ok && i < n_tiles; i += 2) {
+                if (!mbar_wait(&bars->p_full[w], (i >> 1) & 1, abort)) break;
                 tc_fence_after();
-                const uint8_t *V = smem + OFF_KV + (i % STG) * KV_STAGE + 2 * KVSUB;
-                const uint32_t p_tmem = tmem + (uint32_t)((i & 1) * TT);  // P_i over S_i
-                const uint32_t o_tmem = tmem + O_COL + (uint32_t)((i & 1) * DH);
+                const uint8_t *V = smem + OFF_KV + (i % STG) * KV_STAGE + KV_TILE;
 #pragma unroll
                 for (int kk = 0; kk < TT / 16; ++kk) {
-                    // 16 tokens of P = 8 TMEM columns; 16 token rows of V = 2 KB
-                    mma_bf16_ts(o_tmem, p_tmem + (uint32_t)(kk * 8),
-                                sw128_mnmajor_desc(V + kk * 2048, KVSUB), idesc_o,
-                                (i >= 2 || kk > 0) ? 1u : 0u);
+                    // 16 tokens of P = 8 TMEM columns; 16 tokens of V = two 8-token groups
+                    mma_bf16_ts(o_tmem, s_tmem + (uint32_t)(kk * 8),
+                                sw128_mnmajor_desc2(V + kk * 2 * GROUP_STRIDE, HALF_STRIDE, GROUP_STRIDE),
+                                idesc_o, (i >= 2 || kk > 0) ? 1u : 0u);
                 }
                 mma_commit(&bars->kv_empty[i % STG]);
-                mma_commit(&bars->pv_done[i & 1]);
+                mma_commit(&bars->pv_done[w]);
                 if (i + 2 < n_tiles) {
-                    // S buffer i & 1 is free: softmax i has read it (p_full above)
+                    // S buffer w is free: softmax i has read it (p_full above)
                     if (!mbar_wait(&bars->kv_full[(i + 2) % STG], ((i + 2) / STG) & 1, abort)) break;
                     tc_fence_after();
                     issue_s(i + 2);
                 }
             }
-            mma_commit(&bars->fin);  // completes when every MMA above is done
+            mma_commit(&bars->fin);  // completes when every MMA of this issuer is done
         }
         __syncwarp();
     } else if (warp < 8 && (warp & 3) < act_warps) {

@@ -217,7 +217,7 @@ void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, in
 size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits);
 cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st);
 // tcgen05 kernel: head_dim 128, bf16 cache, R <= 128; paged caches need TMA
-// maps of the K and V pools viewed as [n_pages * Hkv * page_size][128].
+// maps of the K and V pools from encode_kv_pages_bf16.
 bool attention_tc_supported(const AttnArgs &a);
 cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
                                 const CUtensorMap *map_v, const CUtensorMap &map_q,

@@ -15,6 +15,9 @@ struct TcPlan {
 };
 
 bool encode_kmajor_bf16(CUtensorMap *map, const void *base, int rows, int K, int box_rows);
+// TMA map of a paged K or V pool [n_page_heads][page_size][128] bf16 whose box
+// is one (page, head) block in the attention kernel's shared-memory tile layout.
+bool encode_kv_pages_bf16(CUtensorMap *map, const void *pool, long long n_page_heads, int page_size);
 // TMA map of rotated queries [rows][Hq][128] fp32 by (k rows x G heads) boxes.
 bool encode_q_group_f32(CUtensorMap *map, const float *q, int rows, int Hq, int G, int k);
 bool tc_supported(int N, int K);

@@ -228,6 +228,24 @@ bool encode_kmajor_bf16(CUtensorMap *map, const void *base, int rows, int K, int
     return r == CUDA_SUCCESS;
 }
 
+bool encode_kv_pages_bf16(CUtensorMap *map, const void *pool, long long n_page_heads, int page_size) {
+    // pool [n_page_heads][page_size][128] bf16 viewed as (64 dims, 8 rows,
+    // 2 dim halves, row groups of 8): one box = one (page, head) block laid out
+    // in shared memory as [row group][dim half][8 rows][128 B], 128-byte swizzle
+    PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+    if (!fn || ((uintptr_t)pool & 15) || page_size % 8 || page_size > 64) return false;
+    const long long groups = n_page_heads * (page_size / 8);
+    if (groups <= 0 || groups > 0x7fffffffLL) return false;
+    cuuint64_t dims[4] = {64, 8, 2, (cuuint64_t)groups};
+    cuuint64_t strides[3] = {256, 128, 2048};
+    cuuint32_t box[4] = {64, 8, 2, (cuuint32_t)(page_size / 8)};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(pool), dims, strides,
+                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 bool encode_q_group_f32(CUtensorMap *map, const float *q, int rows, int Hq, int G, int k) {
     // q [rows = B*k][Hq][128] fp32; one box = the G heads of one kv group for
     // the k rows of one sequence: [k][G][128], unswizzled

@@ -102,6 +102,14 @@ __device__ __forceinline__ void tma_load_3d(void *smem_dst, const CUtensorMap *m
         "l"((uint64_t)map), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
         : "memory");
 }
+__device__ __forceinline__ void tma_load_4d(void *smem_dst, const CUtensorMap *map, uint64_t *bar,
+                                            int c0, int c1, int c2, int c3) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, "
+        "%4, %5, %6}], [%2];" ::"r"(smem_u32(smem_dst)),
+        "l"((uint64_t)map), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+        : "memory");
+}
 __device__ __forceinline__ uint64_t policy_evict_first() {
     uint64_t p;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
@@ -183,6 +191,17 @@ __device__ __forceinline__ uint64_t sw128_kmajor_desc(const void *tile) {
     return d;
 }
 
+// Same with the 8-row groups `sbo` bytes apart (a multiple of 1024).
+__device__ __forceinline__ uint64_t sw128_kmajor_desc_sbo(const void *tile, uint32_t sbo) {
+    const uint64_t addr = smem_u32(tile);
+    uint64_t d = (addr & 0x3FFFFull) >> 4;
+    d |= 1ull << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
+    d |= 1ull << 46;
+    d |= 2ull << 61;
+    return d;
+}
+
 // Shared-memory matrix descriptor for an MN-major operand stored with the
 // 128-byte swizzle: rows run along K (8-row groups 1024 B apart), each row holds
 // 64 consecutive MN elements; successive 64-wide MN chunks are `mn_stride`
@@ -194,6 +213,18 @@ __device__ __forceinline__ uint64_t sw128_mnmajor_desc(const void *tile, uint32_
     d |= (uint64_t)(1024 >> 4) << 32;                    // stride byte offset: 8 K-rows
     d |= 1ull << 46;                                     // descriptor version for sm_100
     d |= 2ull << 61;                                     // 128-byte swizzle
+    return d;
+}
+
+// MN-major with explicit strides: 64-wide MN chunks `lbo` bytes apart, 8-row
+// K groups `sbo` bytes apart.
+__device__ __forceinline__ uint64_t sw128_mnmajor_desc2(const void *tile, uint32_t lbo, uint32_t sbo) {
+    const uint64_t addr = smem_u32(tile);
+    uint64_t d = (addr & 0x3FFFFull) >> 4;
+    d |= (uint64_t)((lbo >> 4) & 0x3FFF) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFF) << 32;
+    d |= 1ull << 46;
+    d |= 2ull << 61;
     return d;
 }
 
