@@ -2,6 +2,7 @@
 """Throughput of the Speculative Probing classify path on one GB300.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 4b] [--impl ours|reference]
+    python bench.py --sweep [all|quick] [--steps K] [--warmup W]
 
 One step = one sp_classify call over one batch of the named seeded workload
 (every stage of the path: input norm, Q/K/V projection, rotation, split-KV
@@ -13,10 +14,17 @@ is timed with CUDA events on the launching stream.  Prints one JSON line.
 Multi-GPU: the path shards by sequence with no exchange step, so N ranks run N
 independent replicas (weak scaling) and `value` counts all ranks' sequences
 over the slowest rank's time.
+
+--sweep times the serving sweep at the d=4096 shape (batch x length x k x
+classes, bf16 paged caches with +-25% ragged lengths drawn on the device) and
+prints one JSON line per point with its stage times, the achieved HBM
+fraction and the projections' weight GB/s and TFLOP/s, then a summary line
+naming the rows (batch x k) where the projections turn tensor-bound.
 """
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -52,6 +60,8 @@ def parse_args():
                         "shared: the soft prompt, whose Q/K/V projection is precomputed")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "quick"],
+                   help="time the serving-sweep points instead of one workload")
     return p.parse_args()
 
 
@@ -230,6 +240,27 @@ def workload_config(spec, w, args):
 
 
 # --------------------------------------------------------------------------- #
+# ranks
+# --------------------------------------------------------------------------- #
+def rank_max(x: float, device) -> float:
+    """Maximum of x over the ranks of the default process group (x itself when
+    there is none): the slowest rank's time."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_available() or not dist.is_initialized() or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def shard_spec(spec, rank: int):
+    """Rank r classifies its own batch of the same configuration: an independent
+    draw (seed + 1000 r) of the workload."""
+    return spec if rank == 0 else dataclasses.replace(spec, seed=spec.seed + 1000 * rank)
+
+
+# --------------------------------------------------------------------------- #
 # our arm
 # --------------------------------------------------------------------------- #
 def run_ours(args, spec, w, rank, world):
@@ -305,11 +336,7 @@ def run_ours(args, spec, w, rank, world):
     if world > 1:
         dist.barrier()
     clk = clocks.stop()
-    ms = sum(step_ms) / len(step_ms)
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = rank_max(sum(step_ms) / len(step_ms), "cuda")
     assert sp.sp_check_status(h) == 0, sp.sp_last_error()
     eager_ms = sum(timed(step, args.steps)) / args.steps
 
@@ -340,11 +367,7 @@ def run_ours(args, spec, w, rank, world):
         el = time.perf_counter() - t0
         if i >= args.warmup:
             e2e_s.append(el)
-    e2e_mean = sum(e2e_s) / len(e2e_s)
-    if world > 1:
-        t = torch.tensor([e2e_mean], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_mean = float(t.item())
+    e2e_mean = rank_max(sum(e2e_s) / len(e2e_s), "cuda")
     h2d = h_ids.numel() * 4 + h_lens.numel() * 4 + (h_rows.numel() * h_rows.element_size()
                                                      if h_rows is not None else 0)
     d2h = h_logits.numel() * 4
@@ -402,8 +425,141 @@ def run_ours(args, spec, w, rank, world):
     model.close()
 
 
+# --------------------------------------------------------------------------- #
+# serving sweep
+# --------------------------------------------------------------------------- #
+QUICK_SWEEP = [f"sweep_B{B}_L{L}_k{k}_C16" for B in (1, 32, 256) for L in (512, 8192)
+               for k in (1, 16)]
+
+
+def run_sweep(args):
+    import torch
+
+    import paper_2608_28099_gb300 as sp
+    from paper_2608_28099_gb300 import build_lib
+    from paper_2608_28099_gb300 import workloads as wl
+
+    torch.cuda.set_device(0)
+    build_lib.build()
+    sp.load_library()
+    hbm, tfl, peak_src = peaks()
+    tfl_sus = tfl
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            tfl_sus = float(json.load(f).get("bf16_tflops_sustained", tfl))
+    except Exception:
+        pass
+    names = wl.SWEEP_POINTS if args.sweep == "all" else QUICK_SWEEP
+    specs = [wl.named(n, rows_per_seq=True) for n in names]
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    max_len = max(s.len_hi for s in specs)
+    max_b = max(s.batch for s in specs)
+    models, base_w = {}, None
+    by_bl = {}
+    for s in specs:
+        by_bl.setdefault((s.batch, s.len_lo, s.len_hi), []).append(s)
+    results = []
+    clocks = ClockSampler(0)
+    clocks.start()
+    for (B, lo, hi), group in by_bl.items():
+        dev = None
+        for s in group:
+            k, C = s.shape.k_rows, s.shape.n_classes
+            if (k, C) not in models:
+                sw = wl.generate_on_device(s)  # weights for this (k, C); pools discarded
+                del sw.k_pool, sw.v_pool
+                models[(k, C)] = (sp.Model(s.shape, sw.weights, max_b, max_len), sw.weights)
+            model, weights = models[(k, C)]
+            dw = wl.generate_on_device(s, weights=weights)
+            cache = sp.DevicePagedCache(dw)
+            h = model.handle
+            ids = torch.arange(B, dtype=torch.int32, device="cuda")
+            r = np.ascontiguousarray(dw.rows)
+            rows = torch.from_numpy(r.view(np.int16)).cuda()
+            logits = torch.empty((B, C), dtype=torch.float32, device="cuda")
+
+            def step():
+                sp.sp_classify(h, torch.cuda.current_stream(), B, ids, cache.seq_lens, cache.desc,
+                               rows, logits)
+
+            for _ in range(args.warmup):
+                step()
+            torch.cuda.synchronize()
+            assert sp.sp_check_status(h) == 0, sp.sp_last_error()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                step()
+            torch.cuda.synchronize()
+            times = []
+            for _ in range(args.steps):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                g.replay()
+                e1.record()
+                torch.cuda.synchronize()
+                times.append(e0.elapsed_time(e1))
+            ms = statistics.median(times)
+            sp.sp_set_option(h, sp.SP_OPT_PROFILE, 1)
+            pg = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(pg):
+                step()
+            acc = {}
+            for _ in range(max(3, args.steps // 2)):
+                flush.zero_()
+                pg.replay()
+                for nme, v in sp.sp_stage_times(h).items():
+                    acc.setdefault(nme, []).append(v)
+            sp.sp_set_option(h, sp.SP_OPT_PROFILE, 0)
+            stage_us = {nme: 1e3 * statistics.median(v) for nme, v in acc.items()}
+            assert sp.sp_check_status(h) == 0, sp.sp_last_error()
+            fake = wl.Workload(s, weights, wl.KVCache(wl.LAYOUT_PAGED, wl.BF16, dw.seq_lens),
+                               dw.seq_ids, dw.rows)
+            st_work, totals = work_model(fake, True)
+            proj = [n for n in ("qkv", "o_proj", "gate_up", "down") if n in st_work]
+            p_bytes = sum(st_work[n]["bytes"] for n in proj)
+            p_flops = sum(st_work[n]["flops"] for n in proj)
+            p_us = sum(stage_us.get(n, 0.0) for n in proj)
+            M = B * k
+            hbm_floor = p_bytes / (hbm * 1e9) * 1e6
+            tensor_floor = 2 * p_flops / (tfl_sus * 1e12) * 1e6  # bf16 hi + lo operand passes
+            line = {"sweep_point": s.name, "B": B, "L": f"U[{lo},{hi}]", "k": k, "C": C,
+                    "rows": M, "us_per_call": ms * 1e3, "seq_per_s": B / (ms / 1e3),
+                    "hbm_gbs": totals["total_bytes"] / (ms / 1e3) / 1e9,
+                    "frac_of_8tbs": totals["total_bytes"] / (ms / 1e3) / 8e12,
+                    "frac_of_measured": totals["total_bytes"] / (ms / 1e3) / (hbm * 1e9),
+                    "attention": {"us": stage_us.get("attention"),
+                                  "gbs": st_work["attention"]["bytes"] / (stage_us.get("attention", 1e9) * 1e3)},
+                    "projections": {"us": p_us, "weight_gbs": p_bytes / (p_us * 1e3) if p_us else None,
+                                    "tflops": p_flops / (p_us * 1e6) if p_us else None,
+                                    "hbm_floor_us": hbm_floor, "tensor_floor_us": tensor_floor,
+                                    "bound": "tensor" if tensor_floor > hbm_floor else "hbm"},
+                    "stages_us": stage_us}
+            results.append(line)
+            print(json.dumps(line), flush=True)
+            del g, pg, cache, dw
+            torch.cuda.empty_cache()
+    clk = clocks.stop()
+    tensor_rows = sorted({r["rows"] for r in results if r["projections"]["bound"] == "tensor"})
+    hbm_rows = sorted({r["rows"] for r in results if r["projections"]["bound"] == "hbm"})
+    summary = {"sweep": args.sweep, "points": len(results),
+               "projection_crossover": {"largest_hbm_bound_rows": max(hbm_rows) if hbm_rows else None,
+                                        "smallest_tensor_bound_rows": min(tensor_rows) if tensor_rows else None,
+                                        "note": "tensor floor counts the hi and lo bf16 passes; "
+                                                "the same tcgen05 kernel serves both sides"},
+               "peaks": {"hbm_gbs": hbm, "bf16_tflops_sustained": tfl_sus, "source": peak_src},
+               "clocks": clk, "steps": args.steps, "warmup": args.warmup,
+               "l2": "flushed between steps (256 MiB write)"}
+    print(json.dumps(summary), flush=True)
+    for m, _ in models.values():
+        m.close()
+
+
 def main():
     args = parse_args()
+    if args.sweep:
+        run_sweep(args)
+        return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     if world > 1:
@@ -416,7 +572,7 @@ def main():
             torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
             dist.init_process_group("nccl")
     from paper_2608_28099_gb300 import workloads as wl
-    spec = wl.named(args.workload, rows_per_seq=(args.rows == "per-seq"))
+    spec = shard_spec(wl.named(args.workload, rows_per_seq=(args.rows == "per-seq")), rank)
     w = wl.generate(spec)
     if args.impl == "reference":
         run_reference(args, spec, w, rank, world)

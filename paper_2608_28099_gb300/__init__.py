@@ -287,3 +287,22 @@ class DeviceCache:
         ts = ([self.k_flat, self.v_flat] if self.host.layout == SP_KV_CONTIGUOUS
               else [self.k_pool, self.v_pool])
         return sum(t.numel() * t.element_size() for t in ts)
+
+
+class DevicePagedCache:
+    """sp_kv_cache over a workloads.DeviceWorkload's device-resident pools."""
+
+    def __init__(self, dw, device="cuda"):
+        import numpy as np
+        import torch
+        self.host = dw
+        self.seq_lens = torch.from_numpy(np.ascontiguousarray(dw.seq_lens, dtype=np.int32)).to(device)
+        self.page_table = torch.from_numpy(np.ascontiguousarray(dw.page_table)).to(device)
+        self.k_pool, self.v_pool = dw.k_pool, dw.v_pool
+        self.desc = sp_kv_cache(SP_KV_PAGED, None, None, self.k_pool.data_ptr(),
+                                self.v_pool.data_ptr(), self.page_table.data_ptr(),
+                                dw.shape.page_size, max(dw.n_pages, 1), dw.page_table.shape[1],
+                                len(dw.seq_lens))
+
+    def nbytes(self) -> int:
+        return sum(t.numel() * t.element_size() for t in (self.k_pool, self.v_pool))

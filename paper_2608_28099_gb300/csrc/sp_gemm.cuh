@@ -11,7 +11,12 @@
 namespace sp {
 
 struct TcPlan {
-    int bn, m_tiles, n_tiles, n_kb, kb_per_split, splits;
+    int bn, m_tiles, n_tiles, n_kb;
+    bool persistent;    // persistent stream-K kernel, else one CTA per (tile, K split)
+    int kb_per_split;   // tile kernel: k-blocks per split
+    int units_per_cta;  // persistent: (tile, k-block) units per CTA
+    int grid;           // CTAs
+    int splits;         // partial planes of Y
 };
 
 bool encode_kmajor_bf16(CUtensorMap *map, const void *base, int rows, int K, int box_rows);

@@ -1,23 +1,30 @@
 // Tensor-core projection for the decoder layer (Sec. 3.1: Q/K/V, output,
 // gate/up and down projections): Y[M][N] = X[M][K] W[N][K]^T with bf16 weights.
 //
-// One CTA computes a 128 (weight rows) x BN (activation rows) tile over its
-// share of K with tcgen05.mma, accumulating in TMEM.  Weights are the MMA's A
-// operand (M = 128), activations its B operand (N = BN): the handful of rows a
-// classify call has fill the N side of the instruction instead of wasting
-// 7/8 of a 128-row M tile.  Both operands arrive by TMA in 128-byte swizzled
-// K-major tiles through a STAGES-deep mbarrier ring.
+// Work: tiles of 128 weight rows x BN activation rows, each over K in k-blocks
+// of 64.  Weights are the MMA's A operand (M = 128), activations its B
+// operand (N = BN): the handful of rows a classify call has fill the N side of
+// the instruction instead of wasting 7/8 of a 128-row M tile.  Both operands
+// arrive by TMA in 128-byte swizzled K-major tiles through mbarrier rings.
 //
 // Activations come as two bf16 planes hi = rn(x), lo = rn(x - hi); every
 // k-block issues W*hi and W*lo into the same accumulator, so the product
-// carries ~16 bits of the activation's mantissa for the price of a second MMA
-// (free while the projection is bound by weight bandwidth).
+// carries ~16 bits of the activation's mantissa for the price of a second MMA.
 //
-// Split-K: blockIdx.z takes a contiguous range of k-blocks and stores an fp32
-// partial tile; the consumer kernels add the partials.
-//
-// Roles: warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMA, warp 2 owns
-// TMEM, all four warps run the epilogue (warp w reads TMEM lanes 32w..32w+31).
+// Two schedules, fp32 partials in planes of Y that the consumers add:
+//  * tile kernel: one CTA per (tile, K split); split-K when the tiles alone
+//    leave SMs idle.  Roles: warp 0 lane 0 TMA, warp 1 lane 0 MMA, warp 2
+//    TMEM, all four warps the epilogue (warp w: TMEM lanes 32w..32w+31).
+//  * persistent stream-K kernel, for tile counts that fill the SMs badly:
+//    one CTA per SM owns the contiguous (tile, k-block) units [c L, (c+1) L)
+//    in tile-major order.  Its weight and activation rings run across tile
+//    boundaries (the weight stream never drains) and its accumulator is
+//    double-buffered in TMEM (the epilogue of one tile segment overlaps the
+//    MMAs of the next).  Segment j of a tile (in CTA order) stores plane j;
+//    the CTA with the tile's last segment zero-fills the planes past it, so
+//    every plane is written and the sum order is fixed (no atomics).  Roles:
+//    warps 0-3 epilogue, warp 4 lane 0 weights, warp 5 lane 0 activations,
+//    warp 6 TMEM and MMA.
 #include <cudaTypedefs.h>
 
 #include "sp_common.cuh"
@@ -33,8 +40,9 @@ using namespace sm100;
 constexpr int BK = 64;               // bf16 elements per 128-byte swizzle row
 constexpr int A_BYTES = 128 * BK * 2;
 
+// ---------------------------------------------------------------- tile kernel
 template <int BN>
-struct TcCfg {
+struct TileCfg {
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE = A_BYTES + 2 * B_BYTES;
     static constexpr int STAGES = (BN <= 32) ? 8 : (BN == 64 ? 6 : 4);
@@ -52,10 +60,10 @@ struct TcArgs {
 
 template <int BN>
 __global__ void __launch_bounds__(128, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap map_w,
+    gemm_tile_kernel(const __grid_constant__ CUtensorMap map_w,
                    const __grid_constant__ CUtensorMap map_xhi,
                    const __grid_constant__ CUtensorMap map_xlo, TcArgs g) {
-    using Cfg = TcCfg<BN>;
+    using Cfg = TileCfg<BN>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t *full = (uint64_t *)(smem + Cfg::STAGES * Cfg::STAGE);
@@ -184,17 +192,275 @@ __global__ void __launch_bounds__(128, 1)
 }
 
 template <int BN>
-cudaError_t launch_bn(const CUtensorMap &mw, const CUtensorMap &mh, const CUtensorMap &ml,
+cudaError_t launch_tile(const CUtensorMap &mw, const CUtensorMap &mh, const CUtensorMap &ml,
                       const TcArgs &g, dim3 grid, cudaStream_t st) {
-    const int smem = TcCfg<BN>::SMEM;
+    const int smem = TileCfg<BN>::SMEM;
     static bool attr_set = false;  // per device process-wide (one device per process here)
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN>,
+        cudaError_t e = cudaFuncSetAttribute(gemm_tile_kernel<BN>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    return launch_k(gemm_tc_kernel<BN>, grid, dim3(128), (size_t)smem, st, mw, mh, ml, g);
+    return launch_k(gemm_tile_kernel<BN>, grid, dim3(128), (size_t)smem, st, mw, mh, ml, g);
+}
+
+
+// ------------------------------------------------------ persistent stream-K
+constexpr int GEMM_THREADS = 224;
+constexpr int W_WARP = 4, X_WARP = 5, MMA_WARP_G = 6;
+
+template <int BN>
+struct PkCfg {
+    static constexpr int B_BYTES = BN * BK * 2;       // one activation plane of a k-block
+    static constexpr int X_STAGE = 2 * B_BYTES;       // hi + lo
+    static constexpr int W_STAGES = BN <= 32 ? 8 : (BN == 64 ? 6 : 5);
+    static constexpr int X_STAGES = BN <= 32 ? 4 : 3;
+    static constexpr int ACC_COLS = BN < 32 ? 32 : BN;
+    static constexpr int TMEM_COLS = 2 * ACC_COLS;
+    static constexpr int OFF_X = W_STAGES * A_BYTES;
+    static constexpr int OFF_BAR = OFF_X + X_STAGES * X_STAGE;
+    static constexpr int SMEM = OFF_BAR + 512 /*barriers*/ + 1024 /*align*/;
+    static_assert(SMEM <= 227 * 1024, "shared memory");
+    static_assert((2 * W_STAGES + 2 * X_STAGES + 5) * 8 + 8 <= 512, "barrier area");
+};
+
+struct PkArgs {
+    int M, N, n_kb, m_tiles, tiles;
+    int L;            // units per CTA
+    int planes;       // partial planes in y
+    float *y;         // [planes][M][N]
+    size_t plane_stride;
+    int *status;
+};
+
+// The CTA's tile segments: tiles t_first..t_last, k-blocks [lo, hi) of each.
+struct Seg {
+    int t, kb_lo, kb_hi;
+};
+__device__ __forceinline__ Seg segment(const PkArgs &g, long long u0, long long u1, int t) {
+    const long long base = (long long)t * g.n_kb;
+    Seg s;
+    s.t = t;
+    s.kb_lo = (int)(max(u0, base) - base);
+    s.kb_hi = (int)(min(u1, base + g.n_kb) - base);
+    return s;
+}
+
+template <int BN>
+__global__ void __launch_bounds__(GEMM_THREADS, 1)
+    gemm_pk_kernel(const __grid_constant__ CUtensorMap map_w,
+                   const __grid_constant__ CUtensorMap map_xhi,
+                   const __grid_constant__ CUtensorMap map_xlo, PkArgs g) {
+    using Cfg = PkCfg<BN>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t *w_full = (uint64_t *)(smem + Cfg::OFF_BAR);
+    uint64_t *w_empty = w_full + Cfg::W_STAGES;
+    uint64_t *x_full = w_empty + Cfg::W_STAGES;
+    uint64_t *x_empty = x_full + Cfg::X_STAGES;
+    uint64_t *acc_full = x_empty + Cfg::X_STAGES;  // [2]
+    uint64_t *acc_empty = acc_full + 2;             // [2]
+    uint64_t *done = acc_empty + 2;
+    uint32_t *tmem_slot = (uint32_t *)(done + 1);
+    volatile int *abort = (volatile int *)(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long long U = (long long)g.tiles * g.n_kb;
+    const long long u0 = (long long)blockIdx.x * g.L;
+    const long long u1 = min(U, u0 + g.L);
+    pdl_trigger();
+    if (u0 >= U) {
+        pdl_wait();
+        return;  // uniform over the CTA
+    }
+    const int t_first = (int)(u0 / g.n_kb), t_last = (int)((u1 - 1) / g.n_kb);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < Cfg::W_STAGES; ++s) {
+            mbar_init(&w_full[s], 1);
+            mbar_init(&w_empty[s], 1);
+        }
+        for (int s = 0; s < Cfg::X_STAGES; ++s) {
+            mbar_init(&x_full[s], 1);
+            mbar_init(&x_empty[s], 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&acc_full[b], 1);
+            mbar_init(&acc_empty[b], 128);
+        }
+        mbar_init(done, 1);
+        *abort = 0;
+        fence_mbar_init();
+        prefetch_tmap(&map_w);
+        prefetch_tmap(&map_xhi);
+        prefetch_tmap(&map_xlo);
+    }
+    if (warp == MMA_WARP_G) {
+        tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    int issued = 0;  // TMA k-blocks issued by this producer
+    if (warp == W_WARP && lane == 0) {
+        // weights: streamed once (evict-first) and constant, so loading starts
+        // before the previous kernel has finished
+        const uint64_t pol_w = policy_evict_first();
+        int i = 0;
+        bool ok = true;
+        for (int t = t_first; ok && t <= t_last; ++t) {
+            const Seg sg = segment(g, u0, u1, t);
+            const int n0 = (t / g.m_tiles) * 128;
+            for (int kb = sg.kb_lo; kb < sg.kb_hi; ++kb, ++i) {
+                const int s = i % Cfg::W_STAGES;
+                if (i >= Cfg::W_STAGES && !mbar_wait(&w_empty[s], ((i / Cfg::W_STAGES) & 1) ^ 1, abort)) {
+                    ok = false;
+                    break;
+                }
+                mbar_arrive_expect_tx(&w_full[s], A_BYTES);
+                tma_load_2d_hint(smem + s * A_BYTES, &map_w, &w_full[s], kb * BK, n0, pol_w);
+                issued = i + 1;
+            }
+        }
+    } else if (warp == X_WARP && lane == 0) {
+        // activations (re-read by every CTA: evict-last), written by the previous kernel
+        const uint64_t pol_x = policy_evict_last();
+        pdl_wait();
+        int i = 0;
+        bool ok = true;
+        for (int t = t_first; ok && t <= t_last; ++t) {
+            const Seg sg = segment(g, u0, u1, t);
+            const int m0 = (t % g.m_tiles) * BN;
+            for (int kb = sg.kb_lo; kb < sg.kb_hi; ++kb, ++i) {
+                const int s = i % Cfg::X_STAGES;
+                if (i >= Cfg::X_STAGES && !mbar_wait(&x_empty[s], ((i / Cfg::X_STAGES) & 1) ^ 1, abort)) {
+                    ok = false;
+                    break;
+                }
+                uint8_t *st = smem + Cfg::OFF_X + s * Cfg::X_STAGE;
+                mbar_arrive_expect_tx(&x_full[s], Cfg::X_STAGE);
+                tma_load_2d_hint(st, &map_xhi, &x_full[s], kb * BK, m0, pol_x);
+                tma_load_2d_hint(st + Cfg::B_BYTES, &map_xlo, &x_full[s], kb * BK, m0, pol_x);
+                issued = i + 1;
+            }
+        }
+    } else if (warp == MMA_WARP_G && lane == 0) {
+        constexpr uint32_t idesc = idesc_bf16_f32(128, BN);
+        int i = 0, sgi = 0;
+        bool ok = true;
+        for (int t = t_first; ok && t <= t_last; ++t, ++sgi) {
+            const Seg sg = segment(g, u0, u1, t);
+            const int buf = sgi & 1;
+            const uint32_t acc = tmem + (uint32_t)(buf * Cfg::ACC_COLS);
+            // the epilogue has drained this buffer's previous segment
+            if (sgi >= 2 && !mbar_wait(&acc_empty[buf], ((sgi >> 1) - 1) & 1, abort)) break;
+            tc_fence_after();
+            for (int kb = sg.kb_lo; kb < sg.kb_hi; ++kb, ++i) {
+                const int sw = i % Cfg::W_STAGES, sx = i % Cfg::X_STAGES;
+                if (!mbar_wait(&w_full[sw], (i / Cfg::W_STAGES) & 1, abort) ||
+                    !mbar_wait(&x_full[sx], (i / Cfg::X_STAGES) & 1, abort)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint8_t *xs = smem + Cfg::OFF_X + sx * Cfg::X_STAGE;
+                const uint64_t a = sw128_kmajor_desc(smem + sw * A_BYTES);
+                const uint64_t bh = sw128_kmajor_desc(xs);
+                const uint64_t bl = sw128_kmajor_desc(xs + Cfg::B_BYTES);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk) {
+                    // +32 bytes along K per 16-element MMA step (encoded >> 4)
+                    mma_bf16(acc, a + 2 * kk, bh + 2 * kk, idesc, (kb > sg.kb_lo || kk > 0) ? 1u : 0u);
+                    mma_bf16(acc, a + 2 * kk, bl + 2 * kk, idesc, 1u);
+                }
+                mma_commit(&w_empty[sw]);
+                mma_commit(&x_empty[sx]);
+            }
+            if (ok) mma_commit(&acc_full[buf]);
+        }
+        mma_commit(done);  // completes once every MMA issued above has finished
+    } else if (warp < 4) {
+        // epilogue: TMEM -> registers -> fp32 partial plane of each tile segment
+        pdl_wait();  // before writing partials a previous kernel may still be reading
+        const int r = warp * 32 + lane;  // weight row within the tile (TMEM lane)
+        const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+        int sgi = 0;
+        for (int t = t_first; t <= t_last; ++t, ++sgi) {
+            const int buf = sgi & 1;
+            if (!mbar_wait(&acc_full[buf], (sgi >> 1) & 1, abort)) break;
+            tc_fence_after();
+            const int n = (t / g.m_tiles) * 128 + r;
+            const int m0 = (t % g.m_tiles) * BN;
+            const int plane = blockIdx.x - (int)(((long long)t * g.n_kb) / g.L);
+            const int last = (int)((((long long)t + 1) * g.n_kb - 1) / g.L);
+            float *y = g.y + (size_t)plane * g.plane_stride;
+            const uint32_t ta = trow + (uint32_t)(buf * Cfg::ACC_COLS);
+            if constexpr (BN == 16) {
+                float v[16];
+                tmem_ld16(ta, v);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const int m = m0 + j;
+                    if (m < g.M) y[(size_t)m * g.N + n] = v[j];
+                }
+            } else {
+#pragma unroll 1
+                for (int c0 = 0; c0 < BN; c0 += 32) {
+                    float v[32];
+                    tmem_ld32(ta + c0, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int m = m0 + c0 + j;
+                        if (m < g.M) y[(size_t)m * g.N + n] = v[j];
+                    }
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(&acc_empty[buf]);
+            if ((int)blockIdx.x == last) {
+                // planes past the tile's last segment hold zeros
+                for (int p = plane + 1; p < g.planes; ++p) {
+                    float *yz = g.y + (size_t)p * g.plane_stride;
+                    for (int j = 0; j < BN; ++j) {
+                        const int m = m0 + j;
+                        if (m < g.M) yz[(size_t)m * g.N + n] = 0.f;
+                    }
+                }
+            }
+        }
+    }
+    __syncwarp();
+    if (lane == 0) mbar_wait_drain(done, 0);
+    // no TMA write may still be in flight when the CTA's shared memory goes away
+    if (warp == W_WARP && lane == 0)
+        for (int i = issued > Cfg::W_STAGES ? issued - Cfg::W_STAGES : 0; i < issued; ++i)
+            mbar_wait_drain(&w_full[i % Cfg::W_STAGES], (i / Cfg::W_STAGES) & 1);
+    if (warp == X_WARP && lane == 0)
+        for (int i = issued > Cfg::X_STAGES ? issued - Cfg::X_STAGES : 0; i < issued; ++i)
+            mbar_wait_drain(&x_full[i % Cfg::X_STAGES], (i / Cfg::X_STAGES) & 1);
+    tc_fence_before();
+    __syncthreads();
+    if (threadIdx.x == 0 && *abort && g.status) atomicOr(g.status, SP_DEV_TIMEOUT);
+    if (warp == MMA_WARP_G) tmem_dealloc(tmem, Cfg::TMEM_COLS);
+}
+
+template <int BN>
+cudaError_t launch_pk(const CUtensorMap &mw, const CUtensorMap &mh, const CUtensorMap &ml,
+                      const PkArgs &g, int grid, cudaStream_t st) {
+    const int smem = PkCfg<BN>::SMEM;
+    static bool attr_set = false;  // per device process-wide (one device per process here)
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(gemm_pk_kernel<BN>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    return launch_k(gemm_pk_kernel<BN>, dim3(grid), dim3(GEMM_THREADS), (size_t)smem, st, mw, mh, ml,
+                    g);
 }
 
 }  // namespace
@@ -270,6 +536,16 @@ int tc_bn_for(int M) {
 
 bool tc_supported(int N, int K) { return N % 128 == 0 && K % BK == 0 && K >= BK; }
 
+// Partial planes the stream-K split needs: the most CTAs any tile spans.
+static int planes_for(long long tiles, int n_kb, long long L) {
+    int most = 1;
+    for (long long t = 0; t < tiles; ++t) {
+        const long long c0 = t * n_kb / L, c1 = ((t + 1) * n_kb - 1) / L;
+        if (c1 - c0 + 1 > most) most = (int)(c1 - c0 + 1);
+    }
+    return most;
+}
+
 TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes) {
     TcPlan p;
     p.bn = tc_bn_for(M);
@@ -277,21 +553,66 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes) {
     p.n_tiles = N / 128;
     p.n_kb = K / BK;
     const int tiles = p.m_tiles * p.n_tiles;
+    // Tile kernel: split K until one wave of CTAs covers the SMs (>= 2 k-blocks
+    // per split, partials within the buffer).
     int S = 1;
     if (tiles < n_sm) {
         S = n_sm / tiles;
-        const int max_s = p.n_kb / 2 > 0 ? p.n_kb / 2 : 1;  // >= 2 k-blocks per split
+        const int max_s = p.n_kb / 2 > 0 ? p.n_kb / 2 : 1;
         if (S > max_s) S = max_s;
     }
     while (S > 1 && (size_t)S * M * N * sizeof(float) > y_capacity_bytes) --S;
     p.kb_per_split = ceil_div(p.n_kb, S);
     p.splits = ceil_div(p.n_kb, p.kb_per_split);  // no empty split
+    p.persistent = false;
+    p.grid = tiles * p.splits;
+    p.units_per_cta = p.kb_per_split;
+    // Persistent stream-K when the tile kernel's last wave would leave more
+    // than a fifth of the SMs idle and the extra partial planes are cheap
+    // (estimates in units of one CTA's k-block time, 16 KB of weights).
+    const int waves = ceil_div(tiles * p.splits, n_sm);
+    const double fill = (double)tiles * p.splits / ((double)waves * n_sm);
+    if (waves > 1 && fill < 0.8) {
+        const long long U = (long long)tiles * p.n_kb;
+        long long L = (U + n_sm - 1) / n_sm;
+        if (L < 2) L = 2;
+        const int planes = planes_for(tiles, p.n_kb, L);
+        const double plane_units = 2.0 * (double)M * N * 4.0 / ((double)n_sm * 16384.0);
+        const double cost_tile = (double)waves * (p.kb_per_split + 4);
+        const double cost_pk = (double)L + 4.0 + planes * plane_units;
+        if (cost_pk < cost_tile && (size_t)planes * M * N * sizeof(float) <= y_capacity_bytes) {
+            p.persistent = true;
+            p.units_per_cta = (int)L;
+            p.splits = planes;
+            p.grid = (int)((U + L - 1) / L);
+        }
+    }
     return p;
 }
 
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
                            float *y, int *status, cudaStream_t st) {
+    if (p.persistent) {
+        PkArgs g;
+        g.M = M;
+        g.N = N;
+        g.n_kb = p.n_kb;
+        g.m_tiles = p.m_tiles;
+        g.tiles = p.m_tiles * p.n_tiles;
+        g.L = p.units_per_cta;
+        g.planes = p.splits;
+        g.y = y;
+        g.plane_stride = (size_t)M * N;
+        g.status = status;
+        switch (p.bn) {
+        case 16: return launch_pk<16>(map_w, map_xhi, map_xlo, g, p.grid, st);
+        case 32: return launch_pk<32>(map_w, map_xhi, map_xlo, g, p.grid, st);
+        case 64: return launch_pk<64>(map_w, map_xhi, map_xlo, g, p.grid, st);
+        case 128: return launch_pk<128>(map_w, map_xhi, map_xlo, g, p.grid, st);
+        default: return cudaErrorInvalidValue;
+        }
+    }
     TcArgs g;
     g.M = M;
     g.N = N;
@@ -303,10 +624,10 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
     g.status = status;
     dim3 grid(p.m_tiles, p.n_tiles, p.splits);
     switch (p.bn) {
-    case 16: return launch_bn<16>(map_w, map_xhi, map_xlo, g, grid, st);
-    case 32: return launch_bn<32>(map_w, map_xhi, map_xlo, g, grid, st);
-    case 64: return launch_bn<64>(map_w, map_xhi, map_xlo, g, grid, st);
-    case 128: return launch_bn<128>(map_w, map_xhi, map_xlo, g, grid, st);
+    case 16: return launch_tile<16>(map_w, map_xhi, map_xlo, g, grid, st);
+    case 32: return launch_tile<32>(map_w, map_xhi, map_xlo, g, grid, st);
+    case 64: return launch_tile<64>(map_w, map_xhi, map_xlo, g, grid, st);
+    case 128: return launch_tile<128>(map_w, map_xhi, map_xlo, g, grid, st);
     default: return cudaErrorInvalidValue;
     }
 }

@@ -295,6 +295,90 @@ def generate(spec: WorkloadSpec) -> Workload:
     return Workload(spec, weights, cache, seq_ids, rows)
 
 
+@dataclasses.dataclass
+class DeviceWorkload:
+    """A paged workload whose K/V pools live only on the device (see
+    generate_on_device).  Host side: lengths, page table, weights, rows."""
+    spec: WorkloadSpec
+    weights: Weights
+    seq_lens: np.ndarray      # int32 [B]
+    page_table: np.ndarray    # int32 [B][max_pages]
+    n_pages: int
+    k_pool: object            # torch int16 (bf16 bits) [n_pages][Hkv][P][dh] on the device
+    v_pool: object
+    seq_ids: np.ndarray
+    rows: Optional[np.ndarray]
+
+    @property
+    def shape(self) -> Shape:
+        return self.spec.shape
+
+    def host_cache(self, ids) -> KVCache:
+        """The sequences `ids` copied back into a host paged cache (renumbered
+        0..len(ids)-1, pages compacted) for a CPU consumer."""
+        import torch
+        ids = [int(i) for i in ids]
+        P = self.shape.page_size
+        lens = self.seq_lens[ids].astype(np.int32)
+        n_seq_pages = [(int(L) + P - 1) // P for L in lens]
+        max_pages = max(1, max(n_seq_pages) if n_seq_pages else 1)
+        phys = [self.page_table[i, :n] for i, n in zip(ids, n_seq_pages)]
+        flat = np.concatenate(phys) if phys else np.zeros(0, np.int32)
+        sel = torch.as_tensor(flat.astype(np.int64), device=self.k_pool.device)
+        k = self.k_pool.index_select(0, sel).cpu().numpy().view(np.uint16) if len(flat) else None
+        v = self.v_pool.index_select(0, sel).cpu().numpy().view(np.uint16) if len(flat) else None
+        hkv, dh = self.shape.n_kv_heads, self.shape.head_dim
+        if k is None:
+            k = np.zeros((1, hkv, P, dh), np.uint16)
+            v = np.zeros_like(k)
+        table = np.full((len(ids), max_pages), -1, dtype=np.int32)
+        base = 0
+        for j, n in enumerate(n_seq_pages):
+            table[j, :n] = np.arange(base, base + n, dtype=np.int32)
+            base += n
+        return KVCache(LAYOUT_PAGED, BF16, lens, k_pool=k, v_pool=v, page_table=table, page_size=P)
+
+
+def generate_on_device(spec: WorkloadSpec, device="cuda", weights: Optional[Weights] = None
+                       ) -> DeviceWorkload:
+    """A paged bf16 workload too large to draw on the host: lengths, page
+    permutation, weights and rows come from the same numpy streams as
+    generate(spec); the K/V values are N(0, 1) drawn on the device by a torch
+    generator seeded from the cache stream (so they differ from generate()'s
+    values but follow the same distribution)."""
+    import torch
+    assert spec.layout == LAYOUT_PAGED and spec.shape.kv_dtype == BF16
+    ss = np.random.SeedSequence(spec.seed)
+    s_struct, s_w, s_kv, s_rows = ss.spawn(4)
+    rng_struct = np.random.default_rng(s_struct)
+    lens = draw_lengths(spec, rng_struct)
+    if weights is None:
+        weights = draw_weights(spec.shape, np.random.default_rng(s_w), spec.head_bias)
+    sh = spec.shape
+    P = sh.page_size
+    n_seq_pages = [(int(L) + P - 1) // P for L in lens]
+    n_pages = int(sum(n_seq_pages))
+    max_pages = max(1, max(n_seq_pages) if n_seq_pages else 1)
+    perm = rng_struct.permutation(n_pages).astype(np.int32)
+    table = np.full((len(lens), max_pages), -1, dtype=np.int32)
+    base = 0
+    for b, n in enumerate(n_seq_pages):
+        table[b, :n] = perm[base:base + n]
+        base += n
+    gen = torch.Generator(device=device)
+    gen.manual_seed(int(np.random.default_rng(s_kv).integers(0, 2**62)))
+    shape4 = (max(n_pages, 1), sh.n_kv_heads, P, sh.head_dim)
+    k_pool = torch.randn(shape4, generator=gen, device=device, dtype=torch.float32).to(torch.bfloat16)
+    v_pool = torch.randn(shape4, generator=gen, device=device, dtype=torch.float32).to(torch.bfloat16)
+    rows = None
+    if spec.rows_per_seq:
+        rows = _normal(np.random.default_rng(s_rows), (spec.batch, sh.k_rows, sh.d_model), 0.02,
+                       sh.w_dtype)
+    return DeviceWorkload(spec, weights, lens.astype(np.int32), table, n_pages,
+                          k_pool.view(torch.int16), v_pool.view(torch.int16),
+                          np.arange(spec.batch, dtype=np.int32), rows)
+
+
 def contiguous_to_paged(cache: KVCache, page_size: int, seed: int) -> KVCache:
     """Re-lay a contiguous cache into shuffled pages holding the same values."""
     assert cache.layout == LAYOUT_CONTIGUOUS

@@ -11,7 +11,11 @@ pytestmark = pytest.mark.gpu
 
 SHAPES = [(1, 128, 64), (5, 256, 192), (16, 128, 2560), (17, 384, 640), (64, 128, 128),
           (100, 256, 4096), (128, 6144, 2560), (129, 128, 256), (300, 256, 1024),
-          (1024, 512, 4096)]
+          (1024, 512, 4096),
+          # tile counts that fill the SMs badly take the persistent stream-K
+          # schedule (two partial planes, zero-filled where a tile has one
+          # segment; several row tiles)
+          (1, 24576, 4096), (20, 20480, 256), (512, 6144, 4096)]
 
 
 def run(M, N, K, path, seed):

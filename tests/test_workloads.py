@@ -1,5 +1,6 @@
 """Host logic of the seeded input generator (no method arithmetic)."""
 import numpy as np
+import pytest
 
 from paper_2608_28099_gb300 import workloads as wl
 
@@ -45,3 +46,29 @@ def test_named_shapes():
     s = wl.named("sweep_B8_L2048_k4_C16")
     assert (s.batch, s.len_lo, s.len_hi, s.shape.k_rows, s.shape.n_classes) == (8, 1536, 2560, 4, 16)
     assert len(wl.SWEEP_POINTS) == 160
+
+
+def test_device_generator_matches_host_structure():
+    """The device-drawn sweep inputs share lengths, page table, weights and rows
+    with generate(); host_cache() hands back exactly the pooled pages."""
+    torch = pytest.importorskip("torch")
+    spec = wl.named("sweep_B8_L512_k4_C2", rows_per_seq=True)
+    host = wl.generate(spec)
+    dev = wl.generate_on_device(spec, device="cpu")
+    assert np.array_equal(dev.seq_lens, host.cache.seq_lens)
+    assert np.array_equal(dev.page_table, host.cache.page_table)
+    assert dev.n_pages == host.cache.n_pages
+    assert np.array_equal(dev.weights.w_down, host.weights.w_down)
+    assert np.array_equal(dev.rows, host.rows)
+    ids = [5, 2]
+    hc = dev.host_cache(ids)
+    kp = dev.k_pool.numpy().view(np.uint16)
+    for j, b in enumerate(ids):
+        L = int(dev.seq_lens[b])
+        assert hc.seq_lens[j] == L
+        for t in range(0, L, 7):
+            src = kp[dev.page_table[b, t // 16], :, t % 16, :]
+            assert np.array_equal(hc.k_pool[hc.page_table[j, t // 16], :, t % 16, :], src)
+    # N(0, 1) values
+    vals = wl.bf16_bits_to_f32(kp[:64].reshape(-1))
+    assert abs(float(vals.mean())) < 0.05 and abs(float(vals.std()) - 1.0) < 0.05
