@@ -45,7 +45,7 @@ FLUSH_BYTES = 256 << 20
 
 # DRAM traffic per launch of the dominant kernel from an ncu capture of the same
 # kernel build (profiles/); None until one is taken for the current kernel.
-TRAFFIC_BYTES = {("4b", "attention"): 77_590_400}  # dram read + write per launch, ncu, 2 launches
+TRAFFIC_BYTES = {}
 
 
 def parse_args():

@@ -186,14 +186,31 @@ size_t max_attention_ws(const sp_config &c, int n_sm, int forced_split) {
 
 // Enqueue the attention step (split units + merge) for AttnArgs with the
 // partial buffers taken from `ws`.
+// Largest split count whose merge runs inside the tensor-core attention kernel.
+constexpr int kFusedMergeSplits = 2;
+
+// The merge counters of the attention workspace: [B][Hkv] ints after the partials.
+int *attention_counters(void *ws, int B, int Hkv, int R, int dh, int n_splits) {
+    const size_t units = (size_t)B * Hkv * n_splits * 2;
+    return (int *)((char *)ws + align256(units * R * dh * sizeof(float)) +
+                   align256(units * R * 2 * sizeof(float)));
+}
+
+// Enqueue the attention step (split units, then the merge: inside the
+// tensor-core kernel, or a separate kernel on the CUDA-core path) for AttnArgs
+// with the partial buffers taken from `ws`.  counters_zeroed: the preceding
+// kernel of this stream cleared the merge counters (else they are cleared here).
 sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_path, int *launches,
-                            cudaStream_t st, cudaEvent_t *ev_attn = nullptr,
+                            cudaStream_t st, bool counters_zeroed, cudaEvent_t *ev_attn = nullptr,
                             cudaEvent_t *ev_merge = nullptr) {
     const size_t need = attention_workspace_bytes(a.B, a.Hkv, a.R, a.dh, a.n_splits);
     if (ws_bytes < need) return fail(SP_ERR_INVALID_ARG, "attention workspace too small (%zu < %zu)", ws_bytes, need);
     a.part_o = (float *)ws;
     a.part_ml = (float *)((char *)ws + align256((size_t)a.B * a.Hkv * a.n_splits * 2 * a.R * a.dh *
                                                  sizeof(float)));
+    // the merge runs inside the tensor-core kernel for up to kFusedMergeSplits units
+    // per (sequence, kv head); beyond that a separate kernel spreads it over the GPU
+    a.counters = attention_counters(ws, a.B, a.Hkv, a.R, a.dh, a.n_splits);
     bool tc = attn_path != 1 && attention_tc_supported(a);
     CUtensorMap mk, mv;
     const CUtensorMap *pk = nullptr, *pv = nullptr;
@@ -209,7 +226,11 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
     if (attn_path == 2 && !tc)
         return fail(SP_ERR_UNSUPPORTED, "tensor-core attention needs head_dim 128, a bf16 cache "
                                         "and at most 128 query rows per kv head");
-    a.subs = tc ? 2 : 1;
+    a.subs = 1;  // one partial per unit on both paths
+    const bool fused = tc && a.n_splits <= kFusedMergeSplits;
+    if (!fused) a.counters = nullptr;
+    if (fused && !counters_zeroed)
+        SP_CUDA(cudaMemsetAsync(a.counters, 0, (size_t)a.B * a.Hkv * sizeof(int), st));
     if (ev_attn) cudaEventRecordWithFlags(ev_attn[0], st, cudaEventRecordExternal);
     if (tc)
         SP_CUDA(launch_attention_tc(a, pk, pv, mq, st));
@@ -217,9 +238,9 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
         SP_CUDA(launch_attention_simt(a, st));
     if (ev_attn) cudaEventRecordWithFlags(ev_attn[1], st, cudaEventRecordExternal);
     if (ev_merge) cudaEventRecordWithFlags(ev_merge[0], st, cudaEventRecordExternal);
-    SP_CUDA(launch_attention_merge(a, st));
+    if (!fused) SP_CUDA(launch_attention_merge(a, st));
     if (ev_merge) cudaEventRecordWithFlags(ev_merge[1], st, cudaEventRecordExternal);
-    *launches += 2;
+    *launches += fused ? 1 : 2;
     return SP_OK;
 }
 
@@ -492,6 +513,11 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     r.rope_cs = h->rope_cs;
     r.q = h->q; r.k_new = h->k_new; r.v_new = h->v_new;
     r.status = h->status;
+    // the attention's merge counters for this call's plan
+    int split_tokens = 0, n_splits = 0;
+    plan_attention(batch, hkv, k, c.max_seq_len, h->opt_split, h->n_sm, &split_tokens, &n_splits);
+    r.zero_ints = attention_counters(h->attn_ws, batch, hkv, G * k, dh, n_splits);
+    r.n_zero = batch * hkv;
     mark(SP_STAGE_ROPE, 0);
     SP_CUDA(launch_qkv_rope(r, st));
     mark(SP_STAGE_ROPE, 1);
@@ -502,7 +528,8 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     memset(&a, 0, sizeof a);
     a.B = batch; a.Hq = hq; a.Hkv = hkv; a.dh = dh; a.k = k; a.G = G; a.R = G * k;
     a.kv_bf16 = c.kv_dtype == SP_BF16;
-    plan_attention(batch, hkv, k, c.max_seq_len, h->opt_split, h->n_sm, &a.split_tokens, &a.n_splits);
+    a.split_tokens = split_tokens;
+    a.n_splits = n_splits;
     a.max_seq_len = c.max_seq_len;
     a.seq_ids = d_seq_ids; a.seq_lens = d_seq_lens; a.lens_by_batch = lens_by_batch;
     a.kv = to_dev(kv);
@@ -511,7 +538,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     a.gathered = nullptr;
     a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
     a.out = h->o.out(tc_o);
-    s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, &launches, st,
+    s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, &launches, st, true,
                           h->opt_profile ? h->ev[SP_STAGE_ATTN] : nullptr,
                           h->opt_profile ? h->ev[SP_STAGE_MERGE] : nullptr);
     if (s != SP_OK) return s;
@@ -656,7 +683,7 @@ sp_status sp_attend(sp_stream stream, const sp_attn_dims *dm, int batch, const i
     if (dm->path < 0 || dm->path > 2) return fail(SP_ERR_INVALID_ARG, "bad attention path");
     int launches = 0;
     return enqueue_attention(a, d_workspace, workspace_bytes, dm->path, &launches,
-                             (cudaStream_t)stream);
+                             (cudaStream_t)stream, false);
 }
 
 size_t sp_project_workspace_bytes(int M, int N, int K) {

@@ -271,7 +271,8 @@ size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits) {
     const size_t units = (size_t)B * Hkv * n_splits * 2;  // up to two partials per unit
     size_t o = units * R * dh * sizeof(float);
     o = (o + 255) & ~(size_t)255;
-    return o + ((units * R * 2 * sizeof(float) + 255) & ~(size_t)255);
+    o += (units * R * 2 * sizeof(float) + 255) & ~(size_t)255;
+    return o + (((size_t)B * Hkv * sizeof(int) + 255) & ~(size_t)255);  // merge counters
 }
 
 cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st) {

@@ -19,8 +19,12 @@
 //   O_w  += P_i V_i           P written as bf16 over the first half of S_w (A
 //                             operand from TMEM), V read in place from shared
 //                             memory as an MN-major B operand
-// Each warpgroup keeps its own (max, sum, O_w) and writes its own partial, so
-// a work unit yields two partials that the merge combines like splits.  The
+// Each warpgroup keeps its own (max, sum, O_w); at the end warpgroup 0 folds
+// warpgroup 1's state into its own (both O accumulators sit on the same TMEM
+// lanes) and writes the unit's one partial.  The last unit of a (sequence, kv
+// head) to finish (a counter per pair, cleared by the preceding kernel)
+// combines the pair's partials in the exp2 domain and writes the output; with
+// many units per pair the host leaves that to attn_merge_kernel instead.  The
 // even and odd tiles form two independent pipelines, each with its own MMA
 // issuing warp: one thread issuing small-N MMAs back to back leaves the tensor
 // pipe idle between them, two keep it busy.
@@ -67,7 +71,8 @@ constexpr int OFF_KV = 0;
 constexpr int MAX_SPLIT_PAGES = 1024;          // page ids of one split staged in smem
 constexpr int OFF_PAGES = OFF_KV + STG * KV_STAGE;
 constexpr int OFF_BAR = OFF_PAGES + MAX_SPLIT_PAGES * 4;
-constexpr int SMEM_BYTES = OFF_BAR + 256 + 1024;
+constexpr int OFF_ML = OFF_BAR + 256;           // warpgroup 1's (max, sum) per row
+constexpr int SMEM_BYTES = OFF_ML + 1024 + 1024;
 constexpr int THREADS = 384;                   // 2 softmax warpgroups, 2 producers, 2 MMA
 constexpr int PRODUCER_WARP = 8, MMA_WARP = 9, MMA_WARP1 = 10, PRODUCER_WARP1 = 11;
 constexpr float RESCALE_LOG2 = 8.f;            // tolerate p <= 2^8 before rescaling O
@@ -92,6 +97,7 @@ struct Bars {
     uint64_t kv_full[STG], kv_empty[STG], s_full[2], p_full[2], pv_done[2], fin, q_full;  // fin: 2 arrivals
     uint32_t tmem;
     int abort;
+    int last;  // this CTA merges its (sequence, kv head)
 };
 
 __global__ void __launch_bounds__(THREADS, 1)
@@ -481,33 +487,53 @@ __global__ void __launch_bounds__(THREADS, 1)
             tc_fence_before();
             mbar_arrive(&bars->p_full[wg]);
         }
-        // epilogue: this warpgroup's unnormalised partial of the unit
-        const int my_last = (n_tiles - 1 - wg) >= 0 ? n_tiles - 1 - ((n_tiles - 1 - wg) & 1) : -1;
-        const size_t unit = (((size_t)b * a.Hkv + g) * a.n_splits + s_idx) * 2 + wg;
-        float *po = a.part_o + (unit * R + row) * DH;
-        if (my_last < 0) {
-            // no tile for this warpgroup: an empty partial
-            if (active) {
-                for (int c = 0; c < DH; c += 4) *(float4 *)(po + c) = make_float4(0.f, 0.f, 0.f, 0.f);
-                a.part_ml[(unit * R + row) * 2] = -INFINITY;
-                a.part_ml[(unit * R + row) * 2 + 1] = 0.f;
-            }
-        } else if (ok && mbar_wait(&bars->pv_done[wg], (my_last >> 1) & 1, abort)) {
-            tc_fence_after();
+        // epilogue: warpgroup 1 hands its (max, sum) to warpgroup 0 through shared
+        // memory; warpgroup 0 combines (max, sum, O) of both and writes the unit's
+        // unnormalised partial
+        float *sm_ml = (float *)(smem + OFF_ML);
+        const int last0 = n_tiles >= 1 ? n_tiles - 1 - ((n_tiles - 1) & 1) : -1;  // WG0's last tile
+        const int last1 = n_tiles >= 2 ? n_tiles - 1 - (n_tiles & 1) : -1;        // WG1's last tile
+        if (wg == 1) {
+            sm_ml[row] = last1 >= 0 ? m : -INFINITY;
+            sm_ml[128 + row] = last1 >= 0 ? l : 0.f;
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(64 * act_warps) : "memory");
+        if (wg == 0) {
+            const size_t unit = ((size_t)b * a.Hkv + g) * a.n_splits + s_idx;
+            float *po = a.part_o + (unit * R + row) * DH;
+            const float m1 = sm_ml[row], l1 = sm_ml[128 + row];
+            const float mc = fmaxf(m, m1);
+            const float a0 = (m == -INFINITY) ? 0.f : fast_exp2(m - mc);
+            const float a1 = (m1 == -INFINITY) ? 0.f : fast_exp2(m1 - mc);
+            bool have = ok && last0 >= 0 && mbar_wait(&bars->pv_done[0], (last0 >> 1) & 1, abort);
+            if (have && last1 >= 0) have = mbar_wait(&bars->pv_done[1], (last1 >> 1) & 1, abort);
+            have = __all_sync(0xffffffffu, have);  // the TMEM loads below are warp-collective
+            if (have) {
+                tc_fence_after();
 #pragma unroll 1
-            for (int c0 = 0; c0 < DH; c0 += 32) {
-                float o32[32];
-                tmem_ld32(lane_base + o_col + c0, o32);
-                if (active) {
+                for (int c0 = 0; c0 < DH; c0 += 32) {
+                    float o0[32], o1[32];
+                    tmem_ld32(lane_base + O_COL + c0, o0);
+                    if (last1 >= 0) {
+                        tmem_ld32(lane_base + O_COL + DH + c0, o1);
+                    } else {
 #pragma unroll
-                    for (int j = 0; j < 32; j += 4)
-                        *(float4 *)(po + c0 + j) = make_float4(o32[j], o32[j + 1], o32[j + 2], o32[j + 3]);
+                        for (int j = 0; j < 32; ++j) o1[j] = 0.f;
+                    }
+                    if (active) {
+#pragma unroll
+                        for (int j = 0; j < 32; j += 4)
+                            *(float4 *)(po + c0 + j) =
+                                make_float4(a0 * o0[j] + a1 * o1[j], a0 * o0[j + 1] + a1 * o1[j + 1],
+                                            a0 * o0[j + 2] + a1 * o1[j + 2], a0 * o0[j + 3] + a1 * o1[j + 3]);
+                    }
+                }
+                if (active) {
+                    a.part_ml[(unit * R + row) * 2] = mc;
+                    a.part_ml[(unit * R + row) * 2 + 1] = a0 * l + a1 * l1;
                 }
             }
-            if (active) {
-                a.part_ml[(unit * R + row) * 2] = m;
-                a.part_ml[(unit * R + row) * 2 + 1] = l;
-            }
+            __threadfence();  // the partial is visible device-wide before this unit is counted
         }
     }
     // every MMA must be finished before TMEM and shared memory go away
@@ -516,6 +542,55 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
     if (threadIdx.x == 0 && *abort && a.status) atomicOr(a.status, SP_DEV_TIMEOUT);
     if (warp == MMA_WARP) tmem_dealloc(tmem, TMEM_COLS);
+
+    // ---------------------------------------------------------------- merge
+    if (!a.counters) return;  // merged by a separate kernel
+    const int n_units = min(a.n_splits, ceil_div(total, a.split_tokens));
+    int *counter = a.counters + (size_t)b * a.Hkv + g;
+    if (threadIdx.x == 0) {
+        bars->last = atomicAdd(counter, 1) == n_units - 1;
+        __threadfence();
+    }
+    __syncthreads();
+    if (!bars->last) return;
+    // every unit of the pair has written its partial: combine them.  Pass 1: per
+    // row, the normalised weight of each partial (shared memory, over the
+    // free K/V ring); pass 2: per (row, 4 columns), the weighted sum.
+    const size_t p0 = ((size_t)b * a.Hkv + g) * a.n_splits;
+    float *wn = (float *)(smem + OFF_KV);  // [R][n_units]
+    for (int rr = threadIdx.x; rr < R; rr += THREADS) {
+        float mmax = -INFINITY;
+#pragma unroll 8
+        for (int p = 0; p < n_units; ++p) mmax = fmaxf(mmax, __ldcg(a.part_ml + ((p0 + p) * R + rr) * 2));
+        float l = 0.f;
+#pragma unroll 8
+        for (int p = 0; p < n_units; ++p) {
+            const float2 ml = __ldcg((const float2 *)(a.part_ml + ((p0 + p) * R + rr) * 2));
+            const float w = (ml.x == -INFINITY) ? 0.f : exp2f(ml.x - mmax);
+            wn[rr * n_units + p] = w;
+            l += w * ml.y;
+        }
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        for (int p = 0; p < n_units; ++p) wn[rr * n_units + p] *= inv;
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < R * (DH / 4); idx += THREADS) {
+        const int rr = idx / (DH / 4), c = (idx % (DH / 4)) * 4;
+        float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+        for (int p = 0; p < n_units; ++p) {
+            const float w = wn[rr * n_units + p];
+            const float4 op = __ldcg((const float4 *)(a.part_o + ((p0 + p) * R + rr) * DH + c));
+            o.x += w * op.x;
+            o.y += w * op.y;
+            o.z += w * op.z;
+            o.w += w * op.w;
+        }
+        const int hl = rr / k, r = rr - hl * k;
+        const int h = g * a.G + hl;
+        act_store4(a.out, (((size_t)b * k + r) * a.Hq + h) * DH + c, o);
+    }
+    if (threadIdx.x == 0) *counter = 0;  // ready for a launch that does not clear it
 }
 
 }  // namespace

@@ -202,9 +202,12 @@ struct AttnArgs {
     const float *q;               // [B][k][Hq][dh], rotated
     const float *k_new;           // [B][k][Hkv][dh], rotated
     const float *v_new;           // [B][k][Hkv][dh]
-    int subs;                     // partials per work unit (1 CUDA-core, 2 tensor-core)
+    int subs;                     // partials per work unit (1)
     float *part_o;                // [B][Hkv][n_splits][subs][R][dh], unnormalised
     float *part_ml;               // [B][Hkv][n_splits][subs][R][2] (max in log2 units, sum)
+    int *counters;                // [B][Hkv] finished units, zero before the launch, or NULL:
+                                  // the tensor-core kernel's last unit of a (sequence, kv head)
+                                  // merges; NULL leaves the merge to attn_merge_kernel
     int *status;
     int *gathered;                // [B][max_pages] or NULL
     float scale_log2;             // log2(e) / sqrt(dh)
@@ -242,6 +245,8 @@ struct QkvRopeArgs {
     const float2 *rope_cs;   // [max_seq_len + k][dh/2] (cos, sin)
     float *q, *k_new, *v_new;
     int *status;
+    int *zero_ints;          // optional: n_zero ints cleared for the next kernel
+    int n_zero;
 };
 cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st);
 

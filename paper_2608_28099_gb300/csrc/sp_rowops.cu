@@ -67,6 +67,8 @@ __global__ void __launch_bounds__(256) rmsnorm_rows_kernel(const T *__restrict__
 __global__ void qkv_rope_kernel(QkvRopeArgs a) {
     pdl_trigger();
     pdl_wait();
+    if (a.zero_ints && blockIdx.x == 0 && blockIdx.y == 0)
+        for (int t = threadIdx.x; t < a.n_zero; t += blockDim.x) a.zero_ints[t] = 0;
     const int m = blockIdx.y;
     const int b = m / a.k, r = m % a.k;
     const int dh = a.dh, half = dh >> 1;
