@@ -7,9 +7,11 @@
 // the instruction instead of wasting 7/8 of a 128-row M tile.  Both operands
 // arrive by TMA in 128-byte swizzled K-major tiles through mbarrier rings.
 //
-// Activations come as two bf16 planes hi = rn(x), lo = rn(x - hi); every
-// k-block issues W*hi and W*lo into the same accumulator, so the product
-// carries ~16 bits of the activation's mantissa for the price of a second MMA.
+// Activations come as two bf16 planes hi = rn(x), lo = rn(x - hi), stored one
+// after the other in each stage, so [hi; lo] is a single B operand of 2 BN rows:
+// one MMA of N = 2 BN per 16-wide k-step reads the weight tile once and leaves
+// W hi^T in TMEM columns [0, BN) and W lo^T in [BN, 2 BN); the epilogue adds
+// the halves.  The product carries ~16 bits of the activation's mantissa.
 //
 // Two schedules, fp32 partials in planes of Y that the consumers add:
 //  * tile kernel: one CTA per (tile, K split); split-K when the tiles alone
@@ -46,7 +48,7 @@ struct TileCfg {
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE = A_BYTES + 2 * B_BYTES;
     static constexpr int STAGES = (BN <= 32) ? 8 : (BN == 64 ? 6 : 4);
-    static constexpr int TMEM_COLS = BN < 32 ? 32 : BN;
+    static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;  // hi and lo halves
     static constexpr int SMEM = STAGES * STAGE + 1024 /*align*/ + 256 /*barriers*/;
 };
 
@@ -129,7 +131,7 @@ __global__ void __launch_bounds__(128, 1)
         }
     } else if (warp == 1 && lane == 0) {
         // MMA issuer
-        constexpr uint32_t idesc = idesc_bf16_f32(128, BN);
+        constexpr uint32_t idesc = idesc_bf16_f32(128, 2 * BN);
         for (int i = 0; i < nkb; ++i) {
             const int s = i % Cfg::STAGES;
             const uint32_t ph = (i / Cfg::STAGES) & 1;
@@ -137,13 +139,11 @@ __global__ void __launch_bounds__(128, 1)
             tc_fence_after();
             uint8_t *st = smem + s * Cfg::STAGE;
             const uint64_t a = sw128_kmajor_desc(st);
-            const uint64_t bh = sw128_kmajor_desc(st + A_BYTES);
-            const uint64_t bl = sw128_kmajor_desc(st + A_BYTES + Cfg::B_BYTES);
+            const uint64_t bh = sw128_kmajor_desc(st + A_BYTES);  // [hi; lo], 2 BN rows
 #pragma unroll
             for (int kk = 0; kk < BK / 16; ++kk) {
                 // +32 bytes along K per 16-element MMA step (encoded >> 4)
                 mma_bf16(tmem, a + 2 * kk, bh + 2 * kk, idesc, (i > 0 || kk > 0) ? 1u : 0u);
-                mma_bf16(tmem, a + 2 * kk, bl + 2 * kk, idesc, 1u);
             }
             mma_commit(&empty[s]);
         }
@@ -160,22 +160,24 @@ __global__ void __launch_bounds__(128, 1)
         float *y = g.y + (size_t)blockIdx.z * g.split_stride;
         const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
         if constexpr (BN == 16) {
-            float v[16];
+            float v[16], u[16];
             tmem_ld16(trow, v);
+            tmem_ld16(trow + 16, u);
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
                 const int m = m0 + j;
-                if (m < g.M) y[(size_t)m * g.N + n] = v[j];
+                if (m < g.M) y[(size_t)m * g.N + n] = v[j] + u[j];
             }
         } else {
 #pragma unroll 1
             for (int c0 = 0; c0 < BN; c0 += 32) {
-                float v[32];
+                float v[32], u[32];
                 tmem_ld32(trow + c0, v);
+                tmem_ld32(trow + BN + c0, u);
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
                     const int m = m0 + c0 + j;
-                    if (m < g.M) y[(size_t)m * g.N + n] = v[j];
+                    if (m < g.M) y[(size_t)m * g.N + n] = v[j] + u[j];
                 }
             }
         }
@@ -216,8 +218,8 @@ struct PkCfg {
     static constexpr int X_STAGE = 2 * B_BYTES;       // hi + lo
     static constexpr int W_STAGES = BN <= 32 ? 8 : (BN == 64 ? 6 : 5);
     static constexpr int X_STAGES = BN <= 32 ? 4 : 3;
-    static constexpr int ACC_COLS = BN < 32 ? 32 : BN;
-    static constexpr int TMEM_COLS = 2 * ACC_COLS;
+    static constexpr int ACC_COLS = 2 * BN < 32 ? 32 : 2 * BN;  // hi and lo halves
+    static constexpr int TMEM_COLS = 2 * ACC_COLS;              // double-buffered
     static constexpr int OFF_X = W_STAGES * A_BYTES;
     static constexpr int OFF_BAR = OFF_X + X_STAGES * X_STAGE;
     static constexpr int SMEM = OFF_BAR + 512 /*barriers*/ + 1024 /*align*/;
@@ -349,7 +351,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             }
         }
     } else if (warp == MMA_WARP_G && lane == 0) {
-        constexpr uint32_t idesc = idesc_bf16_f32(128, BN);
+        constexpr uint32_t idesc = idesc_bf16_f32(128, 2 * BN);
         int i = 0, sgi = 0;
         bool ok = true;
         for (int t = t_first; ok && t <= t_last; ++t, ++sgi) {
@@ -369,13 +371,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 tc_fence_after();
                 const uint8_t *xs = smem + Cfg::OFF_X + sx * Cfg::X_STAGE;
                 const uint64_t a = sw128_kmajor_desc(smem + sw * A_BYTES);
-                const uint64_t bh = sw128_kmajor_desc(xs);
-                const uint64_t bl = sw128_kmajor_desc(xs + Cfg::B_BYTES);
+                const uint64_t bh = sw128_kmajor_desc(xs);  // [hi; lo], 2 BN rows
 #pragma unroll
                 for (int kk = 0; kk < BK / 16; ++kk) {
                     // +32 bytes along K per 16-element MMA step (encoded >> 4)
                     mma_bf16(acc, a + 2 * kk, bh + 2 * kk, idesc, (kb > sg.kb_lo || kk > 0) ? 1u : 0u);
-                    mma_bf16(acc, a + 2 * kk, bl + 2 * kk, idesc, 1u);
                 }
                 mma_commit(&w_empty[sw]);
                 mma_commit(&x_empty[sx]);
@@ -400,22 +400,24 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             float *y = g.y + (size_t)plane * g.plane_stride;
             const uint32_t ta = trow + (uint32_t)(buf * Cfg::ACC_COLS);
             if constexpr (BN == 16) {
-                float v[16];
+                float v[16], u[16];
                 tmem_ld16(ta, v);
+                tmem_ld16(ta + 16, u);
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
                     const int m = m0 + j;
-                    if (m < g.M) y[(size_t)m * g.N + n] = v[j];
+                    if (m < g.M) y[(size_t)m * g.N + n] = v[j] + u[j];
                 }
             } else {
 #pragma unroll 1
                 for (int c0 = 0; c0 < BN; c0 += 32) {
-                    float v[32];
+                    float v[32], u[32];
                     tmem_ld32(ta + c0, v);
+                    tmem_ld32(ta + BN + c0, u);
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
                         const int m = m0 + c0 + j;
-                        if (m < g.M) y[(size_t)m * g.N + n] = v[j];
+                        if (m < g.M) y[(size_t)m * g.N + n] = v[j] + u[j];
                     }
                 }
             }
