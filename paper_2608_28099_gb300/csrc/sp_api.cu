@@ -178,39 +178,33 @@ size_t max_attention_ws(const sp_config &c, int n_sm, int forced_split) {
     for (int B = 1; B <= c.max_batch; ++B) {
         int split, ns;
         plan_attention(B, c.n_kv_heads, c.k_rows, c.max_seq_len, forced_split, n_sm, &split, &ns);
-        size_t b = attention_workspace_bytes(B, c.n_kv_heads, G * c.k_rows, c.head_dim, ns);
+        size_t b = attention_workspace_bytes(B, c.n_kv_heads, G * c.k_rows, c.head_dim, ns, n_sm);
         if (b > best) best = b;
     }
     return best;
 }
 
-// Enqueue the attention step (split units + merge) for AttnArgs with the
-// partial buffers taken from `ws`.
-// Largest split count whose merge runs inside the tensor-core attention kernel.
-constexpr int kFusedMergeSplits = 2;
+// The merge counters of the attention workspace: [B][Hkv] ints at its start.
+int *attention_counters(void *ws) { return (int *)ws; }
 
-// The merge counters of the attention workspace: [B][Hkv] ints after the partials.
-int *attention_counters(void *ws, int B, int Hkv, int R, int dh, int n_splits) {
-    const size_t units = (size_t)B * Hkv * n_splits * 2;
-    return (int *)((char *)ws + align256(units * R * dh * sizeof(float)) +
-                   align256(units * R * 2 * sizeof(float)));
-}
-
-// Enqueue the attention step (split units, then the merge: inside the
-// tensor-core kernel, or a separate kernel on the CUDA-core path) for AttnArgs
-// with the partial buffers taken from `ws`.  counters_zeroed: the preceding
-// kernel of this stream cleared the merge counters (else they are cleared here).
-sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_path, int *launches,
-                            cudaStream_t st, bool counters_zeroed, cudaEvent_t *ev_attn = nullptr,
-                            cudaEvent_t *ev_merge = nullptr) {
-    const size_t need = attention_workspace_bytes(a.B, a.Hkv, a.R, a.dh, a.n_splits);
+// Enqueue the attention step for AttnArgs with the counters and partial
+// buffers taken from `ws`: the tensor-core kernel (balanced over the SMs, merge
+// inside) or the CUDA-core split kernel followed by its merge kernel.
+// counters_zeroed: the preceding kernel of this stream cleared the merge
+// counters (else they are cleared here).
+sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_path, int n_sm,
+                            int forced_split, int *launches, cudaStream_t st, bool counters_zeroed,
+                            cudaEvent_t *ev_attn = nullptr, cudaEvent_t *ev_merge = nullptr) {
+    a.tc_ctas = attn_tc_ctas(n_sm, a.Hkv);
+    a.tc_min_tiles = forced_split > 0 ? forced_split / 64 : kAttnMinTiles;
+    const size_t need = attention_workspace_bytes(a.B, a.Hkv, a.R, a.dh, a.n_splits, n_sm);
     if (ws_bytes < need) return fail(SP_ERR_INVALID_ARG, "attention workspace too small (%zu < %zu)", ws_bytes, need);
-    a.part_o = (float *)ws;
-    a.part_ml = (float *)((char *)ws + align256((size_t)a.B * a.Hkv * a.n_splits * 2 * a.R * a.dh *
-                                                 sizeof(float)));
-    // the merge runs inside the tensor-core kernel for up to kFusedMergeSplits units
-    // per (sequence, kv head); beyond that a separate kernel spreads it over the GPU
-    a.counters = attention_counters(ws, a.B, a.Hkv, a.R, a.dh, a.n_splits);
+    const size_t pairs = (size_t)a.B * a.Hkv;
+    size_t parts = pairs * a.n_splits;
+    if ((size_t)a.tc_ctas + pairs > parts) parts = (size_t)a.tc_ctas + pairs;
+    a.counters = attention_counters(ws);
+    a.part_o = (float *)((char *)ws + align256(pairs * sizeof(int)));
+    a.part_ml = (float *)((char *)a.part_o + align256(parts * a.R * a.dh * sizeof(float)));
     bool tc = attn_path != 1 && attention_tc_supported(a);
     CUtensorMap mk, mv;
     const CUtensorMap *pk = nullptr, *pv = nullptr;
@@ -221,26 +215,21 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
         pk = &mk;
         pv = &mv;
     }
-    CUtensorMap mq;
-    if (tc) tc = encode_q_group_f32(&mq, a.q, a.B * a.k, a.Hq, a.G, a.k);
     if (attn_path == 2 && !tc)
-        return fail(SP_ERR_UNSUPPORTED, "tensor-core attention needs head_dim 128, a bf16 cache "
-                                        "and at most 128 query rows per kv head");
-    a.subs = 1;  // one partial per unit on both paths
-    const bool fused = tc && a.n_splits <= kFusedMergeSplits;
-    if (!fused) a.counters = nullptr;
-    if (fused && !counters_zeroed)
-        SP_CUDA(cudaMemsetAsync(a.counters, 0, (size_t)a.B * a.Hkv * sizeof(int), st));
+        return fail(SP_ERR_UNSUPPORTED, "tensor-core attention needs head_dim 128, a bf16 cache, "
+                                        "at most 128 query rows per kv head and at most 2048 sequences");
+    a.subs = 1;  // one partial per unit on the CUDA-core path
+    if (tc && !counters_zeroed) SP_CUDA(cudaMemsetAsync(a.counters, 0, pairs * sizeof(int), st));
     if (ev_attn) cudaEventRecordWithFlags(ev_attn[0], st, cudaEventRecordExternal);
     if (tc)
-        SP_CUDA(launch_attention_tc(a, pk, pv, mq, st));
+        SP_CUDA(launch_attention_tc(a, pk, pv, st));
     else
         SP_CUDA(launch_attention_simt(a, st));
     if (ev_attn) cudaEventRecordWithFlags(ev_attn[1], st, cudaEventRecordExternal);
     if (ev_merge) cudaEventRecordWithFlags(ev_merge[0], st, cudaEventRecordExternal);
-    if (!fused) SP_CUDA(launch_attention_merge(a, st));
+    if (!tc) SP_CUDA(launch_attention_merge(a, st));
     if (ev_merge) cudaEventRecordWithFlags(ev_merge[1], st, cudaEventRecordExternal);
-    *launches += fused ? 1 : 2;
+    *launches += tc ? 1 : 2;
     return SP_OK;
 }
 
@@ -516,7 +505,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     // the attention's merge counters for this call's plan
     int split_tokens = 0, n_splits = 0;
     plan_attention(batch, hkv, k, c.max_seq_len, h->opt_split, h->n_sm, &split_tokens, &n_splits);
-    r.zero_ints = attention_counters(h->attn_ws, batch, hkv, G * k, dh, n_splits);
+    r.zero_ints = attention_counters(h->attn_ws);
     r.n_zero = batch * hkv;
     mark(SP_STAGE_ROPE, 0);
     SP_CUDA(launch_qkv_rope(r, st));
@@ -538,7 +527,8 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     a.gathered = nullptr;
     a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
     a.out = h->o.out(tc_o);
-    s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, &launches, st, true,
+    s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, h->n_sm, h->opt_split,
+                          &launches, st, true,
                           h->opt_profile ? h->ev[SP_STAGE_ATTN] : nullptr,
                           h->opt_profile ? h->ev[SP_STAGE_MERGE] : nullptr);
     if (s != SP_OK) return s;
@@ -634,7 +624,8 @@ size_t sp_attend_workspace_bytes(const sp_attn_dims *dm, int batch) {
     plan_attention(batch, dm->n_kv_heads, dm->k_rows, dm->max_seq_len, dm->split_tokens, sm_count(),
                    &split, &ns);
     return attention_workspace_bytes(batch, dm->n_kv_heads,
-                                     (dm->n_q_heads / dm->n_kv_heads) * dm->k_rows, dm->head_dim, ns);
+                                     (dm->n_q_heads / dm->n_kv_heads) * dm->k_rows, dm->head_dim, ns,
+                                     sm_count());
 }
 
 sp_status sp_attend(sp_stream stream, const sp_attn_dims *dm, int batch, const int *d_seq_ids,
@@ -682,8 +673,8 @@ sp_status sp_attend(sp_stream stream, const sp_attn_dims *dm, int batch, const i
     a.out.lo = nullptr;
     if (dm->path < 0 || dm->path > 2) return fail(SP_ERR_INVALID_ARG, "bad attention path");
     int launches = 0;
-    return enqueue_attention(a, d_workspace, workspace_bytes, dm->path, &launches,
-                             (cudaStream_t)stream, false);
+    return enqueue_attention(a, d_workspace, workspace_bytes, dm->path, sm_count(), dm->split_tokens,
+                             &launches, (cudaStream_t)stream, false);
 }
 
 size_t sp_project_workspace_bytes(int M, int N, int K) {

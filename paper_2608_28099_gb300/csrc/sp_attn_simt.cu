@@ -267,12 +267,14 @@ void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, in
     *n_splits = ceil_div(total, chunk);
 }
 
-size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits) {
-    const size_t units = (size_t)B * Hkv * n_splits * 2;  // up to two partials per unit
-    size_t o = units * R * dh * sizeof(float);
-    o = (o + 255) & ~(size_t)255;
-    o += (units * R * 2 * sizeof(float) + 255) & ~(size_t)255;
-    return o + (((size_t)B * Hkv * sizeof(int) + 255) & ~(size_t)255);  // merge counters
+size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits, int n_sm) {
+    const size_t pairs = (size_t)B * Hkv;
+    size_t parts = pairs * n_splits;
+    const size_t tc_slots = (size_t)attn_tc_ctas(n_sm, Hkv) + pairs;
+    if (tc_slots > parts) parts = tc_slots;
+    const auto al = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    return al(pairs * sizeof(int)) + al(parts * R * dh * sizeof(float)) +
+           al(parts * R * 2 * sizeof(float));
 }
 
 cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st) {

@@ -2,12 +2,24 @@
 // (Sec. 3.3, Eq. 1-3) on tcgen05 tensor cores, for head_dim 128, bf16 caches
 // and up to 128 query rows per (sequence, kv head).
 //
-// One CTA = one work unit (split s, kv head g, sequence b), the same units and
-// partial outputs as the CUDA-core kernel, so the same merge follows.  All
-// R = G * k query rows of the KV head's group share every K/V tile: the GQA
-// group and the k soft-prompt rows together form the M side of the MMA.
+// Work balance: the keys of every sequence b are cut into 64-token tiles, and
+// the tiles of all sequences, in order, form one list of T tiles per kv head.
+// The persistent grid holds n groups of Hkv CTAs (n Hkv <= SMs); CTA (j, g)
+// attends kv head g over the equal share [j T / n, (j+1) T / n) of the list,
+// whatever the mix of lengths, so a ragged batch keeps every SM streaming
+// until the end, and the Hkv heads of a token range are read at the same time
+// (a token's keys of all heads sit together in the cache: whole cache rows or
+// pages are read while they are open).  A share crosses sequence boundaries:
+// each piece of a sequence inside it is a segment.  A (sequence, kv head) pair
+// that lies inside one share is finished there (normalised output); otherwise
+// each of its segments leaves an unnormalised partial (max, sum, O) in slot
+// (j + b) Hkv + g (unique: segments are ordered by both j and b), and the CTA
+// that completes the pair's last segment (a counter per pair, zero before the
+// launch) combines the partials in the exp2 domain.
 //
-// Per 64-token tile i (w = i & 1):
+// All R = G * k query rows of the KV head's group share every K/V tile: the
+// GQA group and the k soft-prompt rows together form the M side of the MMA.
+// Per 64-token tile i of a segment (w = i & 1):
 //   S_i   = Q K_i^T           M = 128 query rows, N = 64 tokens, K = 128 dims,
 //                             Q split into bf16 hi + lo held in TMEM (the
 //                             MMA's A operand, two MMAs per step), into TMEM
@@ -19,29 +31,28 @@
 //   O_w  += P_i V_i           P written as bf16 over the first half of S_w (A
 //                             operand from TMEM), V read in place from shared
 //                             memory as an MN-major B operand
-// Each warpgroup keeps its own (max, sum, O_w); at the end warpgroup 0 folds
-// warpgroup 1's state into its own (both O accumulators sit on the same TMEM
-// lanes) and writes the unit's one partial.  The last unit of a (sequence, kv
-// head) to finish (a counter per pair, cleared by the preceding kernel)
-// combines the pair's partials in the exp2 domain and writes the output; with
-// many units per pair the host leaves that to attn_merge_kernel instead.  The
-// even and odd tiles form two independent pipelines, each with its own MMA
-// issuing warp: one thread issuing small-N MMAs back to back leaves the tensor
-// pipe idle between them, two keep it busy.
-// Tiles come from a 6-stage ring: TMA for whole cache tiles of a paged pool
-// (one box per (page, kv head) block of K and of V, issued by two lead warps
-// taking alternate tiles), cp.async for contiguous caches, plain loads for the
-// tile holding the sequence end and the new keys (and for pages that fail the
-// bounds check, which are zero-filled and reported).
+// At the end of a segment warpgroup 0 folds warpgroup 1's state into its own
+// (both O accumulators sit on the same TMEM lanes), writes the output or the
+// partial, and loads the next segment's queries into TMEM.  The even and odd
+// tiles form two independent pipelines, each with its own MMA issuing warp:
+// one thread issuing small-N MMAs back to back leaves the tensor pipe idle
+// between them, two keep it busy.
+// Tiles come from a 6-stage ring that runs across segment boundaries (the K/V
+// stream never drains): TMA for whole cache tiles of a paged pool (one box per
+// (page, kv head) block of K and of V, issued by two lead warps taking
+// alternate tiles), cp.async for contiguous caches, plain loads for the tile
+// holding the sequence end and the new keys.  A page id outside the pool is
+// never dereferenced: its block is zero-filled and the status word records it.
 //
 // Tile layout in shared memory (K and V alike, 64 tokens x 128 dims bf16):
 // [8-token group][dim half][8 tokens][64 dims], 128-byte swizzle, so that a
 // (page, head) block of 16/32/64 tokens is one TMA box and both MMAs read the
 // tile with uniform strides (8-token groups 2048 B apart, dim halves 1024 B).
 //
-// Warps 0-3 and 4-7: the two softmax warpgroups (+ epilogue); warps 8 and 11:
-// producers; warp 9: TMEM owner and MMA issuer of even tiles; warp 10: MMA
-// issuer of odd tiles.  Every wait is time-limited (SP_DEV_TIMEOUT).
+// Warps 0-3 and 4-7: the two softmax warpgroups (+ epilogue, merge); warps 8
+// and 11: producers; warp 9: TMEM owner and MMA issuer of even tiles; warp 10:
+// MMA issuer of odd tiles.  Softmax warps that own no query row (R <= 96)
+// join the producers.  Every wait is time-limited (SP_DEV_TIMEOUT).
 #include <cudaTypedefs.h>
 #include <string.h>
 
@@ -57,21 +68,15 @@ using namespace sm100;
 constexpr int DH = 128;
 constexpr int TT = 64;                         // tokens per tile
 constexpr int STG = 6;                         // K/V ring depth
-// cp.async tiles in flight beyond the current one.  Tile j is published at
-// producer iteration j + DEFER, which first waits for stage j + DEFER - STG to
-// be released; the MMA warp needs tiles 0 and 1 before its first PV and tile
-// i + 2 before it releases stage i + 1, so DEFER <= STG - 2 (else deadlock).
-constexpr int DEFER = STG - 2;
-static_assert(DEFER >= 0 && DEFER <= STG - 2, "cp.async publication depth");
 constexpr int KV_TILE = TT * DH * 2;           // K or V of one tile, 16 KB
 constexpr int KV_STAGE = 2 * KV_TILE;          // K then V
 constexpr uint32_t GROUP_STRIDE = 2048;        // 8-token groups
 constexpr uint32_t HALF_STRIDE = 1024;         // 64-dim halves within a group
+constexpr int MAX_B = 2048;                    // sequences per launch (tile prefix in smem)
 constexpr int OFF_KV = 0;
-constexpr int MAX_SPLIT_PAGES = 1024;          // page ids of one split staged in smem
-constexpr int OFF_PAGES = OFF_KV + STG * KV_STAGE;
-constexpr int OFF_BAR = OFF_PAGES + MAX_SPLIT_PAGES * 4;
-constexpr int OFF_ML = OFF_BAR + 256;           // warpgroup 1's (max, sum) per row
+constexpr int OFF_PREFIX = OFF_KV + STG * KV_STAGE;
+constexpr int OFF_BAR = OFF_PREFIX + (MAX_B + 4) * 4;
+constexpr int OFF_ML = OFF_BAR + 512;           // warpgroup 1's (max, sum) per row; merge scales
 constexpr int SMEM_BYTES = OFF_ML + 1024 + 1024;
 constexpr int THREADS = 384;                   // 2 softmax warpgroups, 2 producers, 2 MMA
 constexpr int PRODUCER_WARP = 8, MMA_WARP = 9, MMA_WARP1 = 10, PRODUCER_WARP1 = 11;
@@ -80,6 +85,11 @@ constexpr float RESCALE_LOG2 = 8.f;            // tolerate p <= 2^8 before resca
 // P_w (64 bf16 per row) overwrites the first 32 columns of S_w once S_w is read.
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t O_COL = 128, QHI_COL = 384, QLO_COL = 448;
+// named barriers (id 0 is __syncthreads): the epilogue and the segment start,
+// both over the softmax warps of the two warpgroups
+constexpr int BAR_EPI = 1, BAR_SEG = 2;
+
+static_assert(OFF_BAR % 16 == 0 && SMEM_BYTES <= 227 * 1024, "shared memory layout");
 
 // byte offset of 16-byte chunk c16 (0..15, 8 dims each) of token row `row`
 // (0..63) in a K or V tile
@@ -93,36 +103,109 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
     return *reinterpret_cast<uint32_t *>(&v);
 }
 
+__device__ __forceinline__ void named_sync(int id, int n) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
 struct Bars {
     uint64_t kv_full[STG], kv_empty[STG], s_full[2], p_full[2], pv_done[2], fin, q_full;  // fin: 2 arrivals
     uint32_t tmem;
     int abort;
-    int last;  // this CTA merges its (sequence, kv head)
+    int n_pend;                // partial segments written (counted at the end), <= 2
+    int p_b[2], p_j0[2], p_j1[2];
+    int n_merge;               // pairs this CTA completes (merged at the end), <= 2
+    int m_b[2], m_j0[2], m_j1[2];
+    int wsum[THREADS / 32];    // tile-prefix scan
 };
+static_assert(sizeof(Bars) <= 512, "barrier block");
+
+// A CTA's piece of one sequence: tiles [t_a, t_a + n) of sequence b, which
+// starts at tile xp of the list and has nt tiles.
+struct Seg {
+    int b, t_a, n, nt, xp;
+};
+
+// Segment holding tile x (x < x_end <= T), clipped at x_end.  prefix[b] is the
+// first tile of sequence b; it grows strictly (every sequence has a tile for
+// its new keys).
+__device__ __forceinline__ Seg seg_at(const int *prefix, int B, int x, int x_end) {
+    int lo = 0, hi = B - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (prefix[mid] <= x) lo = mid;
+        else hi = mid - 1;
+    }
+    Seg s;
+    s.b = lo;
+    s.xp = prefix[lo];
+    s.nt = prefix[lo + 1] - s.xp;
+    s.t_a = x - s.xp;
+    s.n = min(s.nt - s.t_a, x_end - x);
+    return s;
+}
+
+// Group whose share [j T / n, (j+1) T / n) holds tile x: the largest j with
+// floor(j T / n) <= x, i.e. ceil((x + 1) n / T) - 1.
+__device__ __forceinline__ int group_of(long long x, int n, long long T) {
+    return (int)(((x + 1) * n + T - 1) / T) - 1;
+}
 
 __global__ void __launch_bounds__(THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap map_k,
-                   const __grid_constant__ CUtensorMap map_v,
-                   const __grid_constant__ CUtensorMap map_q, AttnArgs a) {
+                   const __grid_constant__ CUtensorMap map_v, AttnArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     Bars *bars = (Bars *)(smem + OFF_BAR);
+    int *prefix = (int *)(smem + OFF_PREFIX);
     volatile int *abort = &bars->abort;
-    const int s_idx = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int R = a.R, k = a.k;
+    const int R = a.R, k = a.k, B = a.B, Hkv = a.Hkv;
+    const bool paged = a.kv.layout == SP_KV_PAGED;
+    const int act_warps = (R + 31) / 32;  // softmax warps that own real query rows
     pdl_trigger();
 
-    const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs,
-                                  a.max_seq_len,
-                                  (threadIdx.x == 0 && s_idx == 0 && g == 0) ? a.status : nullptr);
-    const int L = sq.len;
-    const int total = L + k;
-    const int t_begin = s_idx * a.split_tokens;
-    if (t_begin >= total) return;  // uniform over the CTA; the merge never reads this unit
-    const int t_end = min(total, t_begin + a.split_tokens);
-    const int n_tiles = (t_end - t_begin + TT - 1) / TT;
-    const int act_warps = (R + 31) / 32;  // softmax warps that own real query rows
+    // ---- the tile list: prefix[b] = sum_{b' < b} ceil((L_b' + k) / TT).
+    // Lengths and ids come from the caller, not from the previous kernel, so
+    // this runs before pdl_wait.
+    {
+        const int per = (B + THREADS - 1) / THREADS;
+        const int b0 = min(B, (int)threadIdx.x * per), b1 = min(B, b0 + per);
+        int sum = 0;
+        for (int bb = b0; bb < b1; ++bb) {
+            const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, bb, a.kv.n_seqs,
+                                          a.max_seq_len, blockIdx.x == 0 ? a.status : nullptr);
+            const int v = ceil_div(sq.len + k, TT);
+            prefix[bb] = v;
+            sum += v;
+        }
+        int incl = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        if (lane == 31) bars->wsum[warp] = incl;
+        __syncthreads();
+        int run = incl - sum;
+        for (int w = 0; w < warp; ++w) run += bars->wsum[w];
+        for (int bb = b0; bb < b1; ++bb) {
+            const int v = prefix[bb];
+            prefix[bb] = run;
+            run += v;
+        }
+        if (threadIdx.x == 0) {
+            int tot = 0;
+            for (int w = 0; w < THREADS / 32; ++w) tot += bars->wsum[w];
+            prefix[B] = tot;
+        }
+    }
+    __syncthreads();
+    const int T = prefix[B];
+    const int n_grp = min((int)gridDim.x / Hkv, ceil_div(T, max(1, a.tc_min_tiles)));
+    const int grp = blockIdx.x / Hkv, g = blockIdx.x - grp * Hkv;
+    if (grp >= n_grp) return;  // uniform over the CTA: no tile for this one
+    const int x0 = (int)((long long)grp * T / n_grp), x1 = (int)((long long)(grp + 1) * T / n_grp);
+
     // producers: warps 8 and 11, plus the softmax warps that own no rows (they
     // help with the cp.async and plain-load tiles; warps 8 and 11 issue TMA)
     const int n_prod = 2 + 2 * (4 - act_warps);
@@ -131,7 +214,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int pidx = warp == PRODUCER_WARP    ? 0
                      : warp == PRODUCER_WARP1 ? 1
                                               : 2 + (warp >> 2) * (4 - act_warps) + ((warp & 3) - act_warps);
-    const bool paged = a.kv.layout == SP_KV_PAGED;
+    const int n_cons = 64 * act_warps;  // softmax threads of both warpgroups
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STG; ++i) {
@@ -146,8 +229,9 @@ __global__ void __launch_bounds__(THREADS, 1)
         mbar_init(&bars->fin, 2);
         mbar_init(&bars->q_full, 1);
         bars->abort = 0;
+        bars->n_merge = 0;
+        bars->n_pend = 0;
         fence_mbar_init();
-        prefetch_tmap(&map_q);
         if (paged) {
             prefetch_tmap(&map_k);
             prefetch_tmap(&map_v);
@@ -157,210 +241,197 @@ __global__ void __launch_bounds__(THREADS, 1)
         tmem_alloc(&bars->tmem, TMEM_COLS);
         tmem_relinquish();
     }
-    // the producer stages this split's page ids while warpgroup 0 writes Q
-    const int P = a.kv.page_size;
-    const int *ptab = paged ? a.kv.page_table + (size_t)max(sq.sid, 0) * a.kv.max_pages : nullptr;
-    int *spages = (int *)(smem + OFF_PAGES);
-    const int lp0 = paged ? t_begin / P : 0;
-    const int n_lp = paged ? min(MAX_SPLIT_PAGES, max(0, ceil_div(min(t_end, L) - t_begin, P))) : 0;
-    pdl_wait();  // the rotated queries and new keys come from the previous kernel
+    // No griddepcontrol.wait here: the cache, page table and lengths belong to the
+    // caller, so the producers start streaming cache tiles while the previous
+    // kernel (which writes the rotated queries and new keys) drains.  Every
+    // thread that reads its output, or writes memory an earlier kernel may still
+    // read, calls pdl_wait() first: producers before a tile with new keys, the
+    // softmax warps before the first queries they load.
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = bars->tmem;
-    // one TMA brings this group's queries [k][G][128] fp32 into the first ring
-    // stages (free until the pipeline starts)
-    float *qs = (float *)(smem + OFF_KV);
-    if (warp == PRODUCER_WARP) {
-        if (lane == 0) {
-            mbar_arrive_expect_tx(&bars->q_full, (uint32_t)(R * DH * 4));
-            tma_load_3d(qs, &map_q, &bars->q_full, 0, g * a.G, b * k);
-        }
-        for (int j = lane; j < n_lp; j += 32)
-            spages[j] = (lp0 + j < a.kv.max_pages) ? ptab[lp0 + j] : -1;
-    }
-    // Q -> bf16 hi/lo in TMEM (row rr = hl*k + r on lane rr; zero past R),
-    // scaled to log2 units: 64 columns of packed pairs for hi, 64 for lo
-    if (warp < 4) {
-        const int row = threadIdx.x;
-        const uint32_t lane_base = tmem + ((uint32_t)(warp * 32) << 16);
-        const bool have_q = mbar_wait_drain(&bars->q_full, 0);
-        const float4 *src = nullptr;
-        if (row < R && have_q) {
-            const int hl = row / k, r = row - hl * k;
-            src = (const float4 *)(qs + (r * a.G + hl) * DH);
-        }
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            uint32_t hi[32], lo[32];
-#pragma unroll
-            for (int c4 = 0; c4 < 16; ++c4) {
-                const float4 x = src ? src[half * 16 + c4] : make_float4(0.f, 0.f, 0.f, 0.f);
-                const float v[4] = {x.x * a.scale_log2, x.y * a.scale_log2, x.z * a.scale_log2,
-                                    x.w * a.scale_log2};
-                float h[4], l4[4];
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    h[e] = __bfloat162float(__float2bfloat16_rn(v[e]));
-                    l4[e] = v[e] - h[e];
-                }
-                hi[2 * c4] = pack_bf16(h[0], h[1]);
-                hi[2 * c4 + 1] = pack_bf16(h[2], h[3]);
-                lo[2 * c4] = pack_bf16(l4[0], l4[1]);
-                lo[2 * c4 + 1] = pack_bf16(l4[2], l4[3]);
-            }
-            tmem_st32u(lane_base + QHI_COL + half * 32, hi);
-            tmem_st32u(lane_base + QLO_COL + half * 32, lo);
-        }
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
+    const int P = a.kv.page_size;
 
     if (is_producer) {
         // ------------------------------------------------------------ producers
         const int ptid = pidx * 32 + lane, pstride = 32 * n_prod;
-        const bool tma_warp = pidx < 2;  // warps 8 and 11 issue TMA for even and odd tiles
-        int issued = 0;
-        bool deferred[STG] = {false, false, false};  // contiguous tiles awaiting cp.async
+        const int npg = paged ? TT / P : 0;  // pages per tile
+        int ci = 0;                          // CTA-local tile counter (ring position)
         int bad = 0;
-        for (int i = 0; i < n_tiles; ++i) {
-            const int st = i % STG;
-            if (!mbar_wait(&bars->kv_empty[st], ((i / STG) & 1) ^ 1, abort)) break;
-            const int t0 = t_begin + i * TT;
-            uint8_t *K = smem + OFF_KV + st * KV_STAGE;
-            uint8_t *V = K + KV_TILE;
-            const bool lead = pidx == (i & 1);
-            bool pure = (t0 + TT <= L);
-            if (pure && paged) {
-                const int npg = TT / P;
-                bool ok = true;
-                const int jl = (t0 - t_begin) / P;  // index into spages
-                if (lane < npg) {
-                    const int lp = t0 / P + lane;
-                    const int page = jl + lane < n_lp ? spages[jl + lane]
-                                                      : (lp < a.kv.max_pages ? ptab[lp] : -1);
-                    ok = page >= 0 && page < a.kv.n_pages;
-                    if (ok && a.gathered) a.gathered[(size_t)b * a.kv.max_pages + lp] = page;
+        bool stop = false, waited = false;
+        for (int x = x0; x < x1 && !stop;) {
+            const Seg sg = seg_at(prefix, B, x, x1);
+            x += sg.n;
+            const int b = sg.b;
+            const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs,
+                                          a.max_seq_len, nullptr);
+            const int L = sq.len, total = L + k;
+            const int *ptab = paged ? a.kv.page_table + (size_t)max(sq.sid, 0) * a.kv.max_pages : nullptr;
+            for (int i = 0; i < sg.n; ++i, ++ci) {
+                const int st = ci % STG;
+                const int t0 = (sg.t_a + i) * TT;
+                const bool lead = pidx == (ci & 1);
+                const bool pure = t0 + TT <= L;  // cache tokens only (TMA when paged)
+                // this tile's page ids, requested before the ring wait hides their latency
+                int page = -1;
+                const int lp = t0 / max(P, 1) + lane;
+                if (pure && paged && lead && lane < npg) page = lp < a.kv.max_pages ? ptab[lp] : -1;
+                // warp-uniform verdict: the lead warp's collectives below need every lane
+                if (!__all_sync(0xffffffffu, mbar_wait(&bars->kv_empty[st], ((ci / STG) & 1) ^ 1, abort))) {
+                    stop = true;
+                    break;
                 }
-                pure = __all_sync(0xffffffffu, ok);  // every producer warp reaches the same verdict
-                if (pure && !lead) {
-                    mbar_arrive(&bars->kv_full[st]);
-                } else if (pure) {
-                    // one TMA box per lane: lane = 2 * page + (K, V), each the
-                    // (page, head) block of P tokens; lane 0 registers the
-                    // stage's bytes before any box is issued
-                    if (lane == 0) mbar_arrive_expect_tx(&bars->kv_full[st], KV_STAGE);
-                    __syncwarp();
-                    if (lane < 2 * npg) {
-                        const int j = lane >> 1, part = lane & 1;
-                        const int page = jl + j < n_lp ? spages[jl + j] : ptab[t0 / P + j];
-                        const int grp = (page * a.Hkv + g) * (P / 8);
-                        tma_load_4d((part ? V : K) + j * P * 256, part ? &map_v : &map_k,
-                                    &bars->kv_full[st], 0, 0, 0, grp);
+                uint8_t *K = smem + OFF_KV + st * KV_STAGE;
+                uint8_t *V = K + KV_TILE;
+                if (pure && paged) {
+                    if (!lead) {
+                        mbar_arrive(&bars->kv_full[st]);
+                    } else {
+                        // one TMA box per lane: lane = 2 * page + (K, V), each the
+                        // (page, head) block of P tokens; a page outside the pool
+                        // is zero-filled instead.  Lane 0 registers the stage's
+                        // bytes before any box is issued.
+                        const bool ok = lane < npg && page >= 0 && page < a.kv.n_pages;
+                        const unsigned okm = __ballot_sync(0xffffffffu, ok);
+                        if (ok && a.gathered) a.gathered[(size_t)b * a.kv.max_pages + lp] = page;
+                        if (lane == 0)
+                            mbar_arrive_expect_tx(&bars->kv_full[st], (uint32_t)__popc(okm) * 2u * P * DH * 2u);
+                        __syncwarp();
+                        const int j = (lane >> 1) & 3, part = lane & 1;
+                        const int pj = __shfl_sync(0xffffffffu, page, j);
+                        if (lane < 2 * npg && ((okm >> j) & 1)) {
+                            const int grp = (pj * Hkv + g) * (P / 8);
+                            tma_load_4d((part ? V : K) + j * P * 256, part ? &map_v : &map_k,
+                                        &bars->kv_full[st], 0, 0, 0, grp);
+                        }
+                        const unsigned want = (1u << npg) - 1u;
+                        if ((okm & want) != want) {
+                            bad = 1;
+                            for (int jj = 0; jj < npg; ++jj) {
+                                if ((okm >> jj) & 1) continue;
+                                for (int e = lane; e < P * 16; e += 32) {
+                                    st_shared_v4(K + jj * P * 256 + e * 16, 0, 0, 0, 0);
+                                    st_shared_v4(V + jj * P * 256 + e * 16, 0, 0, 0, 0);
+                                }
+                            }
+                            fence_proxy_async();
+                        }
+                        if (lane != 0) mbar_arrive(&bars->kv_full[st]);
                     }
-                    if (lane != 0) mbar_arrive(&bars->kv_full[st]);
-                }
-            } else if (pure) {
-                // contiguous: token-major rows of 256 B, 16-byte cp.async per chunk
-                const bf16 *kb = (const bf16 *)a.kv.k_seq[sq.sid];
-                const bf16 *vb = (const bf16 *)a.kv.v_seq[sq.sid];
-                for (int idx = ptid; idx < TT * 16; idx += pstride) {
-                    const int row = idx >> 4, c16 = idx & 15;
-                    const size_t src = ((size_t)(t0 + row) * a.Hkv + g) * DH + c16 * 8;
-                    const uint32_t dst = kv_off(row, c16);
-                    cp_async16(K + dst, kb + src);
-                    cp_async16(V + dst, vb + src);
-                }
-                deferred[st] = true;
-            }
-            if (!pure) {
-                // the sequence end / new keys / a bad page: plain loads, zero fill
-                for (int idx = ptid; idx < TT * 16; idx += pstride) {
-                    const int row = idx >> 4, c16 = idx & 15;
-                    const int t = t0 + row;
-                    const uint32_t dst = kv_off(row, c16);
-                    uint4 kv4 = make_uint4(0, 0, 0, 0), vv4 = make_uint4(0, 0, 0, 0);
-                    if (t < L) {
-                        const bf16 *ks = nullptr, *vs = nullptr;
-                        if (paged) {
-                            const int lp = t / P;
-                            const int page = lp < a.kv.max_pages ? ptab[lp] : -1;
-                            if (page >= 0 && page < a.kv.n_pages) {
-                                const size_t o = (((size_t)page * a.Hkv + g) * P + t % P) * DH + c16 * 8;
-                                ks = (const bf16 *)a.kv.k_pool + o;
-                                vs = (const bf16 *)a.kv.v_pool + o;
-                                if (c16 == 0 && a.gathered && (t % P == 0 || row == 0))
-                                    a.gathered[(size_t)b * a.kv.max_pages + lp] = page;
+                } else {
+                    // cp.async tiles: cache rows (a contiguous cache, or the sequence-end
+                    // tile of a paged one) copied 16 bytes at a time, the k new keys and
+                    // values converted to bf16 through registers, rows past the end
+                    // zero-filled.  This thread's arrival on kv_full fires when its
+                    // copies have landed; the MMA warps fence the async proxy after
+                    // their wait.
+                    const int n_cache = max(0, min(TT, L - t0));             // rows [0, n_cache)
+                    const int n_new = max(0, min(TT, total - t0)) - n_cache;  // then new keys
+                    if (n_new > 0 && !waited) {
+                        pdl_wait();  // the new keys come from the previous kernel
+                        waited = true;
+                    }
+                    if (n_cache > 0 && paged) {
+                        // this tile's page ids: lane j loads logical page t0 / P + j
+                        int mine = -1;
+                        if (lane < npg) {
+                            const int lpt = t0 / P + lane;
+                            mine = lpt < a.kv.max_pages ? ptab[lpt] : -1;
+                            if (pidx == 0 && a.gathered && lane * P < n_cache && mine >= 0 &&
+                                mine < a.kv.n_pages)
+                                a.gathered[(size_t)b * a.kv.max_pages + lpt] = mine;
+                        }
+                        const int pg0 = __shfl_sync(0xffffffffu, mine, 0);
+                        const int pg1 = __shfl_sync(0xffffffffu, mine, 1);
+                        const int pg2 = __shfl_sync(0xffffffffu, mine, 2);
+                        const int pg3 = __shfl_sync(0xffffffffu, mine, 3);
+                        for (int idx = ptid; idx < n_cache * 16; idx += pstride) {
+                            const int row = idx >> 4, c16 = idx & 15, q = row / P;
+                            const uint32_t dst = kv_off(row, c16);
+                            const int pg = q == 0 ? pg0 : q == 1 ? pg1 : q == 2 ? pg2 : pg3;
+                            if (pg >= 0 && pg < a.kv.n_pages) {
+                                const size_t o = (((size_t)pg * Hkv + g) * P + (t0 + row) % P) * DH + c16 * 8;
+                                cp_async16(K + dst, (const bf16 *)a.kv.k_pool + o);
+                                cp_async16(V + dst, (const bf16 *)a.kv.v_pool + o);
                             } else {
+                                st_shared_v4(K + dst, 0, 0, 0, 0);
+                                st_shared_v4(V + dst, 0, 0, 0, 0);
                                 bad = 1;
                             }
-                        } else {
-                            const size_t o = ((size_t)t * a.Hkv + g) * DH + c16 * 8;
-                            ks = (const bf16 *)a.kv.k_seq[sq.sid] + o;
-                            vs = (const bf16 *)a.kv.v_seq[sq.sid] + o;
                         }
-                        if (ks) {
-                            kv4 = *(const uint4 *)ks;
-                            vv4 = *(const uint4 *)vs;
+                    } else if (n_cache > 0) {
+                        // contiguous: token-major rows of 256 B
+                        const bf16 *kb = (const bf16 *)a.kv.k_seq[sq.sid];
+                        const bf16 *vb = (const bf16 *)a.kv.v_seq[sq.sid];
+                        for (int idx = ptid; idx < n_cache * 16; idx += pstride) {
+                            const int row = idx >> 4, c16 = idx & 15;
+                            const size_t src = ((size_t)(t0 + row) * Hkv + g) * DH + c16 * 8;
+                            const uint32_t dst = kv_off(row, c16);
+                            cp_async16(K + dst, kb + src);
+                            cp_async16(V + dst, vb + src);
                         }
-                    } else if (t < total) {
-                        const size_t o = (((size_t)b * k + (t - L)) * a.Hkv + g) * DH + c16 * 8;
-                        const float4 *kf = (const float4 *)(a.k_new + o);
-                        const float4 *vf = (const float4 *)(a.v_new + o);
-                        const float4 k0 = kf[0], k1 = kf[1], v0 = vf[0], v1 = vf[1];
-                        kv4 = make_uint4(pack_bf16(k0.x, k0.y), pack_bf16(k0.z, k0.w),
-                                         pack_bf16(k1.x, k1.y), pack_bf16(k1.z, k1.w));
-                        vv4 = make_uint4(pack_bf16(v0.x, v0.y), pack_bf16(v0.z, v0.w),
-                                         pack_bf16(v1.x, v1.y), pack_bf16(v1.z, v1.w));
                     }
-                    st_shared_v4(K + dst, kv4.x, kv4.y, kv4.z, kv4.w);
-                    st_shared_v4(V + dst, vv4.x, vv4.y, vv4.z, vv4.w);
+                    // new keys/values [B][k][Hkv][dh] fp32: two chunks per thread in flight
+                    for (int idx = ptid; idx < n_new * 16; idx += 2 * pstride) {
+                        float4 kf[2][2], vf[2][2];
+#pragma unroll
+                        for (int u = 0; u < 2; ++u) {
+                            const int j = idx + u * pstride;
+                            if (j < n_new * 16) {
+                                const int rr = (t0 + n_cache + (j >> 4)) - L, c16 = j & 15;
+                                const size_t o = (((size_t)b * k + rr) * Hkv + g) * DH + c16 * 8;
+                                kf[u][0] = *(const float4 *)(a.k_new + o);
+                                kf[u][1] = *(const float4 *)(a.k_new + o + 4);
+                                vf[u][0] = *(const float4 *)(a.v_new + o);
+                                vf[u][1] = *(const float4 *)(a.v_new + o + 4);
+                            }
+                        }
+#pragma unroll
+                        for (int u = 0; u < 2; ++u) {
+                            const int j = idx + u * pstride;
+                            if (j >= n_new * 16) continue;
+                            const uint32_t dst = kv_off(n_cache + (j >> 4), j & 15);
+                            st_shared_v4(K + dst, pack_bf16(kf[u][0].x, kf[u][0].y), pack_bf16(kf[u][0].z, kf[u][0].w),
+                                         pack_bf16(kf[u][1].x, kf[u][1].y), pack_bf16(kf[u][1].z, kf[u][1].w));
+                            st_shared_v4(V + dst, pack_bf16(vf[u][0].x, vf[u][0].y), pack_bf16(vf[u][0].z, vf[u][0].w),
+                                         pack_bf16(vf[u][1].x, vf[u][1].y), pack_bf16(vf[u][1].z, vf[u][1].w));
+                        }
+                    }
+                    const int n_fill = n_cache + n_new;
+                    for (int idx = ptid; idx < (TT - n_fill) * 16; idx += pstride) {
+                        const uint32_t dst = kv_off(n_fill + (idx >> 4), idx & 15);
+                        st_shared_v4(K + dst, 0, 0, 0, 0);
+                        st_shared_v4(V + dst, 0, 0, 0, 0);
+                    }
+                    fence_proxy_async();  // this thread's shared-memory stores
+                    cp_async_mbar_arrive(&bars->kv_full[st]);
                 }
-                fence_proxy_async();
-                mbar_arrive(&bars->kv_full[st]);
-            }
-            cp_async_commit();  // one (possibly empty) group per tile
-            issued = i + 1;
-            // a contiguous tile is published once its copies have landed, DEFER
-            // tiles later (see DEFER)
-            cp_async_wait<DEFER>();
-            const int j = i - DEFER;
-            if (j >= 0 && deferred[j % STG]) {
-                fence_proxy_async();
-                mbar_arrive(&bars->kv_full[j % STG]);
-                deferred[j % STG] = false;
             }
         }
-        cp_async_wait<0>();
-        for (int j = issued - DEFER; j < issued; ++j) {
-            if (j >= 0 && deferred[j % STG]) {
-                fence_proxy_async();
-                mbar_arrive(&bars->kv_full[j % STG]);
-                deferred[j % STG] = false;
-            }
-        }
-        if (tma_warp && lane == 0) {
+        asm volatile("cp.async.wait_all;" ::: "memory");  // nothing lands after the CTA is gone
+        if (pidx < 2 && lane == 0) {
             // drain TMA writes still in flight (only possible after an abort)
-            for (int j = issued > STG ? issued - STG : 0; j < issued; ++j)
-                if ((j & 1) == pidx) mbar_wait_drain(&bars->kv_full[j % STG], (j / STG) & 1);
+            for (int jd = ci > STG ? ci - STG : 0; jd < ci; ++jd)
+                if ((jd & 1) == pidx) mbar_wait_drain(&bars->kv_full[jd % STG], (jd / STG) & 1);
         }
         bad = __any_sync(0xffffffffu, bad);
         if (bad && lane == 0 && a.status) atomicOr(a.status, SP_DEV_BAD_PAGE);
     } else if (warp == MMA_WARP || warp == MMA_WARP1) {
         // ------------------------------------------------------------ MMA issuers
-        // Pipeline w = warp - MMA_WARP takes tiles i = w, w + 2, ...: S_w, then
-        // per tile i: PV_i (after softmax i) and S_{i+2} (reusing S buffer w).
-        // PV_i does not wait for any later tile's data, so stage i is released
-        // as soon as its softmax is done.
+        // Pipeline w = warp - MMA_WARP takes the tiles i = w, w + 2, ... of each
+        // segment: S_w once the segment's queries are in TMEM, then per tile i:
+        // PV_i (after softmax i) and S_{i+2} (reusing S buffer w).  PV_i does not
+        // wait for any later tile's data, so stage i is released as soon as its
+        // softmax is done.
         const int w = warp - MMA_WARP;
         if (lane == 0) {
             constexpr uint32_t idesc_s = idesc_bf16_f32(128, TT);
             constexpr uint32_t idesc_o = idesc_bf16_f32_bmn(128, DH);
             const uint32_t s_tmem = tmem + (uint32_t)(w * TT);  // S_w; P_w over its first half
             const uint32_t o_tmem = tmem + O_COL + (uint32_t)(w * DH);
-            auto issue_s = [&](int i) {
-                const uint8_t *K = smem + OFF_KV + (i % STG) * KV_STAGE;
+            auto issue_s = [&](int cst) {
+                const uint8_t *K = smem + OFF_KV + cst * KV_STAGE;
 #pragma unroll
                 for (int kk = 0; kk < DH / 16; ++kk) {
                     // 16 dims = 32 B along a 128-byte row of dim half kk / 4
@@ -375,235 +446,382 @@ __global__ void __launch_bounds__(THREADS, 1)
                 mma_commit(&bars->s_full[w]);
             };
             bool ok = true;
-            if (w < n_tiles) {
-                ok = mbar_wait(&bars->kv_full[w % STG], (w / STG) & 1, abort);
-                if (ok) {
-                    tc_fence_after();
-                    issue_s(w);
-                }
-            }
-            for (int i = w; ok && i < n_tiles; i += 2) {
-                if (!mbar_wait(&bars->p_full[w], (i >> 1) & 1, abort)) break;
+            int ci0 = 0, kw = 0, j = 0;
+            for (int x = x0; ok && x < x1; ++j) {
+                const Seg sg = seg_at(prefix, B, x, x1);
+                x += sg.n;
+                if (!mbar_wait(&bars->q_full, (uint32_t)(j & 1), abort)) break;
                 tc_fence_after();
-                const uint8_t *V = smem + OFF_KV + (i % STG) * KV_STAGE + KV_TILE;
-#pragma unroll
-                for (int kk = 0; kk < TT / 16; ++kk) {
-                    // 16 tokens of P = 8 TMEM columns; 16 tokens of V = two 8-token groups
-                    mma_bf16_ts(o_tmem, s_tmem + (uint32_t)(kk * 8),
-                                sw128_mnmajor_desc2(V + kk * 2 * GROUP_STRIDE, HALF_STRIDE, GROUP_STRIDE),
-                                idesc_o, (i >= 2 || kk > 0) ? 1u : 0u);
+                if (w < sg.n) {
+                    const int cw = ci0 + w;
+                    ok = mbar_wait(&bars->kv_full[cw % STG], (cw / STG) & 1, abort);
+                    if (ok) {
+                        tc_fence_after();
+                        fence_proxy_async();  // cp.async data -> tensor-core reads
+                        issue_s(cw % STG);
+                    }
                 }
-                mma_commit(&bars->kv_empty[i % STG]);
-                mma_commit(&bars->pv_done[w]);
-                if (i + 2 < n_tiles) {
-                    // S buffer w is free: softmax i has read it (p_full above)
-                    if (!mbar_wait(&bars->kv_full[(i + 2) % STG], ((i + 2) / STG) & 1, abort)) break;
+                for (int i = w; ok && i < sg.n; i += 2, ++kw) {
+                    if (!mbar_wait(&bars->p_full[w], (uint32_t)(kw & 1), abort)) {
+                        ok = false;
+                        break;
+                    }
                     tc_fence_after();
-                    issue_s(i + 2);
+                    const int cst = (ci0 + i) % STG;
+                    const uint8_t *V = smem + OFF_KV + cst * KV_STAGE + KV_TILE;
+#pragma unroll
+                    for (int kk = 0; kk < TT / 16; ++kk) {
+                        // 16 tokens of P = 8 TMEM columns; 16 tokens of V = two 8-token groups
+                        mma_bf16_ts(o_tmem, s_tmem + (uint32_t)(kk * 8),
+                                    sw128_mnmajor_desc2(V + kk * 2 * GROUP_STRIDE, HALF_STRIDE, GROUP_STRIDE),
+                                    idesc_o, (i >= 2 || kk > 0) ? 1u : 0u);
+                    }
+                    mma_commit(&bars->kv_empty[cst]);
+                    mma_commit(&bars->pv_done[w]);
+                    if (i + 2 < sg.n) {
+                        // S buffer w is free: softmax i has read it (p_full above)
+                        const int cn = ci0 + i + 2;
+                        if (!mbar_wait(&bars->kv_full[cn % STG], (cn / STG) & 1, abort)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        fence_proxy_async();  // cp.async data -> tensor-core reads
+                        issue_s(cn % STG);
+                    }
                 }
+                ci0 += sg.n;
             }
             mma_commit(&bars->fin);  // completes when every MMA of this issuer is done
         }
         __syncwarp();
     } else if (warp < 8 && (warp & 3) < act_warps) {
-        // ------------------------------------------------------------ softmax
-        const int wg = warp >> 2;       // warpgroup: tiles i with (i & 1) == wg
+        // ------------------------------------------------------------ softmax + epilogue
+        const int wg = warp >> 2;           // warpgroup: tiles i with (i & 1) == wg
         const int row = threadIdx.x & 127;  // == TMEM lane
+        const int ct = wg * 32 * act_warps + (warp & 3) * 32 + lane;  // 0 .. n_cons-1
         const bool active = row < R;
         const int r_soft = row % k;
         const uint32_t lane_base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
         const uint32_t s_col = (uint32_t)(wg * TT), o_col = O_COL + (uint32_t)(wg * DH);
-        float m = -INFINITY, l = 0.f;
+        float *sm_ml = (float *)(smem + OFF_ML);
+        // The queries of sequence b for kv head g -> bf16 hi/lo in TMEM (row rr =
+        // hl*k + r on lane rr; zero past R), scaled to log2 units.  Warpgroup wg
+        // converts dims [64 wg, 64 wg + 64): TMEM columns [32 wg, 32 wg + 32) of
+        // the hi and of the lo block (two bf16 per column).  Both warpgroups'
+        // warps w and w + 4 reach the same TMEM lanes.
+        auto load_q = [&](int b) {
+            const float4 *src = nullptr;
+            if (active) {
+                const int hl = row / k, r = row - hl * k;
+                src = (const float4 *)(a.q + (((size_t)b * k + r) * a.Hq + g * a.G + hl) * DH) + wg * 16;
+            }
+            uint32_t hi[32], lo[32];
+            float4 xs[16];
+#pragma unroll
+            for (int c4 = 0; c4 < 16; ++c4) xs[c4] = src ? src[c4] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int c4 = 0; c4 < 16; ++c4) {
+                const float v[4] = {xs[c4].x * a.scale_log2, xs[c4].y * a.scale_log2,
+                                    xs[c4].z * a.scale_log2, xs[c4].w * a.scale_log2};
+                float h[4], l4[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    h[e] = __bfloat162float(__float2bfloat16_rn(v[e]));
+                    l4[e] = v[e] - h[e];
+                }
+                hi[2 * c4] = pack_bf16(h[0], h[1]);
+                hi[2 * c4 + 1] = pack_bf16(h[2], h[3]);
+                lo[2 * c4] = pack_bf16(l4[0], l4[1]);
+                lo[2 * c4 + 1] = pack_bf16(l4[2], l4[3]);
+            }
+            tmem_st32u(lane_base + QHI_COL + wg * 32, hi);
+            tmem_st32u(lane_base + QLO_COL + wg * 32, lo);
+            tc_fence_before();
+        };
+        pdl_wait();  // the rotated queries come from the previous kernel
+        load_q(seg_at(prefix, B, x0, x1).b);
         bool ok = true;
-        for (int i = wg; i < n_tiles; i += 2) {
-            const uint32_t ph = (i >> 1) & 1;
-            if (!mbar_wait(&bars->s_full[wg], ph, abort)) {
-                ok = false;
-                break;
-            }
-            tc_fence_after();
-            float sv[TT];
+        int k0 = 0, k1 = 0;  // tiles done so far by pipeline 0 / 1 (barrier phases)
+        for (int x = x0; x < x1;) {
+            const int xs = x;  // segment start (its other fields are recomputed after the tiles)
+            int n_tiles, lim_rel;
             {
-                float t32[32];
-                tmem_ld32(lane_base + s_col, t32);
-#pragma unroll
-                for (int j = 0; j < 32; ++j) sv[j] = t32[j];
-                tmem_ld32(lane_base + s_col + 32, t32);
-#pragma unroll
-                for (int j = 0; j < 32; ++j) sv[32 + j] = t32[j];
+                const Seg sg = seg_at(prefix, B, x, x1);
+                n_tiles = sg.n;
+                const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, sg.b, a.kv.n_seqs,
+                                              a.max_seq_len, nullptr);
+                // this row sees tokens t < min(L + k, L + r + 1); relative to the segment start:
+                lim_rel = min(sq.len + k, sq.len + r_soft + 1) - sg.t_a * TT;
             }
-            const int t0 = t_begin + i * TT;
-            if (t0 + TT > L) {
-                const int lim = min(total, L + r_soft + 1);  // visible: t < lim
-#pragma unroll
-                for (int j = 0; j < TT; ++j)
-                    if (t0 + j >= lim) sv[j] = -INFINITY;
-            }
-            // tile max as an 8-way tree
-            float mx[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) mx[e] = fmaxf(sv[e], sv[e + 8]);
-#pragma unroll
-            for (int j = 16; j < TT; j += 8)
-#pragma unroll
-                for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], sv[j + e]);
-            const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                                   fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
-            const bool grow = active && (mt > m + RESCALE_LOG2 || (m == -INFINITY && mt != -INFINITY));
-            const float m_new = grow ? mt : m;
-            const float alpha = grow ? (m == -INFINITY ? 0.f : fast_exp2(m - m_new)) : 1.f;
-            // O_wg and P_wg were last used by PV_{i-2}
-            if (i >= 2) {
-                if (!mbar_wait(&bars->pv_done[wg], ((i - 2) >> 1) & 1, abort)) {
+            x += n_tiles;
+            // this segment's queries are written, and the previous epilogue is complete
+            named_sync(BAR_SEG, n_cons);
+            if (ct == 0) mbar_arrive(&bars->q_full);
+
+            float m = -INFINITY, l = 0.f;
+            int kw = wg ? k1 : k0;
+            for (int i = wg; ok && i < n_tiles; i += 2, ++kw) {
+                // warp-uniform verdicts: the TMEM loads and stores are warp-collective
+                if (!__all_sync(0xffffffffu, mbar_wait(&bars->s_full[wg], (uint32_t)(kw & 1), abort))) {
                     ok = false;
                     break;
                 }
-                if (__any_sync(0xffffffffu, grow)) {
-                    tc_fence_after();
-#pragma unroll 1
-                    for (int c0 = 0; c0 < DH; c0 += 32) {
-                        float o32[32];
-                        tmem_ld32(lane_base + o_col + c0, o32);
+                tc_fence_after();
+                float sv[TT];
+                {
+                    float t32[32];
+                    tmem_ld32(lane_base + s_col, t32);
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) o32[j] *= alpha;
-                        tmem_st32(lane_base + o_col + c0, o32);
+                    for (int jj = 0; jj < 32; ++jj) sv[jj] = t32[jj];
+                    tmem_ld32(lane_base + s_col + 32, t32);
+#pragma unroll
+                    for (int jj = 0; jj < 32; ++jj) sv[32 + jj] = t32[jj];
+                }
+                const int t0 = i * TT;  // relative to the segment start
+                if (t0 + TT > lim_rel) {
+#pragma unroll
+                    for (int jj = 0; jj < TT; ++jj)
+                        if (t0 + jj >= lim_rel) sv[jj] = -INFINITY;
+                }
+                // tile max as an 8-way tree
+                float mx[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) mx[e] = fmaxf(sv[e], sv[e + 8]);
+#pragma unroll
+                for (int jj = 16; jj < TT; jj += 8)
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) mx[e] = fmaxf(mx[e], sv[jj + e]);
+                const float mt = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                                       fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
+                const bool grow = active && (mt > m + RESCALE_LOG2 || (m == -INFINITY && mt != -INFINITY));
+                const float m_new = grow ? mt : m;
+                const float alpha = grow ? (m == -INFINITY ? 0.f : fast_exp2(m - m_new)) : 1.f;
+                // O_wg and P_wg were last used by PV of this pipeline's previous tile
+                if (i >= 2) {
+                    if (!__all_sync(0xffffffffu, mbar_wait(&bars->pv_done[wg], (uint32_t)((kw - 1) & 1), abort))) {
+                        ok = false;
+                        break;
+                    }
+                    if (__any_sync(0xffffffffu, grow)) {
+                        tc_fence_after();
+#pragma unroll 1
+                        for (int c0 = 0; c0 < DH; c0 += 32) {
+                            float o32[32];
+                            tmem_ld32(lane_base + o_col + c0, o32);
+#pragma unroll
+                            for (int jj = 0; jj < 32; ++jj) o32[jj] *= alpha;
+                            tmem_st32(lane_base + o_col + c0, o32);
+                        }
                     }
                 }
-            }
-            l *= alpha;
-            m = m_new;
-            const float mu = (m == -INFINITY) ? 0.f : m;  // a fully masked row gives p = 0
-            float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-            uint32_t pk[TT / 2];
+                l *= alpha;
+                m = m_new;
+                const float mu = (m == -INFINITY) ? 0.f : m;  // a fully masked row gives p = 0
+                float ps[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                uint32_t pk[TT / 2];
 #pragma unroll
-            for (int j = 0; j < TT; j += 2) {
-                const float p0 = fast_exp2(sv[j] - mu);
-                const float p1 = fast_exp2(sv[j + 1] - mu);
-                ps[(j >> 1) & 7] += p0 + p1;
-                pk[j >> 1] = pack_bf16(p0, p1);
+                for (int jj = 0; jj < TT; jj += 2) {
+                    const float p0 = fast_exp2(sv[jj] - mu);
+                    const float p1 = fast_exp2(sv[jj + 1] - mu);
+                    ps[(jj >> 1) & 7] += p0 + p1;
+                    pk[jj >> 1] = pack_bf16(p0, p1);
+                }
+                l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+                tmem_st32u(lane_base + s_col, pk);  // P_i over the first half of S_i
+                tc_fence_before();
+                mbar_arrive(&bars->p_full[wg]);
             }
-            l += ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
-            tmem_st32u(lane_base + s_col, pk);  // P_i over the first half of S_i
-            tc_fence_before();
-            mbar_arrive(&bars->p_full[wg]);
-        }
-        // epilogue: warpgroup 1 hands its (max, sum) to warpgroup 0 through shared
-        // memory; warpgroup 0 combines (max, sum, O) of both and writes the unit's
-        // unnormalised partial
-        float *sm_ml = (float *)(smem + OFF_ML);
-        const int last0 = n_tiles >= 1 ? n_tiles - 1 - ((n_tiles - 1) & 1) : -1;  // WG0's last tile
-        const int last1 = n_tiles >= 2 ? n_tiles - 1 - (n_tiles & 1) : -1;        // WG1's last tile
-        if (wg == 1) {
-            sm_ml[row] = last1 >= 0 ? m : -INFINITY;
-            sm_ml[128 + row] = last1 >= 0 ? l : 0.f;
-        }
-        asm volatile("bar.sync 1, %0;" ::"r"(64 * act_warps) : "memory");
-        if (wg == 0) {
-            const size_t unit = ((size_t)b * a.Hkv + g) * a.n_splits + s_idx;
-            float *po = a.part_o + (unit * R + row) * DH;
+            const int n0 = (n_tiles + 1) >> 1, n1 = n_tiles >> 1;  // tiles of pipeline 0 / 1
+            k0 += n0;
+            k1 += n1;
+
+            // ---- epilogue: warpgroup 1 hands its (max, sum) to warpgroup 0 through
+            // shared memory and loads half of the next segment's queries; warpgroup 0
+            // combines (max, sum, O) of both, writes the pair's output (whole pair in
+            // this CTA's share) or this segment's partial, and loads the other half
+            const Seg sg = seg_at(prefix, B, xs, x1);
+            const int b = sg.b;
+            const int j_first = group_of(sg.xp, n_grp, T);
+            const int j_last = group_of((long long)sg.xp + sg.nt - 1, n_grp, T);
+            const bool whole = j_first == j_last;
+            if (wg == 1) {
+                sm_ml[row] = n1 > 0 ? m : -INFINITY;
+                sm_ml[128 + row] = n1 > 0 ? l : 0.f;
+            }
+            // both warpgroups are past their last S of the segment: Q may be rewritten
+            named_sync(BAR_EPI, n_cons);
+            if (wg == 1) {
+                if (x < x1) load_q(seg_at(prefix, B, x, x1).b);
+                continue;
+            }
             const float m1 = sm_ml[row], l1 = sm_ml[128 + row];
             const float mc = fmaxf(m, m1);
             const float a0 = (m == -INFINITY) ? 0.f : fast_exp2(m - mc);
             const float a1 = (m1 == -INFINITY) ? 0.f : fast_exp2(m1 - mc);
-            bool have = ok && last0 >= 0 && mbar_wait(&bars->pv_done[0], (last0 >> 1) & 1, abort);
-            if (have && last1 >= 0) have = mbar_wait(&bars->pv_done[1], (last1 >> 1) & 1, abort);
+            const float lsum = a0 * l + a1 * l1;
+            bool have = ok && mbar_wait(&bars->pv_done[0], (uint32_t)((k0 - 1) & 1), abort);
+            if (have && n1 > 0) have = mbar_wait(&bars->pv_done[1], (uint32_t)((k1 - 1) & 1), abort);
             have = __all_sync(0xffffffffu, have);  // the TMEM loads below are warp-collective
+            if (!have) ok = false;
+            const size_t slot = ((size_t)grp + b) * Hkv + g;
+            float *po = a.part_o + (slot * R + row) * DH;
+            const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+            const int hl = row / k, r = row - hl * k;
+            const size_t out0 = (((size_t)b * k + r) * a.Hq + g * a.G + hl) * DH;
             if (have) {
                 tc_fence_after();
 #pragma unroll 1
                 for (int c0 = 0; c0 < DH; c0 += 32) {
                     float o0[32], o1[32];
                     tmem_ld32(lane_base + O_COL + c0, o0);
-                    if (last1 >= 0) {
+                    if (n1 > 0) {
                         tmem_ld32(lane_base + O_COL + DH + c0, o1);
                     } else {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) o1[j] = 0.f;
+                        for (int jj = 0; jj < 32; ++jj) o1[jj] = 0.f;
                     }
-                    if (active) {
+                    if (active && whole) {
 #pragma unroll
-                        for (int j = 0; j < 32; j += 4)
-                            *(float4 *)(po + c0 + j) =
-                                make_float4(a0 * o0[j] + a1 * o1[j], a0 * o0[j + 1] + a1 * o1[j + 1],
-                                            a0 * o0[j + 2] + a1 * o1[j + 2], a0 * o0[j + 3] + a1 * o1[j + 3]);
+                        for (int jj = 0; jj < 32; jj += 4)
+                            act_store4(a.out, out0 + c0 + jj,
+                                       make_float4((a0 * o0[jj] + a1 * o1[jj]) * inv,
+                                                   (a0 * o0[jj + 1] + a1 * o1[jj + 1]) * inv,
+                                                   (a0 * o0[jj + 2] + a1 * o1[jj + 2]) * inv,
+                                                   (a0 * o0[jj + 3] + a1 * o1[jj + 3]) * inv));
+                    } else if (active) {
+#pragma unroll
+                        for (int jj = 0; jj < 32; jj += 4)
+                            *(float4 *)(po + c0 + jj) =
+                                make_float4(a0 * o0[jj] + a1 * o1[jj], a0 * o0[jj + 1] + a1 * o1[jj + 1],
+                                            a0 * o0[jj + 2] + a1 * o1[jj + 2],
+                                            a0 * o0[jj + 3] + a1 * o1[jj + 3]);
                     }
                 }
-                if (active) {
-                    a.part_ml[(unit * R + row) * 2] = mc;
-                    a.part_ml[(unit * R + row) * 2 + 1] = a0 * l + a1 * l1;
+                if (active && !whole) {
+                    a.part_ml[(slot * R + row) * 2] = mc;
+                    a.part_ml[(slot * R + row) * 2 + 1] = lsum;
                 }
             }
-            __threadfence();  // the partial is visible device-wide before this unit is counted
+            if (!whole && ct == 0 && bars->n_pend < 2) {
+                // counted at the end of the kernel (only a share's first and last
+                // segments can be partial)
+                const int t = bars->n_pend++;
+                bars->p_b[t] = b;
+                bars->p_j0[t] = j_first;
+                bars->p_j1[t] = j_last;
+            }
+            if (x < x1) load_q(seg_at(prefix, B, x, x1).b);
         }
     }
     // every MMA must be finished before TMEM and shared memory go away
     mbar_wait_drain(&bars->fin, 0);
+    if (warp < 4) __threadfence();  // the partials are visible device-wide before they are counted
     tc_fence_before();
     __syncthreads();
-    if (threadIdx.x == 0 && *abort && a.status) atomicOr(a.status, SP_DEV_TIMEOUT);
-    if (warp == MMA_WARP) tmem_dealloc(tmem, TMEM_COLS);
-
-    // ---------------------------------------------------------------- merge
-    if (!a.counters) return;  // merged by a separate kernel
-    const int n_units = min(a.n_splits, ceil_div(total, a.split_tokens));
-    int *counter = a.counters + (size_t)b * a.Hkv + g;
     if (threadIdx.x == 0) {
-        bars->last = atomicAdd(counter, 1) == n_units - 1;
-        __threadfence();
-    }
-    __syncthreads();
-    if (!bars->last) return;
-    // every unit of the pair has written its partial: combine them.  Pass 1: per
-    // row, the normalised weight of each partial (shared memory, over the
-    // free K/V ring); pass 2: per (row, 4 columns), the weighted sum.
-    const size_t p0 = ((size_t)b * a.Hkv + g) * a.n_splits;
-    float *wn = (float *)(smem + OFF_KV);  // [R][n_units]
-    for (int rr = threadIdx.x; rr < R; rr += THREADS) {
-        float mmax = -INFINITY;
-#pragma unroll 8
-        for (int p = 0; p < n_units; ++p) mmax = fmaxf(mmax, __ldcg(a.part_ml + ((p0 + p) * R + rr) * 2));
-        float l = 0.f;
-#pragma unroll 8
-        for (int p = 0; p < n_units; ++p) {
-            const float2 ml = __ldcg((const float2 *)(a.part_ml + ((p0 + p) * R + rr) * 2));
-            const float w = (ml.x == -INFINITY) ? 0.f : exp2f(ml.x - mmax);
-            wn[rr * n_units + p] = w;
-            l += w * ml.y;
+        if (*abort && a.status) atomicOr(a.status, SP_DEV_TIMEOUT);
+        // count this CTA's partial segments; the CTA completing a pair merges it
+        for (int t = 0; t < bars->n_pend; ++t) {
+            const int b = bars->p_b[t], n_seg = bars->p_j1[t] - bars->p_j0[t] + 1;
+            if (atomicAdd(a.counters + b * Hkv + g, 1) == n_seg - 1) {
+                const int u = bars->n_merge++;
+                bars->m_b[u] = b;
+                bars->m_j0[u] = bars->p_j0[t];
+                bars->m_j1[u] = bars->p_j1[t];
+            }
         }
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        for (int p = 0; p < n_units; ++p) wn[rr * n_units + p] *= inv;
+        __threadfence();  // the other segments' partials are read after their count
     }
+    if (warp == MMA_WARP) tmem_dealloc(tmem, TMEM_COLS);
     __syncthreads();
-    for (int idx = threadIdx.x; idx < R * (DH / 4); idx += THREADS) {
-        const int rr = idx / (DH / 4), c = (idx % (DH / 4)) * 4;
-        float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-        for (int p = 0; p < n_units; ++p) {
-            const float w = wn[rr * n_units + p];
-            const float4 op = __ldcg((const float4 *)(a.part_o + ((p0 + p) * R + rr) * DH + c));
-            o.x += w * op.x;
-            o.y += w * op.y;
-            o.z += w * op.z;
-            o.w += w * op.w;
+
+    // ---- merges, by the whole CTA: every segment of pair (b, g) has written its
+    // partial (slots (j + b) Hkv + g, j = j0 .. j1).  One pass per (row, 4
+    // columns), the partials' loads issued together in chunks of MCH with an
+    // online rescale between chunks, and MIT items in flight per thread.
+    constexpr int MCH = 4, MIT = 2;
+    for (int t = 0; t < bars->n_merge; ++t) {
+        const int b = bars->m_b[t], j0 = bars->m_j0[t], ns = bars->m_j1[t] - j0 + 1;
+        const size_t slot0 = ((size_t)j0 + b) * Hkv + g;  // slot of segment j0 + e: slot0 + e Hkv
+        const int items = R * (DH / 4);
+        for (int i0 = threadIdx.x; i0 < items; i0 += THREADS * MIT) {
+            float mm[MIT], ls[MIT];
+            float4 o[MIT];
+#pragma unroll
+            for (int u = 0; u < MIT; ++u) {
+                mm[u] = -INFINITY;
+                ls[u] = 0.f;
+                o[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            for (int e0 = 0; e0 < ns; e0 += MCH) {
+                float mv[MIT][MCH], lv[MIT][MCH];
+                float4 ov[MIT][MCH];
+#pragma unroll
+                for (int u = 0; u < MIT; ++u) {
+                    const int idx = i0 + u * THREADS;
+                    const int rr = idx / (DH / 4), cq = (idx % (DH / 4)) * 4;
+#pragma unroll
+                    for (int e = 0; e < MCH; ++e) {
+                        const bool in = idx < items && e0 + e < ns;
+                        const size_t sl = slot0 + (size_t)(e0 + e) * Hkv;
+                        const float2 ml = in ? __ldcg((const float2 *)(a.part_ml + (sl * R + rr) * 2))
+                                             : make_float2(-INFINITY, 0.f);
+                        mv[u][e] = ml.x;
+                        lv[u][e] = ml.y;
+                        ov[u][e] = in ? __ldcg((const float4 *)(a.part_o + (sl * R + rr) * DH + cq))
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < MIT; ++u) {
+                    float mn = mm[u];
+#pragma unroll
+                    for (int e = 0; e < MCH; ++e) mn = fmaxf(mn, mv[u][e]);
+                    if (mn == -INFINITY) continue;
+                    const float al = mm[u] == -INFINITY ? 0.f : exp2f(mm[u] - mn);
+                    ls[u] *= al;
+                    o[u].x *= al;
+                    o[u].y *= al;
+                    o[u].z *= al;
+                    o[u].w *= al;
+#pragma unroll
+                    for (int e = 0; e < MCH; ++e) {
+                        const float wgt = mv[u][e] == -INFINITY ? 0.f : exp2f(mv[u][e] - mn);
+                        ls[u] += wgt * lv[u][e];
+                        o[u].x += wgt * ov[u][e].x;
+                        o[u].y += wgt * ov[u][e].y;
+                        o[u].z += wgt * ov[u][e].z;
+                        o[u].w += wgt * ov[u][e].w;
+                    }
+                    mm[u] = mn;
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < MIT; ++u) {
+                const int idx = i0 + u * THREADS;
+                if (idx >= items) continue;
+                const int rr = idx / (DH / 4), cq = (idx % (DH / 4)) * 4;
+                const float inv = ls[u] > 0.f ? 1.f / ls[u] : 0.f;
+                const int hl = rr / k, r = rr - hl * k;
+                act_store4(a.out, (((size_t)b * k + r) * a.Hq + g * a.G + hl) * DH + cq,
+                           make_float4(o[u].x * inv, o[u].y * inv, o[u].z * inv, o[u].w * inv));
+            }
         }
-        const int hl = rr / k, r = rr - hl * k;
-        const int h = g * a.G + hl;
-        act_store4(a.out, (((size_t)b * k + r) * a.Hq + h) * DH + c, o);
+        if (threadIdx.x == 0) a.counters[b * Hkv + g] = 0;  // ready for a launch that does not clear it
     }
-    if (threadIdx.x == 0) *counter = 0;  // ready for a launch that does not clear it
 }
 
 }  // namespace
 
 bool attention_tc_supported(const AttnArgs &a) {
-    return a.dh == DH && a.kv_bf16 && a.R >= 1 && a.R <= 128 && a.split_tokens % TT == 0 &&
+    return a.dh == DH && a.kv_bf16 && a.R >= 1 && a.R <= 128 && a.B >= 1 && a.B <= MAX_B &&
            (a.kv.layout == SP_KV_CONTIGUOUS ||
             (a.kv.page_size == 16 || a.kv.page_size == 32 || a.kv.page_size == 64));
 }
 
 cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
-                                const CUtensorMap *map_v, const CUtensorMap &map_q,
-                                cudaStream_t st) {
+                                const CUtensorMap *map_v, cudaStream_t st) {
     static bool attr = false;
     if (!attr) {
         cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel,
@@ -613,9 +831,8 @@ cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
     }
     CUtensorMap dummy;
     memset(&dummy, 0, sizeof dummy);
-    dim3 grid(a.n_splits, a.Hkv, a.B);
-    return launch_k(attn_tc_kernel, grid, dim3(THREADS), SMEM_BYTES, st, map_k ? *map_k : dummy,
-                    map_v ? *map_v : dummy, map_q, a);
+    return launch_k(attn_tc_kernel, dim3(a.tc_ctas), dim3(THREADS), SMEM_BYTES, st,
+                    map_k ? *map_k : dummy, map_v ? *map_v : dummy, a);
 }
 
 }  // namespace sp

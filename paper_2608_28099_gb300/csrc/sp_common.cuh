@@ -203,11 +203,13 @@ struct AttnArgs {
     const float *k_new;           // [B][k][Hkv][dh], rotated
     const float *v_new;           // [B][k][Hkv][dh]
     int subs;                     // partials per work unit (1)
-    float *part_o;                // [B][Hkv][n_splits][subs][R][dh], unnormalised
-    float *part_ml;               // [B][Hkv][n_splits][subs][R][2] (max in log2 units, sum)
-    int *counters;                // [B][Hkv] finished units, zero before the launch, or NULL:
-                                  // the tensor-core kernel's last unit of a (sequence, kv head)
-                                  // merges; NULL leaves the merge to attn_merge_kernel
+    int tc_ctas;                  // tensor-core kernel: persistent CTAs (one per SM)
+    int tc_min_tiles;             // tensor-core kernel: fewest 64-token tiles per CTA
+    float *part_o;                // CUDA cores: [B][Hkv][n_splits][subs][R][dh]; tensor
+                                  // cores: [tc_ctas + B Hkv][R][dh] (slot c + pair); unnormalised
+    float *part_ml;               // same slots, [R][2] each (max in log2 units, sum)
+    int *counters;                // [B][Hkv] finished segments, zero before the launch (tensor
+                                  // cores: the last segment of a pair merges it)
     int *status;
     int *gathered;                // [B][max_pages] or NULL
     float scale_log2;             // log2(e) / sqrt(dh)
@@ -217,14 +219,22 @@ struct AttnArgs {
 // Plan: tokens per split-KV work unit and number of units per sequence.
 void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, int n_sm,
                     int *split_tokens, int *n_splits);
-size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits);
+// Attention scratch: merge counters [B][Hkv] int, then partials (part_o,
+// part_ml) sized for either kernel: B Hkv n_splits units (CUDA cores) or
+// attn_tc_ctas(n_sm, Hkv) + B Hkv slots (tensor cores).
+size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits, int n_sm);
+// Default fewest tiles per CTA of the tensor-core kernel (64 tokens each).
+constexpr int kAttnMinTiles = 4;
+// Persistent CTAs of the tensor-core kernel: whole groups of Hkv (one CTA per
+// kv head), as many groups as the SMs hold, at least one.
+inline int attn_tc_ctas(int n_sm, int Hkv) { return (n_sm / Hkv > 1 ? n_sm / Hkv : 1) * Hkv; }
 cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st);
-// tcgen05 kernel: head_dim 128, bf16 cache, R <= 128; paged caches need TMA
-// maps of the K and V pools from encode_kv_pages_bf16.
+// tcgen05 kernel: head_dim 128, bf16 cache, R <= 128, B <= 2048; paged caches
+// need TMA maps of the K and V pools from encode_kv_pages_bf16.  The merge
+// runs inside it (counters must be zero at launch).
 bool attention_tc_supported(const AttnArgs &a);
 cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
-                                const CUtensorMap *map_v, const CUtensorMap &map_q,
-                                cudaStream_t st);
+                                const CUtensorMap *map_v, cudaStream_t st);
 cudaError_t launch_attention_merge(const AttnArgs &a, cudaStream_t st);
 
 // ---------------------------------------------------------------------------

@@ -145,8 +145,15 @@ template <int N>
 __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
-// Make this thread's generic-proxy shared-memory writes visible to the async
-// proxy (TMA, tensor cores).
+// Arrive on `bar` once every cp.async this thread has issued so far has landed
+// (the arrival counts toward the barrier's expected count: no increment).
+__device__ __forceinline__ void cp_async_mbar_arrive(uint64_t *bar) {
+    asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+// Make generic-proxy shared-memory writes (this thread's, or those ordered before
+// this point by a barrier wait, e.g. cp.async data) visible to the async proxy
+// (TMA, tensor cores).
 __device__ __forceinline__ void fence_proxy_async() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
