@@ -197,6 +197,9 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
                             cudaEvent_t *ev_attn = nullptr, cudaEvent_t *ev_merge = nullptr) {
     a.tc_ctas = attn_tc_ctas(n_sm, a.Hkv);
     a.tc_min_tiles = forced_split > 0 ? forced_split / 64 : kAttnMinTiles;
+    // few sequences over many groups: each pair has many partials, merged by a
+    // kernel spread over (head, sequence, row) instead of one CTA per pair
+    a.tc_merge_kernel = 4 * a.B < a.tc_ctas / a.Hkv;
     const size_t need = attention_workspace_bytes(a.B, a.Hkv, a.R, a.dh, a.n_splits, n_sm);
     if (ws_bytes < need) return fail(SP_ERR_INVALID_ARG, "attention workspace too small (%zu < %zu)", ws_bytes, need);
     const size_t pairs = (size_t)a.B * a.Hkv;
@@ -229,7 +232,7 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
     if (ev_merge) cudaEventRecordWithFlags(ev_merge[0], st, cudaEventRecordExternal);
     if (!tc) SP_CUDA(launch_attention_merge(a, st));
     if (ev_merge) cudaEventRecordWithFlags(ev_merge[1], st, cudaEventRecordExternal);
-    *launches += tc ? 1 : 2;
+    *launches += tc && !a.tc_merge_kernel ? 1 : 2;
     return SP_OK;
 }
 

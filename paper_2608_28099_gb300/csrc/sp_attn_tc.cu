@@ -75,7 +75,9 @@ constexpr uint32_t HALF_STRIDE = 1024;         // 64-dim halves within a group
 constexpr int MAX_B = 2048;                    // sequences per launch (tile prefix in smem)
 constexpr int OFF_KV = 0;
 constexpr int OFF_PREFIX = OFF_KV + STG * KV_STAGE;
-constexpr int OFF_BAR = OFF_PREFIX + (MAX_B + 4) * 4;
+constexpr int MAX_GRP = 256;                   // groups (cuts table in smem)
+constexpr int OFF_CUTS = OFF_PREFIX + (MAX_B + 4) * 4;
+constexpr int OFF_BAR = OFF_CUTS + (MAX_GRP + 4) * 4;
 constexpr int OFF_ML = OFF_BAR + 512;           // warpgroup 1's (max, sum) per row; merge scales
 constexpr int SMEM_BYTES = OFF_ML + 1024 + 1024;
 constexpr int THREADS = 384;                   // 2 softmax warpgroups, 2 producers, 2 MMA
@@ -144,10 +146,39 @@ __device__ __forceinline__ Seg seg_at(const int *prefix, int B, int x, int x_end
     return s;
 }
 
-// Group whose share [j T / n, (j+1) T / n) holds tile x: the largest j with
-// floor(j T / n) <= x, i.e. ceil((x + 1) n / T) - 1.
-__device__ __forceinline__ int group_of(long long x, int n, long long T) {
-    return (int)(((x + 1) * n + T - 1) / T) - 1;
+// First tile of group j's share.  The even cut j T / n moves to the nearest
+// sequence start when one lies within delta = min(share / 4, SNAP) tiles: a
+// segment boundary costs the consumers a pipeline drain and refill worth a few
+// tiles, so a short sequence is better kept whole than split near its end.
+// Cuts stay strictly increasing (they move by at most a quarter share).
+// Evaluated once per group into a table (cuts[0..n]).
+constexpr int SNAP = 4;
+__device__ __forceinline__ int share_start(const int *prefix, int B, int T, int n, int j) {
+    if (j <= 0) return 0;
+    if (j >= n) return T;
+    const int x = (int)((long long)j * T / n);
+    const int delta = min(T / n / 4, SNAP);
+    if (delta == 0) return x;
+    int lo = 0, hi = B - 1;  // last sequence starting at or before x
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (prefix[mid] <= x) lo = mid;
+        else hi = mid - 1;
+    }
+    const int c0 = prefix[lo], c1 = prefix[lo + 1];
+    const int best = (x - c0 <= c1 - x) ? c0 : c1;
+    return abs(best - x) <= delta ? best : x;
+}
+
+// Group whose share holds tile x (0 <= x < T): the largest j with cuts[j] <= x.
+__device__ __forceinline__ int group_of(const int *cuts, int n, int x) {
+    int lo = 0, hi = n - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (cuts[mid] <= x) lo = mid;
+        else hi = mid - 1;
+    }
+    return lo;
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
@@ -204,7 +235,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int n_grp = min((int)gridDim.x / Hkv, ceil_div(T, max(1, a.tc_min_tiles)));
     const int grp = blockIdx.x / Hkv, g = blockIdx.x - grp * Hkv;
     if (grp >= n_grp) return;  // uniform over the CTA: no tile for this one
-    const int x0 = (int)((long long)grp * T / n_grp), x1 = (int)((long long)(grp + 1) * T / n_grp);
+    int *cuts = (int *)(smem + OFF_CUTS);
+    for (int j = threadIdx.x; j <= n_grp; j += THREADS) cuts[j] = share_start(prefix, B, T, n_grp, j);
+    __syncthreads();
+    const int x0 = cuts[grp], x1 = cuts[grp + 1];
 
     // producers: warps 8 and 11, plus the softmax warps that own no rows (they
     // help with the cp.async and plain-load tiles; warps 8 and 11 issue TMA)
@@ -642,8 +676,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             // this CTA's share) or this segment's partial, and loads the other half
             const Seg sg = seg_at(prefix, B, xs, x1);
             const int b = sg.b;
-            const int j_first = group_of(sg.xp, n_grp, T);
-            const int j_last = group_of((long long)sg.xp + sg.nt - 1, n_grp, T);
+            const int j_first = group_of(cuts, n_grp, sg.xp);
+            const int j_last = group_of(cuts, n_grp, sg.xp + sg.nt - 1);
             const bool whole = j_first == j_last;
             if (wg == 1) {
                 sm_ml[row] = n1 > 0 ? m : -INFINITY;
@@ -703,7 +737,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     a.part_ml[(slot * R + row) * 2 + 1] = lsum;
                 }
             }
-            if (!whole && ct == 0 && bars->n_pend < 2) {
+            if (!whole && ct == 0 && !a.tc_merge_kernel && bars->n_pend < 2) {
                 // counted at the end of the kernel (only a share's first and last
                 // segments can be partial)
                 const int t = bars->n_pend++;
@@ -812,10 +846,72 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
 }
 
+// Merge of the partial segments for small batches (a few long sequences, each
+// spread over many groups): one block per (kv head g, sequence b, query row),
+// one thread per dim, the pair's segments combined in the exp2 domain in
+// chunks of eight with their loads issued together.  Pairs inside one share
+// were finished by the attention kernel.
+__global__ void __launch_bounds__(DH) attn_tc_merge_kernel(AttnArgs a) {
+    pdl_trigger();
+    __shared__ int prefix[MAX_B + 1];
+    __shared__ int cuts[MAX_GRP + 1];
+    const int g = blockIdx.x, b = blockIdx.y, rr = blockIdx.z, c = threadIdx.x;
+    const int B = a.B, Hkv = a.Hkv, R = a.R, k = a.k;
+    if (threadIdx.x == 0) {
+        int run = 0;
+        for (int bb = 0; bb < B; ++bb) {
+            prefix[bb] = run;
+            const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, bb, a.kv.n_seqs,
+                                          a.max_seq_len, nullptr);
+            run += ceil_div(sq.len + k, TT);
+        }
+        prefix[B] = run;
+    }
+    __syncthreads();
+    const int T = prefix[B];
+    const int n_grp = min(a.tc_ctas / Hkv, ceil_div(T, max(1, a.tc_min_tiles)));
+    for (int j = threadIdx.x; j <= n_grp; j += blockDim.x) cuts[j] = share_start(prefix, B, T, n_grp, j);
+    __syncthreads();
+    const int j0 = group_of(cuts, n_grp, prefix[b]);
+    const int j1 = group_of(cuts, n_grp, prefix[b + 1] - 1);
+    if (j0 == j1) return;  // written by the attention kernel
+    pdl_wait();            // the partials come from the attention kernel
+    const int ns = j1 - j0 + 1;
+    float mm = -INFINITY, l = 0.f, o = 0.f;
+    for (int e0 = 0; e0 < ns; e0 += 8) {
+        float mv[8], lv[8], ov[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const bool in = e0 + e < ns;
+            const size_t sl = ((size_t)j0 + e0 + e + b) * Hkv + g;
+            mv[e] = in ? __ldcg(a.part_ml + (sl * R + rr) * 2) : -INFINITY;
+            lv[e] = in ? __ldcg(a.part_ml + (sl * R + rr) * 2 + 1) : 0.f;
+            ov[e] = in ? __ldcg(a.part_o + (sl * R + rr) * DH + c) : 0.f;
+        }
+        float mn = mm;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mn = fmaxf(mn, mv[e]);
+        if (mn == -INFINITY) continue;
+        const float al = mm == -INFINITY ? 0.f : exp2f(mm - mn);
+        l *= al;
+        o *= al;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const float w = mv[e] == -INFINITY ? 0.f : exp2f(mv[e] - mn);
+            l += w * lv[e];
+            o += w * ov[e];
+        }
+        mm = mn;
+    }
+    const int hl = rr / k, r = rr - hl * k;
+    act_store(a.out, (((size_t)b * k + r) * a.Hq + g * a.G + hl) * DH + c, l > 0.f ? o / l : 0.f);
+}
+
 }  // namespace
 
 bool attention_tc_supported(const AttnArgs &a) {
     return a.dh == DH && a.kv_bf16 && a.R >= 1 && a.R <= 128 && a.B >= 1 && a.B <= MAX_B &&
+           a.tc_ctas / a.Hkv <= MAX_GRP &&
            (a.kv.layout == SP_KV_CONTIGUOUS ||
             (a.kv.page_size == 16 || a.kv.page_size == 32 || a.kv.page_size == 64));
 }
@@ -831,8 +927,10 @@ cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
     }
     CUtensorMap dummy;
     memset(&dummy, 0, sizeof dummy);
-    return launch_k(attn_tc_kernel, dim3(a.tc_ctas), dim3(THREADS), SMEM_BYTES, st,
-                    map_k ? *map_k : dummy, map_v ? *map_v : dummy, a);
+    cudaError_t e = launch_k(attn_tc_kernel, dim3(a.tc_ctas), dim3(THREADS), SMEM_BYTES, st,
+                             map_k ? *map_k : dummy, map_v ? *map_v : dummy, a);
+    if (e != cudaSuccess || !a.tc_merge_kernel) return e;
+    return launch_k(attn_tc_merge_kernel, dim3(a.Hkv, a.B, a.R), dim3(DH), 0, st, a);
 }
 
 }  // namespace sp

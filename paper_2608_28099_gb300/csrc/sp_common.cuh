@@ -205,6 +205,8 @@ struct AttnArgs {
     int subs;                     // partials per work unit (1)
     int tc_ctas;                  // tensor-core kernel: persistent CTAs (one per SM)
     int tc_min_tiles;             // tensor-core kernel: fewest 64-token tiles per CTA
+    int tc_merge_kernel;          // tensor-core kernel: 1 = merge in a second kernel (small
+                                  // batches), 0 = inside the attention kernel
     float *part_o;                // CUDA cores: [B][Hkv][n_splits][subs][R][dh]; tensor
                                   // cores: [tc_ctas + B Hkv][R][dh] (slot c + pair); unnormalised
     float *part_ml;               // same slots, [R][2] each (max in log2 units, sum)
@@ -224,14 +226,15 @@ void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, in
 // attn_tc_ctas(n_sm, Hkv) + B Hkv slots (tensor cores).
 size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits, int n_sm);
 // Default fewest tiles per CTA of the tensor-core kernel (64 tokens each).
-constexpr int kAttnMinTiles = 4;
+constexpr int kAttnMinTiles = 8;
 // Persistent CTAs of the tensor-core kernel: whole groups of Hkv (one CTA per
 // kv head), as many groups as the SMs hold, at least one.
 inline int attn_tc_ctas(int n_sm, int Hkv) { return (n_sm / Hkv > 1 ? n_sm / Hkv : 1) * Hkv; }
 cudaError_t launch_attention_simt(const AttnArgs &a, cudaStream_t st);
 // tcgen05 kernel: head_dim 128, bf16 cache, R <= 128, B <= 2048; paged caches
 // need TMA maps of the K and V pools from encode_kv_pages_bf16.  The merge
-// runs inside it (counters must be zero at launch).
+// runs inside it (counters must be zero at launch) or, with tc_merge_kernel,
+// in a second kernel launched behind it (two launches).
 bool attention_tc_supported(const AttnArgs &a);
 cudaError_t launch_attention_tc(const AttnArgs &a, const CUtensorMap *map_k,
                                 const CUtensorMap *map_v, cudaStream_t st);

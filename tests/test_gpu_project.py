@@ -15,7 +15,9 @@ SHAPES = [(1, 128, 64), (5, 256, 192), (16, 128, 2560), (17, 384, 640), (64, 128
           # tile counts that fill the SMs badly take the persistent stream-K
           # schedule (two partial planes, zero-filled where a tile has one
           # segment; several row tiles)
-          (1, 24576, 4096), (20, 20480, 256), (512, 6144, 4096)]
+          (1, 24576, 4096), (20, 20480, 256), (512, 6144, 4096),
+          # partial warps of rows, one k-block, a gate/up-sized product
+          (33, 2560, 9728), (127, 256, 64), (128, 19456, 2560)]
 
 
 def run(M, N, K, path, seed):
