@@ -34,6 +34,12 @@ Readings where the paper is silent (each is listed in the design notes):
 7. head: logits = W_head pooled + bias (bias zero when absent); raw logits, no
    sigmoid.
 8. no final norm before the head; no projection biases.
+9. input fusion (Sec. 3.1, MTP architecture): the layer input is
+   x = W_fc [RMSNorm(h; g_h) ; RMSNorm(e; g_e)] with W_fc stored [d][2d], the
+   normalised hidden state first and the normalised embedding second (the
+   order the paper lists them in); for probing, e is soft-prompt row r and h the
+   base model's last hidden state of the sequence (Sec. 3.2, single-step
+   probing), the same h for all k rows in the parallel form.
 """
 from __future__ import annotations
 
@@ -146,6 +152,18 @@ class Layer:
         self.head_w = np.asarray(weights.head_w, dtype=np.float64)
         self.head_b = (np.zeros(self.head_w.shape[0]) if weights.head_b is None
                        else np.asarray(weights.head_b, dtype=np.float64))
+        fc = getattr(weights, "w_fc", None)
+        self.w_fc = None if fc is None else to_f64(fc, wd)
+        self.g_h = None if fc is None else np.asarray(weights.g_h, dtype=np.float64)
+        self.g_e = None if fc is None else np.asarray(weights.g_e, dtype=np.float64)
+
+    # -- input fusion (reading 9) ---------------------------------------------
+    def fuse(self, hidden: np.ndarray, embed: np.ndarray) -> np.ndarray:
+        """x = W_fc [RMSNorm(h; g_h) ; RMSNorm(e; g_e)] for matching rows of
+        hidden [T, d] and embed [T, d].  Returns [T, d]."""
+        eps = self.shape.rms_eps
+        z = np.concatenate([rms_norm(hidden, self.g_h, eps), rms_norm(embed, self.g_e, eps)], axis=-1)
+        return z @ self.w_fc.T
 
     # -- pieces of the layer -------------------------------------------------
     def project_qkv(self, x: np.ndarray, positions: np.ndarray):
@@ -239,14 +257,22 @@ def sequence_kv(cache, seq_id: int):
     return to_f64(kp, cache.dtype), to_f64(vp, cache.dtype)
 
 
-def classify(layer: Layer, cache, seq_ids, rows=None, traces: list | None = None) -> np.ndarray:
+def classify(layer: Layer, cache, seq_ids, rows=None, traces: list | None = None,
+             hidden=None) -> np.ndarray:
     """Logits [B, C] (float64) for the sequences `seq_ids` of `cache`.
 
     rows: None (every sequence uses the shared soft prompt) or stored
-    per-sequence rows [B, k, d] in the layer's weight dtype."""
+    per-sequence rows [B, k, d] in the layer's weight dtype.
+    hidden: stored base hidden states [B, d] (weight dtype): the rows are then
+    the fused inputs of the soft prompt (reading 9) and `rows` is ignored."""
     out = []
+    k = layer.soft_prompt.shape[0]
     for i, sid in enumerate(np.asarray(seq_ids)):
-        x = layer.soft_prompt if rows is None else to_f64(rows[i], layer.shape.w_dtype)
+        if hidden is not None:
+            h = np.repeat(to_f64(hidden[i], layer.shape.w_dtype)[None, :], k, axis=0)
+            x = layer.fuse(h, layer.soft_prompt)
+        else:
+            x = layer.soft_prompt if rows is None else to_f64(rows[i], layer.shape.w_dtype)
         kc, vc = sequence_kv(cache, int(sid))
         tr = {} if traces is not None else None
         h2 = layer.rows_with_cache(x, kc, vc, trace=tr)

@@ -23,6 +23,8 @@ Sec. 6):
   seeded random permutation; page layout is [page][kv_head][slot][head_dim].
 * contiguous caches: one buffer, sequence b at a token offset, token-major
   [token][kv_head][head_dim].
+* input fusion (optional): a fifth stream draws W_fc [d][2d] N(0, 0.02), the
+  two fusion norm gains 1 + N(0, 0.02) and base hidden states [B][d] N(0, 1).
 """
 from __future__ import annotations
 
@@ -87,6 +89,7 @@ class WorkloadSpec:
     layout: int
     seed: int
     rows_per_seq: bool = False   # draw per-sequence input rows [B][k][d]
+    fused: bool = False          # draw fusion weights and per-sequence hidden states [B][d]
     head_bias: bool = False
     ragged_frac: Optional[float] = None  # sweep: L uniform in [(1-f)L, (1+f)L]
 
@@ -158,6 +161,11 @@ class Weights:
     soft_prompt: np.ndarray  # w_dtype [k][d]
     head_w: np.ndarray     # float32 [C][d]
     head_b: Optional[np.ndarray]  # float32 [C] or None
+    # input fusion in front of the layer (MTP): w_dtype [d][2d] and its two
+    # RMSNorm gains, float32 [d]; None when rows are given directly
+    w_fc: Optional[np.ndarray] = None
+    g_h: Optional[np.ndarray] = None
+    g_e: Optional[np.ndarray] = None
 
 
 @dataclasses.dataclass
@@ -196,6 +204,7 @@ class Workload:
     cache: KVCache
     seq_ids: np.ndarray             # int32 [B] (which cache sequences are classified)
     rows: Optional[np.ndarray]      # w_dtype [B][k][d] or None (shared soft prompt)
+    hidden: Optional[np.ndarray] = None  # w_dtype [B][d]: base hidden states (fused input)
 
     @property
     def shape(self) -> Shape:
@@ -233,6 +242,26 @@ def draw_weights(shape: Shape, rng, head_bias: bool) -> Weights:
     head_b = (0.02 * rng.standard_normal(C)).astype(np.float32) if head_bias else None
     return Weights(w_q, w_k, w_v, w_o, w_gate, w_up, w_down, g_in, g_post,
                    soft_prompt, head_w, head_b)
+
+
+def draw_fusion(shape: Shape, seed: int, batch: int):
+    """Input-fusion weights and base hidden states from a fifth stream of the
+    seed (the first four are untouched): W_fc [d][2d] N(0, 0.02), gains
+    1 + N(0, 0.02), hidden states [B][d] N(0, 1)."""
+    rng = np.random.default_rng(np.random.SeedSequence(seed).spawn(5)[4])
+    d, wd = shape.d_model, shape.w_dtype
+    w_fc = _normal(rng, (d, 2 * d), 0.02, wd)
+    g_h = (1.0 + 0.02 * rng.standard_normal(d)).astype(np.float32)
+    g_e = (1.0 + 0.02 * rng.standard_normal(d)).astype(np.float32)
+    hidden = _normal(rng, (batch, d), 1.0, wd)
+    return w_fc, g_h, g_e, hidden
+
+
+def with_fusion(w: "Workload") -> "Workload":
+    """The same workload with fusion weights and hidden states attached."""
+    w_fc, g_h, g_e, hidden = draw_fusion(w.spec.shape, w.spec.seed, len(w.seq_ids))
+    weights = dataclasses.replace(w.weights, w_fc=w_fc, g_h=g_h, g_e=g_e)
+    return dataclasses.replace(w, weights=weights, hidden=hidden)
 
 
 def draw_cache(shape: Shape, lens: np.ndarray, layout: int, rng_struct, rng_kv) -> KVCache:
@@ -292,7 +321,8 @@ def generate(spec: WorkloadSpec) -> Workload:
         rows = _normal(np.random.default_rng(s_rows), (spec.batch, sh.k_rows, sh.d_model), 0.02,
                        sh.w_dtype)
     seq_ids = np.arange(spec.batch, dtype=np.int32)
-    return Workload(spec, weights, cache, seq_ids, rows)
+    w = Workload(spec, weights, cache, seq_ids, rows)
+    return with_fusion(w) if spec.fused else w
 
 
 @dataclasses.dataclass

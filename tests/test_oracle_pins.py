@@ -34,6 +34,9 @@ class W:
     soft_prompt: np.ndarray
     head_w: np.ndarray
     head_b: np.ndarray = None
+    w_fc: np.ndarray = None    # input fusion (optional)
+    g_h: np.ndarray = None
+    g_e: np.ndarray = None
 
 
 def f32(a):
@@ -253,7 +256,66 @@ def check_cache_untouched():
     assert before == after
 
 
-ALL_CHECKS = [check_hand_example, check_rope_pairs, check_rope_relative_and_norm,
+def check_fusion_hand_example():
+    g = read_golden("fusion_hand_d2.txt")
+    sh = wl.Shape(2, 1, 1, 2, 1, 1, 2, rms_eps=0.0, w_dtype=wl.F32, kv_dtype=wl.F32)
+    _, w = random_layer(30, d=2, hq=1, hkv=1, dh=2, f=1, k=1, C=2)
+    w = dataclasses.replace(w, w_fc=f32(np.reshape(g["w_fc"], (2, 4))), g_h=f32(g["g_h"]),
+                            g_e=f32(g["g_e"]))
+    layer = so.Layer(sh, w)
+    x = layer.fuse(np.array([g["h"]]), np.array([g["e"]]))
+    np.testing.assert_allclose(x.ravel(), g["x"], atol=1e-9)
+
+
+def fused_layer(seed, w_fc_kind, unit_rows=False):
+    sh, w = random_layer(seed, k=3)
+    d = sh.d_model
+    rng = np.random.default_rng(seed + 100)
+    if w_fc_kind == "embed_only":      # [0 | I]
+        fc = np.concatenate([np.zeros((d, d)), np.eye(d)], axis=1)
+    elif w_fc_kind == "hidden_only":   # [I | 0]
+        fc = np.concatenate([np.eye(d), np.zeros((d, d))], axis=1)
+    else:
+        fc = 0.3 * rng.standard_normal((d, 2 * d))
+    w.w_fc = f32(fc)
+    w.g_h = f32(1 + 0.1 * rng.standard_normal(d))
+    w.g_e = f32(np.ones(d)) if w_fc_kind == "embed_only" else f32(1 + 0.1 * rng.standard_normal(d))
+    if unit_rows:
+        e = rng.standard_normal(w.soft_prompt.shape)
+        w.soft_prompt = f32(e / np.sqrt(np.mean(e * e, axis=1, keepdims=True)))
+    return sh, w
+
+
+def check_fusion_with_embedding_only_is_the_row_path():
+    # W_fc = [0 | I], unit gain, eps 0, unit-RMS soft prompt: the fused rows are
+    # the soft-prompt rows themselves, whatever the hidden state
+    sh, w = fused_layer(31, "embed_only", unit_rows=True)
+    sh = dataclasses.replace(sh, rms_eps=0.0)
+    layer = so.Layer(sh, w)
+    cw = wl.custom(sh, [6, 11], wl.LAYOUT_CONTIGUOUS, 32)
+    hidden = f32(np.random.default_rng(33).standard_normal((2, sh.d_model)) * 3)
+    fused = so.classify(layer, cw.cache, cw.seq_ids, hidden=hidden)
+    plain = so.classify(layer, cw.cache, cw.seq_ids)
+    np.testing.assert_allclose(fused, plain, rtol=1e-5, atol=1e-6)
+
+
+def check_fusion_with_hidden_only_ignores_the_prompt():
+    # W_fc = [I | 0]: the soft prompt no longer reaches the layer
+    sh, w = fused_layer(34, "hidden_only")
+    cw = wl.custom(sh, [4, 9], wl.LAYOUT_PAGED, 35)
+    hidden = f32(np.random.default_rng(36).standard_normal((2, sh.d_model)))
+    a = so.classify(so.Layer(sh, w), cw.cache, cw.seq_ids, hidden=hidden)
+    w2 = dataclasses.replace(w, soft_prompt=f32(w.soft_prompt[::-1] * 2 + 1))
+    b = so.classify(so.Layer(sh, w2), cw.cache, cw.seq_ids, hidden=hidden)
+    np.testing.assert_allclose(a, b, rtol=0, atol=1e-12)
+    # and it does depend on the hidden state
+    c = so.classify(so.Layer(sh, w), cw.cache, cw.seq_ids, hidden=f32(hidden * -1 + 0.5))
+    assert np.max(np.abs(a - c)) > 1e-6
+
+
+ALL_CHECKS = [check_fusion_hand_example, check_fusion_with_embedding_only_is_the_row_path,
+              check_fusion_with_hidden_only_ignores_the_prompt,
+              check_hand_example, check_rope_pairs, check_rope_relative_and_norm,
               check_softmax_rows_sum_to_one, check_incremental_equals_full_recompute,
               check_gqa_equals_mha_with_repeated_kv, check_attention_matches_torch_sdpa,
               check_uniform_keys_give_mean_of_values, check_rms_norm, check_silu,
@@ -353,7 +415,37 @@ def _gather_reversed(orig):
     return f
 
 
+def _fusion_order_swapped(orig):
+    def f(self, hidden, embed):
+        eps = self.shape.rms_eps
+        z = np.concatenate([so.rms_norm(embed, self.g_e, eps), so.rms_norm(hidden, self.g_h, eps)],
+                           axis=-1)
+        return z @ self.w_fc.T
+    return f
+
+
+def _fusion_gains_swapped(orig):
+    def f(self, hidden, embed):
+        self.g_h, self.g_e = self.g_e, self.g_h
+        try:
+            return orig(self, hidden, embed)
+        finally:
+            self.g_h, self.g_e = self.g_e, self.g_h
+    return f
+
+
+def _fusion_hidden_unnormalised(orig):
+    def f(self, hidden, embed):
+        eps = self.shape.rms_eps
+        z = np.concatenate([hidden * self.g_h, so.rms_norm(embed, self.g_e, eps)], axis=-1)
+        return z @ self.w_fc.T
+    return f
+
+
 MUTANTS = {
+    "fusion_order_swapped": (so.Layer, "fuse", _fusion_order_swapped),
+    "fusion_gains_swapped": (so.Layer, "fuse", _fusion_gains_swapped),
+    "fusion_hidden_unnormalised": (so.Layer, "fuse", _fusion_hidden_unnormalised),
     "rope_direction_flipped": (so, "rope", _rope_flipped),
     "rope_interleaved_pairs": (so, "rope", _rope_interleaved),
     "softmax_scale_1_over_dh": (so, "attention_probs", _scale_1_over_dh),
