@@ -58,9 +58,11 @@ def parse_args():
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--workload", default="4b")
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--rows", default="per-seq", choices=["per-seq", "shared"],
+    p.add_argument("--rows", default="per-seq", choices=["per-seq", "shared", "hidden"],
                    help="per-seq: per-sequence input rows (full layer per call); "
-                        "shared: the soft prompt, whose Q/K/V projection is precomputed")
+                        "shared: the soft prompt, whose Q/K/V projection is precomputed; "
+                        "hidden: base hidden states through the MTP input fusion "
+                        "(sp_classify_hidden)")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "quick"],
@@ -81,7 +83,7 @@ def peaks():
 # --------------------------------------------------------------------------- #
 # the algorithmic work model (bytes and flops every stage must move/do)
 # --------------------------------------------------------------------------- #
-def work_model(w, per_seq_rows: bool):
+def work_model(w, per_seq_rows: bool, fused: bool = False):
     sh = w.shape
     B, k, d = len(w.seq_ids), sh.k_rows, sh.d_model
     hq, hkv, dh, f, C = sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.d_ff, sh.n_classes
@@ -95,7 +97,10 @@ def work_model(w, per_seq_rows: bool):
         return {"bytes": N * K * es + M * K * es + M * N * es, "flops": 2 * M * N * K}
 
     st = {}
-    if per_seq_rows:
+    if fused:
+        # RMSNorm of the B hidden states and their projection by W_fc's hidden half
+        st["fusion"] = {"bytes": d * d * es + 2 * B * d * es + M * d * 4, "flops": 2 * B * d * d}
+    if per_seq_rows or fused:
         st["qkv"] = gemm(nqkv, d)
     kv_bytes = int(lens.sum()) * hkv * dh * 2 * kes
     st["attention"] = {"bytes": kv_bytes + M * nqkv * 4 + M * hq * dh * 4,
@@ -105,7 +110,8 @@ def work_model(w, per_seq_rows: bool):
     st["down"] = gemm(d, f)
     st["readout"] = {"bytes": C * d * 4 + M * d * 4, "flops": 2 * B * C * d}
     total_bytes = sum(v["bytes"] for v in st.values())
-    weight_bytes = ((nqkv * d if per_seq_rows else 0) + d * hq * dh + 3 * f * d) * es + C * d * 4
+    weight_bytes = ((nqkv * d if (per_seq_rows or fused) else 0) + (d * d if fused else 0)
+                    + d * hq * dh + 3 * f * d) * es + C * d * 4
     return st, {"kv_bytes": kv_bytes, "weight_bytes": weight_bytes, "total_bytes": total_bytes,
                 "total_flops": sum(v["flops"] for v in st.values())}
 
@@ -178,7 +184,8 @@ def cores():
 
 
 def oracle_rate(w, per_seq_rows: bool, seconds: float, max_seqs: int | None = None):
-    """Sequences/s of the oracle over successive sequences of the workload."""
+    """Sequences/s of the oracle over successive sequences of the workload
+    (through the input fusion when the workload carries hidden states)."""
     import oracle.sp_oracle as so
     layer = so.Layer(w.shape, w.weights)
     n = 0
@@ -187,7 +194,8 @@ def oracle_rate(w, per_seq_rows: bool, seconds: float, max_seqs: int | None = No
     while True:
         i = n % B
         rows = w.rows[i:i + 1] if (per_seq_rows and w.rows is not None) else None
-        so.classify(layer, w.cache, w.seq_ids[i:i + 1], rows)
+        hid = w.hidden[i:i + 1] if w.hidden is not None else None
+        so.classify(layer, w.cache, w.seq_ids[i:i + 1], rows, hidden=hid)
         n += 1
         el = time.perf_counter() - t0
         if el >= seconds or (max_seqs is not None and n >= max_seqs):
@@ -206,8 +214,9 @@ def run_reference(args, spec, w, rank, world):
     for step in range(args.warmup + args.steps):
         ids = [(step * per_step + j) % B for j in range(per_step)]
         rows = w.rows[ids] if (per_seq and w.rows is not None) else None
+        hid = w.hidden[ids] if w.hidden is not None else None
         t0 = time.perf_counter()
-        so.classify(layer, w.cache, w.seq_ids[ids], rows)
+        so.classify(layer, w.cache, w.seq_ids[ids], rows, hidden=hid)
         el = time.perf_counter() - t0
         if step >= args.warmup:
             times.append(el)
@@ -239,7 +248,8 @@ def workload_config(spec, w, args):
             "kv_layout": "paged16" if w.cache.layout == 1 else "contiguous",
             "rows": args.rows, "seed": spec.seed,
             "l2": "flushed between steps (256 MiB write)",
-            "timing": "CUDA events per step around a CUDA-graph replay of one sp_classify"}
+            "timing": ("CUDA events per step around a CUDA-graph replay of one "
+                       + ("sp_classify_hidden" if w.hidden is not None else "sp_classify"))}
 
 
 # --------------------------------------------------------------------------- #
@@ -287,18 +297,26 @@ def run_ours(args, spec, w, rank, world):
     h = model.handle
     cache = sp.DeviceCache(w.cache)
     ids = torch.from_numpy(np.ascontiguousarray(w.seq_ids, dtype=np.int32)).cuda()
-    rows = None
+    fused = w.hidden is not None
+    rows = hidden = None
     if per_seq:
         r = np.ascontiguousarray(w.rows)
         rows = torch.from_numpy(r.view(np.int16) if r.dtype == np.uint16 else r).cuda()
+    if fused:
+        r = np.ascontiguousarray(w.hidden)
+        hidden = torch.from_numpy(r.view(np.int16) if r.dtype == np.uint16 else r).cuda()
     logits = torch.empty((B, w.shape.n_classes), dtype=torch.float32, device="cuda")
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     stream = torch.cuda.current_stream()
 
     def step():
         # the stream is looked up per call so that a graph capture sees its own
-        sp.sp_classify(h, torch.cuda.current_stream(), B, ids, cache.seq_lens, cache.desc, rows,
-                       logits)
+        if fused:
+            sp.sp_classify_hidden(h, torch.cuda.current_stream(), B, ids, cache.seq_lens,
+                                  cache.desc, hidden, logits)
+        else:
+            sp.sp_classify(h, torch.cuda.current_stream(), B, ids, cache.seq_lens, cache.desc,
+                           rows, logits)
 
     for _ in range(args.warmup):
         flush.zero_()
@@ -360,29 +378,35 @@ def run_ours(args, spec, w, rank, world):
     h_ids = torch.from_numpy(np.ascontiguousarray(w.seq_ids, dtype=np.int32)).pin_memory()
     h_lens = torch.from_numpy(np.ascontiguousarray(lens[w.seq_ids], dtype=np.int32)).pin_memory()
     h_rows = rows.cpu().pin_memory() if rows is not None else None
+    h_hidden = hidden.cpu().pin_memory() if hidden is not None else None
     h_logits = torch.empty((B, w.shape.n_classes), dtype=torch.float32).pin_memory()
     e2e_s = []
     for i in range(args.warmup + args.steps):
         flush.zero_()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
-        sp.sp_classify_host(h, stream, B, h_ids, h_lens, cache.desc, h_rows, h_logits)
+        if fused:
+            sp.sp_classify_hidden_host(h, stream, B, h_ids, h_lens, cache.desc, h_hidden, h_logits)
+        else:
+            sp.sp_classify_host(h, stream, B, h_ids, h_lens, cache.desc, h_rows, h_logits)
         el = time.perf_counter() - t0
         if i >= args.warmup:
             e2e_s.append(el)
     e2e_mean = rank_max(sum(e2e_s) / len(e2e_s), "cuda")
     h2d = h_ids.numel() * 4 + h_lens.numel() * 4 + (h_rows.numel() * h_rows.element_size()
                                                      if h_rows is not None else 0)
+    if h_hidden is not None:
+        h2d += h_hidden.numel() * h_hidden.element_size()
     d2h = h_logits.numel() * 4
 
     if rank != 0:
         model.close()
         return
     hbm, tfl, peak_src = peaks()
-    st_work, totals = work_model(w, per_seq)
+    st_work, totals = work_model(w, per_seq, fused)
     # dominant kernel: the stage with the largest device time
     named = {"attention": "attention", "qkv": "qkv", "o_proj": "o_proj", "gate_up": "gate_up",
-             "down": "down", "readout": "readout"}
+             "down": "down", "readout": "readout", "fusion": "fusion"}
     cand = {k: v for k, v in stage_ms.items() if k in named and k in st_work}
     dom = max(cand, key=cand.get)
     wk = st_work[dom]
@@ -575,7 +599,8 @@ def main():
             torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
             dist.init_process_group("nccl")
     from paper_2608_28099_gb300 import workloads as wl
-    spec = shard_spec(wl.named(args.workload, rows_per_seq=(args.rows == "per-seq")), rank)
+    spec = shard_spec(wl.named(args.workload, rows_per_seq=(args.rows == "per-seq"),
+                               fused=(args.rows == "hidden")), rank)
     w = wl.generate(spec)
     if args.impl == "reference":
         run_reference(args, spec, w, rank, world)

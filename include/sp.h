@@ -100,12 +100,20 @@ typedef struct sp_config {
  *   w_q [Hq*dh][d], w_k [Hkv*dh][d], w_v [Hkv*dh][d], w_o [d][Hq*dh],
  *   w_gate [d_ff][d], w_up [d_ff][d], w_down [d][d_ff],
  *   soft_prompt [k][d] (w_dtype), g_in [d], g_post [d] (float),
- *   head_w [C][d] (float), head_b [C] (float, may be NULL = zero bias). */
+ *   head_w [C][d] (float), head_b [C] (float, may be NULL = zero bias).
+ * Optional input fusion of an MTP draft layer (Sec. 3.1: the base model's
+ * hidden state and the input embedding are RMS-normalised, concatenated and
+ * projected by W_fc): w_fc [d][2d] (w_dtype; columns [0, d) act on the
+ * normalised hidden state, [d, 2d) on the normalised embedding), g_h [d] and
+ * g_e [d] (float) the two norm gains.  All three NULL: no fusion (then
+ * sp_classify_hidden returns SP_ERR_INVALID_ARG). */
 typedef struct sp_weights {
     const void *w_q, *w_k, *w_v, *w_o, *w_gate, *w_up, *w_down;
     const float *g_in, *g_post;
     const void *soft_prompt;
     const float *head_w, *head_b;
+    const void *w_fc;
+    const float *g_h, *g_e;
 } sp_weights;
 
 /* A resident key/value cache (Sec. 3.3): DEVICE pointers, borrowed for the
@@ -175,6 +183,28 @@ SP_API sp_status sp_classify_host(sp_handle *h, sp_stream stream, int batch, con
                            const int *h_seq_lens, const sp_kv_cache *kv, const void *h_rows,
                            float *h_logits);
 
+/* The classify path fed by base hidden states (Sec. 3.2, single-step probing:
+ * the soft prompt replaces the next token's embedding in the MTP input): the
+ * k input rows of sequence b are
+ *   x_{b,r} = W_fc [RMSNorm(h_b; g_h) ; RMSNorm(soft_prompt_r; g_e)],  r < k,
+ * evaluated in parallel at positions L_b..L_b+k-1 like sp_classify's rows.
+ *   d_hidden [batch][d] device, w_dtype, 16-byte aligned: the base model's
+ *            last hidden state of each classified sequence.
+ * Other arguments as sp_classify.  The handle must have been created with
+ * w_fc, g_h and g_e (SP_ERR_INVALID_ARG otherwise).  Enqueued on `stream`, no
+ * synchronisation, no allocation. */
+SP_API sp_status sp_classify_hidden(sp_handle *h, sp_stream stream, int batch,
+                                    const int *d_seq_ids, const int *d_seq_lens,
+                                    const sp_kv_cache *kv, const void *d_hidden, float *d_logits);
+
+/* sp_classify_hidden from HOST buffers (ids, lengths as in sp_classify_host;
+ * h_hidden [batch][d] w_dtype), logits copied back to h_logits; synchronises
+ * `stream` and returns any device status as SP_ERR_DEVICE_STATUS. */
+SP_API sp_status sp_classify_hidden_host(sp_handle *h, sp_stream stream, int batch,
+                                         const int *h_seq_ids, const int *h_seq_lens,
+                                         const sp_kv_cache *kv, const void *h_hidden,
+                                         float *h_logits);
+
 /* Synchronise `stream`, read and clear the handle's device status word.
  * Returns SP_OK, or SP_ERR_DEVICE_STATUS with the SP_DEV_* bits in *bits. */
 SP_API sp_status sp_check_status(sp_handle *h, sp_stream stream, int *bits);
@@ -212,7 +242,9 @@ enum {
     SP_STAGE_SWIGLU = 8,      /* a5: SwiGLU                                          */
     SP_STAGE_DOWN = 9,        /* a6: down projection                                 */
     SP_STAGE_READOUT = 10,    /* a6-a7: residual, pooling, linear head               */
-    SP_N_STAGES = 11
+    SP_STAGE_FUSION = 11,     /* input fusion: hidden-state norm and its W_fc
+                                 projection (sp_classify_hidden only)             */
+    SP_N_STAGES = 12
 };
 
 /* With SP_OPT_PROFILE on: synchronise on the last call's events and write the

@@ -21,12 +21,12 @@ SP_KV_CONTIGUOUS, SP_KV_PAGED = 0, 1
 SP_DEV_BAD_SEQ_ID, SP_DEV_BAD_LENGTH, SP_DEV_BAD_PAGE = 1, 2, 4
 SP_OPT_SPLIT_TOKENS, SP_OPT_GEMM_PATH, SP_OPT_ATTN_PATH, SP_OPT_PROFILE = 1, 2, 3, 4
 STAGES = ["input_norm", "qkv", "rope", "attention", "merge", "o_proj", "post_norm", "gate_up",
-          "swiglu", "down", "readout"]
+          "swiglu", "down", "readout", "fusion"]
 
 EXPORTED = ["sp_create", "sp_destroy", "sp_classify", "sp_classify_host", "sp_check_status",
             "sp_last_error", "sp_set_option", "sp_last_launch_count", "sp_attend_workspace_bytes",
             "sp_attend", "sp_stage_times", "sp_project_workspace_bytes", "sp_project",
-            "sp_attend_static"]
+            "sp_attend_static", "sp_classify_hidden", "sp_classify_hidden_host"]
 
 
 class sp_config(C.Structure):
@@ -39,7 +39,8 @@ class sp_config(C.Structure):
 
 class sp_weights(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("w_q", "w_k", "w_v", "w_o", "w_gate", "w_up", "w_down",
-                                           "g_in", "g_post", "soft_prompt", "head_w", "head_b")]
+                                           "g_in", "g_post", "soft_prompt", "head_w", "head_b",
+                                           "w_fc", "g_h", "g_e")]
 
 
 class sp_kv_cache(C.Structure):
@@ -79,6 +80,8 @@ def load_library(path: str | None = None):
     lib.sp_destroy.argtypes = [vp]
     lib.sp_classify.argtypes = [vp, vp, i, vp, vp, C.POINTER(sp_kv_cache), vp, vp]
     lib.sp_classify_host.argtypes = [vp, vp, i, vp, vp, C.POINTER(sp_kv_cache), vp, vp]
+    lib.sp_classify_hidden.argtypes = [vp, vp, i, vp, vp, C.POINTER(sp_kv_cache), vp, vp]
+    lib.sp_classify_hidden_host.argtypes = [vp, vp, i, vp, vp, C.POINTER(sp_kv_cache), vp, vp]
     lib.sp_check_status.argtypes = [vp, vp, ip]
     lib.sp_last_error.restype = C.c_char_p
     lib.sp_last_error.argtypes = []
@@ -152,6 +155,19 @@ def sp_classify(handle, stream, batch, seq_ids, seq_lens, kv: sp_kv_cache, rows,
 def sp_classify_host(handle, stream, batch, seq_ids, seq_lens, kv: sp_kv_cache, rows, logits):
     _check(load_library().sp_classify_host(handle, _stream(stream), int(batch), _ptr(seq_ids),
                                            _ptr(seq_lens), C.byref(kv), _ptr(rows), _ptr(logits)))
+
+
+def sp_classify_hidden(handle, stream, batch, seq_ids, seq_lens, kv: sp_kv_cache, hidden, logits):
+    _check(load_library().sp_classify_hidden(handle, _stream(stream), int(batch), _ptr(seq_ids),
+                                             _ptr(seq_lens), C.byref(kv), _ptr(hidden),
+                                             _ptr(logits)))
+
+
+def sp_classify_hidden_host(handle, stream, batch, seq_ids, seq_lens, kv: sp_kv_cache, hidden,
+                            logits):
+    _check(load_library().sp_classify_hidden_host(handle, _stream(stream), int(batch),
+                                                  _ptr(seq_ids), _ptr(seq_lens), C.byref(kv),
+                                                  _ptr(hidden), _ptr(logits)))
 
 
 def sp_check_status(handle, stream=None) -> int:
@@ -231,9 +247,15 @@ class Model:
             arrs[name] = np.ascontiguousarray(getattr(weights, name), dtype=np.float32)
         arrs["head_b"] = (None if weights.head_b is None
                           else np.ascontiguousarray(weights.head_b, dtype=np.float32))
+        fc = getattr(weights, "w_fc", None)
+        arrs["w_fc"] = None if fc is None else np.ascontiguousarray(fc)
+        for name in ("g_h", "g_e"):
+            arrs[name] = (None if fc is None
+                          else np.ascontiguousarray(getattr(weights, name), dtype=np.float32))
+        self._arrs = arrs  # host copies stay alive for the handle's lifetime (read at create)
         w = sp_weights(*[None if arrs[n] is None else arrs[n].ctypes.data for n in (
             "w_q", "w_k", "w_v", "w_o", "w_gate", "w_up", "w_down", "g_in", "g_post",
-            "soft_prompt", "head_w", "head_b")])
+            "soft_prompt", "head_w", "head_b", "w_fc", "g_h", "g_e")])
         self.cfg = make_config(shape, max_batch, max_seq_len)
         self.handle = sp_create(self.cfg, w)
 

@@ -78,6 +78,14 @@ struct sp_handle {
     void *stage_rows = nullptr;
     float *stage_logits = nullptr;
     float *readout_part = nullptr;  // [B][chunks][C] partial head dot products
+    // input fusion (optional): x_{b,r} = W_fc_h RMSNorm(h_b; g_h) + fc_prompt[r]
+    bool fused = false;
+    WeightMat w_fc_h;             // [d][d]: the columns of W_fc acting on the hidden state
+    float *g_h = nullptr;
+    float *fc_prompt = nullptr;   // [k][d] W_fc (embedding columns) RMSNorm(soft_prompt; g_e)
+    ActBuf xh;                    // normalised hidden states [max_batch][d]
+    float *xrows = nullptr;       // fused input rows [max_batch k][d] fp32
+    void *stage_hidden = nullptr; // host-entry staging [max_batch][d] w_dtype
     GemmPlanner gemm;
     // options
     int opt_split = 0, opt_gemm = 0, opt_attn = 0, opt_profile = 0;
@@ -297,6 +305,25 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     if (w->head_b &&
         (st = upload(h, (void **)&h->head_b, w->head_b, C * sizeof(float))) != SP_OK)
         return cleanup(st);
+    // input fusion: W_fc [d][2d] split into its hidden-state half (a projection
+    // of every call) and its embedding half (applied once to the soft prompt below)
+    std::vector<char> w_fc_e;
+    if (w->w_fc || w->g_h || w->g_e) {
+        if (!w->w_fc || !w->g_h || !w->g_e)
+            return cleanup(fail(SP_ERR_INVALID_ARG, "input fusion needs w_fc, g_h and g_e together"));
+        std::vector<char> wh((size_t)d * d * es);
+        w_fc_e.resize((size_t)d * d * es);
+        for (int i = 0; i < d; ++i) {
+            const char *row = (const char *)w->w_fc + (size_t)i * 2 * d * es;
+            memcpy(wh.data() + (size_t)i * d * es, row, (size_t)d * es);
+            memcpy(w_fc_e.data() + (size_t)i * d * es, row + (size_t)d * es, (size_t)d * es);
+        }
+        void *p_fc = nullptr;
+        if ((st = upload(h, &p_fc, wh.data(), wh.size())) != SP_OK) return cleanup(st);
+        init_weight(h->w_fc_h, p_fc, d, d, c.w_dtype == SP_BF16);
+        if ((st = upload(h, (void **)&h->g_h, w->g_h, d * sizeof(float))) != SP_OK) return cleanup(st);
+        h->fused = true;
+    }
 
     // rotary table: angle (position p, pair i) = p * theta^(-2i/dh), evaluated in double
     {
@@ -342,7 +369,11 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
                             M * d * es,                 // stage rows
                             (size_t)c.max_batch * C * 4,  // stage logits
                             (size_t)k * h->nqkv * 4,    // qkv_shared
-                            readout_scratch_bytes(c.max_batch, d, C)};  // readout partials
+                            readout_scratch_bytes(c.max_batch, d, C),   // readout partials
+                            h->fused ? (size_t)c.max_batch * d * 4 : 0,  // xh
+                            h->fused ? M * d * 4 : 0,                    // xrows
+                            h->fused ? (size_t)k * d * 4 : 0,            // fc_prompt
+                            h->fused ? (size_t)c.max_batch * d * es : 0};  // stage hidden
     for (size_t sz : sizes) total += align256(sz);
     void *arena = nullptr;
     if ((st = dev_alloc(h, &arena, total)) != SP_OK) return cleanup(st);
@@ -365,6 +396,11 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     h->stage_logits = (float *)h->arena.take(sizes[14]);
     h->qkv_shared = (float *)h->arena.take(sizes[15]);
     h->readout_part = (float *)h->arena.take(sizes[16]);
+    void *p_xh = h->arena.take(sizes[17]);
+    h->xrows = (float *)h->arena.take(sizes[18]);
+    h->fc_prompt = (float *)h->arena.take(sizes[19]);
+    h->stage_hidden = h->arena.take(sizes[20]);
+    if (h->fused) init_act(h->xh, p_xh, c.max_batch, d, h->w_fc_h.tc);
     init_act(h->xn, p_xn, (int)M, d, h->w_qkv.tc);
     init_act(h->o, p_o_act, (int)M, hq * dh, h->w_o.tc);
     init_act(h->n, p_n, (int)M, d, h->w_gu.tc);
@@ -381,6 +417,26 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
         if (e == cudaSuccess) e = cudaDeviceSynchronize();
         if (e != cudaSuccess)
             return cleanup(fail(SP_ERR_CUDA, "shared prompt projection failed: %s", cudaGetErrorString(e)));
+    }
+    // the soft prompt's share of the fused input: fc_prompt = W_fc_e RMSNorm(e; g_e),
+    // fp32, on CUDA cores (temporaries freed before returning)
+    if (h->fused) {
+        void *p_we = nullptr, *p_ge = nullptr, *p_en = nullptr;
+        cudaError_t e = cudaMalloc(&p_we, w_fc_e.size());
+        if (e == cudaSuccess) e = cudaMalloc(&p_ge, d * sizeof(float));
+        if (e == cudaSuccess) e = cudaMalloc(&p_en, (size_t)k * d * sizeof(float));
+        if (e == cudaSuccess) e = cudaMemcpy(p_we, w_fc_e.data(), w_fc_e.size(), cudaMemcpyHostToDevice);
+        if (e == cudaSuccess) e = cudaMemcpy(p_ge, w->g_e, d * sizeof(float), cudaMemcpyHostToDevice);
+        ActOut en = {(float *)p_en, nullptr, nullptr};
+        if (e == cudaSuccess)
+            e = launch_rmsnorm_rows(wb, h->soft_prompt, 0, (const float *)p_ge, c.rms_eps, k, d, en, 0);
+        if (e == cudaSuccess) e = launch_gemm_simt(wb, p_en, p_we, h->fc_prompt, k, d, d, 0);
+        if (e == cudaSuccess) e = cudaDeviceSynchronize();
+        cudaFree(p_we);
+        cudaFree(p_ge);
+        cudaFree(p_en);
+        if (e != cudaSuccess)
+            return cleanup(fail(SP_ERR_CUDA, "fused prompt projection failed: %s", cudaGetErrorString(e)));
     }
     *out = h;
     return SP_OK;
@@ -451,7 +507,7 @@ sp_status sp_stage_times(sp_handle *h, float *ms, int n) {
 
 static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const int *d_seq_ids,
                                const int *d_seq_lens, int lens_by_batch, const sp_kv_cache *kv,
-                               const void *d_rows, float *d_logits) {
+                               const void *d_rows, float *d_logits, const void *d_hidden = nullptr) {
     if (!h) return fail(SP_ERR_INVALID_ARG, "handle is NULL");
     const sp_config &c = h->cfg;
     if (batch < 1 || batch > c.max_batch)
@@ -463,6 +519,10 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         return fail(SP_ERR_INVALID_ARG, "batch %d exceeds n_seqs %d with implicit ids", batch, kv->n_seqs);
     if (d_rows && ((uintptr_t)d_rows & 15))
         return fail(SP_ERR_INVALID_ARG, "d_rows must be 16-byte aligned");
+    if (d_hidden && !h->fused)
+        return fail(SP_ERR_INVALID_ARG, "the handle was created without input fusion (w_fc)");
+    if (d_hidden && ((uintptr_t)d_hidden & 15))
+        return fail(SP_ERR_INVALID_ARG, "d_hidden must be 16-byte aligned");
 
     const int d = c.d_model, hq = c.n_q_heads, hkv = c.n_kv_heads, dh = c.head_dim, f = c.d_ff;
     const int k = c.k_rows, C = c.n_classes, G = hq / hkv;
@@ -485,7 +545,28 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
 
     // a1-a2: pre-norm, Q/K/V projection, rotation at positions L_b + r
     PartIn yqkv = {h->qkv_shared, 1, 0};
-    if (d_rows) {
+    if (d_hidden) {
+        // input fusion: u_b = W_fc_h RMSNorm(h_b; g_h); x_{b,r} = u_b + fc_prompt[r],
+        // stored for the residual, and x_hat = RMSNorm(x; g_in) for Q/K/V
+        const bool tc_fc = h->gemm.use_tc(h->w_fc_h, h->xh, h->opt_gemm);
+        int ns_fc = 1;
+        mark(SP_STAGE_FUSION, 0);
+        SP_CUDA(launch_rmsnorm_rows(wb, d_hidden, 0, h->g_h, c.rms_eps, batch, d, h->xh.out(tc_fc), st));
+        ++launches;
+        s = h->gemm.run(wb, h->opt_gemm, h->xh, h->w_fc_h, h->y, batch, h->status, st, &launches, &ns_fc);
+        mark(SP_STAGE_FUSION, 1);
+        if (s != SP_OK) return fail(s, "fusion projection launch failed");
+        mark(SP_STAGE_INPUT_NORM, 0);
+        SP_CUDA(launch_residual_norm(0, PartIn{h->y, ns_fc, (size_t)batch * d}, h->fc_prompt, k,
+                                     h->g_in, c.rms_eps, M, d, h->xrows, h->xn.out(tc_qkv), st, k));
+        mark(SP_STAGE_INPUT_NORM, 1);
+        ++launches;
+        mark(SP_STAGE_QKV, 0);
+        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns);
+        mark(SP_STAGE_QKV, 1);
+        if (s != SP_OK) return fail(s, "Q/K/V projection launch failed");
+        yqkv = PartIn{h->y, ns, stride_qkv};
+    } else if (d_rows) {
         mark(SP_STAGE_INPUT_NORM, 0);
         SP_CUDA(launch_rmsnorm_rows(wb, d_rows, 0, h->g_in, c.rms_eps, M, d, h->xn.out(tc_qkv), st));
         mark(SP_STAGE_INPUT_NORM, 1);
@@ -498,7 +579,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     }
     QkvRopeArgs r;
     r.y = yqkv;
-    r.shared = d_rows ? 0 : 1;
+    r.shared = (d_rows || d_hidden) ? 0 : 1;
     r.B = batch; r.k = k; r.Hq = hq; r.Hkv = hkv; r.dh = dh;
     r.seq_ids = d_seq_ids; r.seq_lens = d_seq_lens; r.lens_by_batch = lens_by_batch;
     r.n_seqs = kv->n_seqs; r.max_seq_len = c.max_seq_len;
@@ -538,14 +619,15 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     if (h->opt_profile) h->ev_used[SP_STAGE_ATTN] = h->ev_used[SP_STAGE_MERGE] = true;
 
     // a4: output projection + residual, post-norm
-    const void *x = d_rows ? d_rows : h->soft_prompt;
-    const int row_mod = d_rows ? 0 : k;
+    const void *x = d_hidden ? (const void *)h->xrows : d_rows ? d_rows : h->soft_prompt;
+    const int row_mod = (d_rows || d_hidden) ? 0 : k;
+    const int x_bf16 = d_hidden ? 0 : wb;
     mark(SP_STAGE_O_PROJ, 0);
     s = h->gemm.run(wb, h->opt_gemm, h->o, h->w_o, h->y, M, h->status, st, &launches, &ns);
     mark(SP_STAGE_O_PROJ, 1);
     if (s != SP_OK) return fail(s, "output projection launch failed");
     mark(SP_STAGE_POST_NORM, 0);
-    SP_CUDA(launch_residual_norm(wb, PartIn{h->y, ns, (size_t)M * d}, x, row_mod, h->g_post,
+    SP_CUDA(launch_residual_norm(x_bf16, PartIn{h->y, ns, (size_t)M * d}, x, row_mod, h->g_post,
                                  c.rms_eps, M, d, h->h1, h->n.out(tc_gu), st));
     mark(SP_STAGE_POST_NORM, 1);
     ++launches;
@@ -596,6 +678,39 @@ sp_status sp_classify_host(sp_handle *h, sp_stream stream, int batch, const int 
                                 cudaMemcpyHostToDevice, st));
     sp_status s = classify_impl(h, st, batch, h_seq_ids ? h->stage_ids : nullptr, h->stage_lens, 1,
                                 kv, h_rows ? h->stage_rows : nullptr, h->stage_logits);
+    if (s != SP_OK) return s;
+    SP_CUDA(cudaMemcpyAsync(h_logits, h->stage_logits, (size_t)batch * c.n_classes * sizeof(float),
+                            cudaMemcpyDeviceToHost, st));
+    int bits = 0;
+    return sp_check_status(h, stream, &bits);
+}
+
+sp_status sp_classify_hidden(sp_handle *h, sp_stream stream, int batch, const int *d_seq_ids,
+                             const int *d_seq_lens, const sp_kv_cache *kv, const void *d_hidden,
+                             float *d_logits) {
+    if (!d_hidden) return fail(SP_ERR_INVALID_ARG, "d_hidden is NULL");
+    return classify_impl(h, (cudaStream_t)stream, batch, d_seq_ids, d_seq_lens, 0, kv, nullptr,
+                         d_logits, d_hidden);
+}
+
+sp_status sp_classify_hidden_host(sp_handle *h, sp_stream stream, int batch, const int *h_seq_ids,
+                                  const int *h_seq_lens, const sp_kv_cache *kv,
+                                  const void *h_hidden, float *h_logits) {
+    if (!h) return fail(SP_ERR_INVALID_ARG, "handle is NULL");
+    const sp_config &c = h->cfg;
+    if (batch < 1 || batch > c.max_batch)
+        return fail(SP_ERR_INVALID_ARG, "batch %d outside 1..max_batch (%d)", batch, c.max_batch);
+    if (!h_seq_lens || !h_logits || !h_hidden)
+        return fail(SP_ERR_INVALID_ARG, "seq_lens, hidden and logits are required");
+    if (!h->fused) return fail(SP_ERR_INVALID_ARG, "the handle was created without input fusion (w_fc)");
+    cudaStream_t st = (cudaStream_t)stream;
+    if (h_seq_ids)
+        SP_CUDA(cudaMemcpyAsync(h->stage_ids, h_seq_ids, batch * sizeof(int), cudaMemcpyHostToDevice, st));
+    SP_CUDA(cudaMemcpyAsync(h->stage_lens, h_seq_lens, batch * sizeof(int), cudaMemcpyHostToDevice, st));
+    SP_CUDA(cudaMemcpyAsync(h->stage_hidden, h_hidden, (size_t)batch * c.d_model * h->es,
+                            cudaMemcpyHostToDevice, st));
+    sp_status s = classify_impl(h, st, batch, h_seq_ids ? h->stage_ids : nullptr, h->stage_lens, 1,
+                                kv, nullptr, h->stage_logits, h->stage_hidden);
     if (s != SP_OK) return s;
     SP_CUDA(cudaMemcpyAsync(h_logits, h->stage_logits, (size_t)batch * c.n_classes * sizeof(float),
                             cudaMemcpyDeviceToHost, st));

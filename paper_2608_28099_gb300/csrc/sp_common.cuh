@@ -263,10 +263,11 @@ struct QkvRopeArgs {
 };
 cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st);
 
-// h1 = x + y ; n = RMSNorm(h1) * gain   (x: input rows, bf16 or fp32)
+// h1 = x + y ; n = RMSNorm(h1) * gain   (x: input rows, bf16 or fp32; row m
+// reads x row m % row_mod (row_mod > 0) or m, and y row m / y_div)
 cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mod,
                                  const float *gain, float eps, int M, int d, float *h1, ActOut n,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int y_div = 1);
 
 // a[m][j] = silu(g) * u for gate/up columns laid out in blocks of `blk`
 // (gate block i at columns 2*i*blk.., up block right after it)

@@ -96,9 +96,11 @@ __global__ void qkv_rope_kernel(QkvRopeArgs a) {
     }
 }
 
-// h1 = x + y, n = RMSNorm(h1): one block per row, 4-element vectors.
+// h1 = x + y, n = RMSNorm(h1): one block per row, 4-element vectors.  Row m
+// reads x row (row_mod ? m % row_mod : m) and y row m / y_div.
 template <typename TX>
-__global__ void __launch_bounds__(1024) residual_norm_kernel(PartIn y, const TX *__restrict__ x,
+__global__ void __launch_bounds__(1024) residual_norm_kernel(PartIn y, int y_div,
+                                                             const TX *__restrict__ x,
                                                              int row_mod,
                                                              const float *__restrict__ gain,
                                                              float eps, int d,
@@ -113,7 +115,7 @@ __global__ void __launch_bounds__(1024) residual_norm_kernel(PartIn y, const TX 
     float ss = 0.f;
 #pragma unroll 2
     for (int c = threadIdx.x; c < nch; c += blockDim.x) {
-        const float4 yv = part_get4(y, (size_t)m * d + c * 4);
+        const float4 yv = part_get4(y, (size_t)(m / y_div) * d + c * 4);
         float4 v = make_float4(to_f(xr[c * 4]) + yv.x, to_f(xr[c * 4 + 1]) + yv.y,
                                to_f(xr[c * 4 + 2]) + yv.z, to_f(xr[c * 4 + 3]) + yv.w);
         *(float4 *)(hr + c * 4) = v;
@@ -306,12 +308,12 @@ cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st) {
 
 cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mod,
                                  const float *gain, float eps, int M, int d, float *h1, ActOut n,
-                                 cudaStream_t st) {
+                                 cudaStream_t st, int y_div) {
     if (x_bf16)
-        return launch_k(residual_norm_kernel<bf16>, dim3(M), dim3(kWideThreads), 0, st, y,
+        return launch_k(residual_norm_kernel<bf16>, dim3(M), dim3(kWideThreads), 0, st, y, y_div,
                         (const bf16 *)x, row_mod, gain, eps, d, h1, n);
     else
-        return launch_k(residual_norm_kernel<float>, dim3(M), dim3(kWideThreads), 0, st, y,
+        return launch_k(residual_norm_kernel<float>, dim3(M), dim3(kWideThreads), 0, st, y, y_div,
                         (const float *)x, row_mod, gain, eps, d, h1, n);
 }
 
