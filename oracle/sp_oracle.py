@@ -40,6 +40,12 @@ Readings where the paper is silent (each is listed in the design notes):
    order the paper lists them in); for probing, e is soft-prompt row r and h the
    base model's last hidden state of the sequence (Sec. 3.2, single-step
    probing), the same h for all k rows in the parallel form.
+10. recursive probing SP-k (Sec. 3.2, "Recursive probing"): step 1 fuses the
+   base hidden state h with soft-prompt row 1; step i > 1 fuses the layer output
+   of step i-1 with row i.  Step i is one layer pass of one row at position
+   L + i - 1 whose attention sees the cache and the new keys/values of steps
+   1..i (the KV caching of Fig. 2).  The head reads the pooled step outputs
+   (reading 2: MEAN by default, LAST = the k-th step's output).
 """
 from __future__ import annotations
 
@@ -278,6 +284,38 @@ def classify(layer: Layer, cache, seq_ids, rows=None, traces: list | None = None
         h2 = layer.rows_with_cache(x, kc, vc, trace=tr)
         if traces is not None:
             traces.append(tr)
+        out.append(layer.readout(h2))
+    return np.array(out).reshape(len(out), layer.head_w.shape[0])
+
+
+def classify_recursive(layer: Layer, cache, seq_ids, hidden, traces: list | None = None
+                       ) -> np.ndarray:
+    """Logits [B, C] of recursive probing (reading 10), one step at a time.
+
+    hidden: stored base hidden states [B, d] (weight dtype)."""
+    sh = layer.shape
+    k = layer.soft_prompt.shape[0]
+    out = []
+    for i, sid in enumerate(np.asarray(seq_ids)):
+        kc, vc = sequence_kv(cache, int(sid))
+        L = kc.shape[0]
+        prev = to_f64(hidden[i], sh.w_dtype)[None, :]          # [1, d]
+        keys, values = kc, vc
+        xs, outs = [], []
+        for step in range(k):
+            x = layer.fuse(prev, layer.soft_prompt[step:step + 1])        # [1, d]
+            q, k_new, v_new = layer.project_qkv(x, np.array([L + step]))
+            keys = np.concatenate([keys, k_new], axis=0)
+            values = np.concatenate([values, v_new], axis=0)
+            visible = np.ones((1, keys.shape[0]), dtype=bool)           # all earlier keys
+            o = attention(q, keys, values, visible, sh.group)
+            a = layer.finish(x, o)                                       # [1, d]
+            xs.append(x[0])
+            outs.append(a[0])
+            prev = a
+        h2 = np.array(outs)
+        if traces is not None:
+            traces.append({"x": np.array(xs), "h2": h2})
         out.append(layer.readout(h2))
     return np.array(out).reshape(len(out), layer.head_w.shape[0])
 

@@ -313,7 +313,58 @@ def check_fusion_with_hidden_only_ignores_the_prompt():
     assert np.max(np.abs(a - c)) > 1e-6
 
 
-ALL_CHECKS = [check_fusion_hand_example, check_fusion_with_embedding_only_is_the_row_path,
+def check_recursive_k1_equals_parallel_fused():
+    sh, w = fused_layer(40, "random")
+    sh = dataclasses.replace(sh, k_rows=1)
+    w = dataclasses.replace(w, soft_prompt=w.soft_prompt[:1])
+    layer = so.Layer(sh, w)
+    cw = wl.custom(sh, [0, 7, 12], wl.LAYOUT_CONTIGUOUS, 41)
+    hidden = f32(np.random.default_rng(42).standard_normal((3, sh.d_model)))
+    a = so.classify_recursive(layer, cw.cache, cw.seq_ids, hidden)
+    b = so.classify(layer, cw.cache, cw.seq_ids, hidden=hidden)
+    np.testing.assert_allclose(a, b, rtol=1e-12, atol=1e-12)
+
+
+def check_recursive_equals_stepwise_reconstruction():
+    # rebuild SP-k from pinned pieces, differently: at step i fuse the previous
+    # output with prompt row i, then run the parallel causal path over ALL rows
+    # so far and take its last output
+    for pool in (wl.POOL_MEAN, wl.POOL_LAST):
+        sh, w = fused_layer(43, "random")
+        sh = dataclasses.replace(sh, pool=pool)
+        layer = so.Layer(sh, w)
+        cw = wl.custom(sh, [0, 6, 11], wl.LAYOUT_PAGED, 44)
+        hidden = f32(np.random.default_rng(45).standard_normal((3, sh.d_model)))
+        got = so.classify_recursive(layer, cw.cache, cw.seq_ids, hidden)
+        for b in range(3):
+            kc, vc = so.sequence_kv(cw.cache, b)
+            prev = hidden[b].astype(np.float64)[None, :]
+            rows, outs = [], []
+            for i in range(sh.k_rows):
+                rows.append(layer.fuse(prev, layer.soft_prompt[i:i + 1])[0])
+                h2 = layer.rows_with_cache(np.array(rows), kc, vc)
+                outs.append(h2[-1])
+                prev = h2[-1:]
+            np.testing.assert_allclose(got[b], layer.readout(np.array(outs)), rtol=1e-9, atol=1e-12)
+
+
+def check_recursive_embedding_only_is_the_row_path():
+    # W_fc = [0 | I] with unit gain, eps 0, unit-RMS rows: every step's input is
+    # its prompt row, so the recursion is the causal pass over the prompt rows
+    sh, w = fused_layer(46, "embed_only", unit_rows=True)
+    sh = dataclasses.replace(sh, rms_eps=0.0)
+    layer = so.Layer(sh, w)
+    cw = wl.custom(sh, [3, 10], wl.LAYOUT_CONTIGUOUS, 47)
+    hidden = f32(np.random.default_rng(48).standard_normal((2, sh.d_model)))
+    a = so.classify_recursive(layer, cw.cache, cw.seq_ids, hidden)
+    b = so.classify(layer, cw.cache, cw.seq_ids)
+    np.testing.assert_allclose(a, b, rtol=1e-5, atol=1e-6)
+
+
+ALL_CHECKS = [check_recursive_k1_equals_parallel_fused,
+              check_recursive_equals_stepwise_reconstruction,
+              check_recursive_embedding_only_is_the_row_path,
+              check_fusion_hand_example, check_fusion_with_embedding_only_is_the_row_path,
               check_fusion_with_hidden_only_ignores_the_prompt,
               check_hand_example, check_rope_pairs, check_rope_relative_and_norm,
               check_softmax_rows_sum_to_one, check_incremental_equals_full_recompute,
@@ -442,7 +493,42 @@ def _fusion_hidden_unnormalised(orig):
     return f
 
 
+def _recursive_variant(feed_input=False, fixed_position=False, no_append=False, row_zero=False):
+    """classify_recursive with one planted mistake (same loop otherwise)."""
+    def f(layer, cache, seq_ids, hidden, traces=None):
+        sh = layer.shape
+        k = layer.soft_prompt.shape[0]
+        out = []
+        for i, sid in enumerate(np.asarray(seq_ids)):
+            kc, vc = so.sequence_kv(cache, int(sid))
+            L = kc.shape[0]
+            prev = so.to_f64(hidden[i], sh.w_dtype)[None, :]
+            keys, values, outs = kc, vc, []
+            for step in range(k):
+                e = layer.soft_prompt[0:1] if row_zero else layer.soft_prompt[step:step + 1]
+                x = layer.fuse(prev, e)
+                q, kn, vn = layer.project_qkv(x, np.array([L if fixed_position else L + step]))
+                ks = np.concatenate([kc if no_append else keys, kn], axis=0)
+                vs = np.concatenate([vc if no_append else values, vn], axis=0)
+                keys, values = ks, vs
+                o = so.attention(q, ks, vs, np.ones((1, ks.shape[0]), dtype=bool), sh.group)
+                a = layer.finish(x, o)
+                outs.append(a[0])
+                prev = x if feed_input else a
+            out.append(layer.readout(np.array(outs)))
+        return np.array(out)
+    return f
+
+
 MUTANTS = {
+    "recursion_feeds_layer_input": (so, "classify_recursive",
+                                    lambda orig: _recursive_variant(feed_input=True)),
+    "recursion_fixed_position": (so, "classify_recursive",
+                                 lambda orig: _recursive_variant(fixed_position=True)),
+    "recursion_forgets_new_keys": (so, "classify_recursive",
+                                   lambda orig: _recursive_variant(no_append=True)),
+    "recursion_reuses_first_prompt_row": (so, "classify_recursive",
+                                          lambda orig: _recursive_variant(row_zero=True)),
     "fusion_order_swapped": (so.Layer, "fuse", _fusion_order_swapped),
     "fusion_gains_swapped": (so.Layer, "fuse", _fusion_gains_swapped),
     "fusion_hidden_unnormalised": (so.Layer, "fuse", _fusion_hidden_unnormalised),
