@@ -63,6 +63,8 @@ def parse_args():
                         "shared: the soft prompt, whose Q/K/V projection is precomputed; "
                         "hidden: base hidden states through the MTP input fusion "
                         "(sp_classify_hidden)")
+    p.add_argument("--recursive", action="store_true",
+                   help="with --rows hidden: recursive probing SP-k (k single-row steps)")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--sweep", nargs="?", const="all", default=None, choices=["all", "quick"],
@@ -83,7 +85,7 @@ def peaks():
 # --------------------------------------------------------------------------- #
 # the algorithmic work model (bytes and flops every stage must move/do)
 # --------------------------------------------------------------------------- #
-def work_model(w, per_seq_rows: bool, fused: bool = False):
+def work_model(w, per_seq_rows: bool, fused: bool = False, recursive: bool = False):
     sh = w.shape
     B, k, d = len(w.seq_ids), sh.k_rows, sh.d_model
     hq, hkv, dh, f, C = sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.d_ff, sh.n_classes
@@ -112,8 +114,15 @@ def work_model(w, per_seq_rows: bool, fused: bool = False):
     total_bytes = sum(v["bytes"] for v in st.values())
     weight_bytes = ((nqkv * d if (per_seq_rows or fused) else 0) + (d * d if fused else 0)
                     + d * hq * dh + 3 * f * d) * es + C * d * 4
-    return st, {"kv_bytes": kv_bytes, "weight_bytes": weight_bytes, "total_bytes": total_bytes,
-                "total_flops": sum(v["flops"] for v in st.values())}
+    totals = {"kv_bytes": kv_bytes, "weight_bytes": weight_bytes, "total_bytes": total_bytes,
+              "total_flops": sum(v["flops"] for v in st.values())}
+    if recursive:
+        # k steps of one row per sequence: every step reads all weights and the
+        # cache again; the flops are those of the parallel form (B k rows in all)
+        call = {"bytes": k * (kv_bytes + weight_bytes), "flops": totals["total_flops"]}
+        return {"call": call}, {"kv_bytes": k * kv_bytes, "weight_bytes": k * weight_bytes,
+                                "total_bytes": call["bytes"], "total_flops": call["flops"]}
+    return st, totals
 
 
 # --------------------------------------------------------------------------- #
@@ -183,7 +192,8 @@ def cores():
         return os.cpu_count() or 1
 
 
-def oracle_rate(w, per_seq_rows: bool, seconds: float, max_seqs: int | None = None):
+def oracle_rate(w, per_seq_rows: bool, seconds: float, max_seqs: int | None = None,
+                recursive: bool = False):
     """Sequences/s of the oracle over successive sequences of the workload
     (through the input fusion when the workload carries hidden states)."""
     import oracle.sp_oracle as so
@@ -195,7 +205,10 @@ def oracle_rate(w, per_seq_rows: bool, seconds: float, max_seqs: int | None = No
         i = n % B
         rows = w.rows[i:i + 1] if (per_seq_rows and w.rows is not None) else None
         hid = w.hidden[i:i + 1] if w.hidden is not None else None
-        so.classify(layer, w.cache, w.seq_ids[i:i + 1], rows, hidden=hid)
+        if recursive:
+            so.classify_recursive(layer, w.cache, w.seq_ids[i:i + 1], hid)
+        else:
+            so.classify(layer, w.cache, w.seq_ids[i:i + 1], rows, hidden=hid)
         n += 1
         el = time.perf_counter() - t0
         if el >= seconds or (max_seqs is not None and n >= max_seqs):
@@ -216,7 +229,10 @@ def run_reference(args, spec, w, rank, world):
         rows = w.rows[ids] if (per_seq and w.rows is not None) else None
         hid = w.hidden[ids] if w.hidden is not None else None
         t0 = time.perf_counter()
-        so.classify(layer, w.cache, w.seq_ids[ids], rows, hidden=hid)
+        if recursive_mode(args):
+            so.classify_recursive(layer, w.cache, w.seq_ids[ids], hid)
+        else:
+            so.classify(layer, w.cache, w.seq_ids[ids], rows, hidden=hid)
         el = time.perf_counter() - t0
         if step >= args.warmup:
             times.append(el)
@@ -236,6 +252,10 @@ def run_reference(args, spec, w, rank, world):
     print(json.dumps(line), flush=True)
 
 
+def recursive_mode(args) -> bool:
+    return bool(args.recursive) and args.rows == "hidden"
+
+
 def workload_config(spec, w, args):
     sh = w.shape
     lens = w.cache.seq_lens[w.seq_ids]
@@ -247,6 +267,7 @@ def workload_config(spec, w, args):
             "n_classes": sh.n_classes,
             "kv_layout": "paged16" if w.cache.layout == 1 else "contiguous",
             "rows": args.rows, "seed": spec.seed,
+            "form": "recursive SP-k" if recursive_mode(args) else "parallel k rows",
             "l2": "flushed between steps (256 MiB write)",
             "timing": ("CUDA events per step around a CUDA-graph replay of one "
                        + ("sp_classify_hidden" if w.hidden is not None else "sp_classify"))}
@@ -295,6 +316,9 @@ def run_ours(args, spec, w, rank, world):
     lens = w.cache.seq_lens
     model = sp.Model(w.shape, w.weights, B, int(lens.max(initial=0)))
     h = model.handle
+    recursive = recursive_mode(args)
+    if recursive:
+        sp.sp_set_option(h, sp.SP_OPT_RECURSIVE, 1)
     cache = sp.DeviceCache(w.cache)
     ids = torch.from_numpy(np.ascontiguousarray(w.seq_ids, dtype=np.int32)).cuda()
     fused = w.hidden is not None
@@ -403,11 +427,14 @@ def run_ours(args, spec, w, rank, world):
         model.close()
         return
     hbm, tfl, peak_src = peaks()
-    st_work, totals = work_model(w, per_seq, fused)
+    st_work, totals = work_model(w, per_seq, fused, recursive)
     # dominant kernel: the stage with the largest device time
     named = {"attention": "attention", "qkv": "qkv", "o_proj": "o_proj", "gate_up": "gate_up",
              "down": "down", "readout": "readout", "fusion": "fusion"}
     cand = {k: v for k, v in stage_ms.items() if k in named and k in st_work}
+    if not cand:  # no per-stage markers (recursive form): the whole call
+        stage_ms = dict(stage_ms, call=ms)
+        cand = {"call": ms}
     dom = max(cand, key=cand.get)
     wk = st_work[dom]
     dur_s = stage_ms[dom] / 1e3
@@ -426,7 +453,7 @@ def run_ours(args, spec, w, rank, world):
     path_bytes = totals["total_bytes"]
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        rate, n, el = oracle_rate(w, per_seq, args.cpu_seconds)
+        rate, n, el = oracle_rate(w, per_seq, args.cpu_seconds, recursive=recursive)
         cpu = {"value": rate, "unit": UNIT, "cores": cores(), "kind": "oracle",
                "sample": f"{n} sequences of workload {spec.name} one at a time, {el:.1f} s"}
     value = world * B / (ms / 1e3)

@@ -223,10 +223,15 @@ enum {
                                  2 = tensor-core kernels wherever supported       */
     SP_OPT_ATTN_PATH = 3,     /* 0 = automatic, 1 = CUDA-core kernel only,
                                  2 = tensor-core kernel wherever supported        */
-    SP_OPT_PROFILE = 4        /* 1 = record CUDA events around every stage of
+    SP_OPT_PROFILE = 4,       /* 1 = record CUDA events around every stage of
                                  sp_classify on its stream (as external event
                                  nodes when the call is captured in a graph),
                                  0 = off (default)                              */
+    SP_OPT_RECURSIVE = 5      /* 1 = sp_classify_hidden runs recursive probing
+                                 SP-k (Sec. 3.2): k steps of one row each, step i
+                                 fusing step i-1's output with soft-prompt row i
+                                 (no per-stage event markers); 0 = the parallel
+                                 form (default)                                   */
 };
 
 /* Stages of sp_classify, in launch order. */

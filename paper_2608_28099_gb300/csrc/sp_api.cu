@@ -88,7 +88,8 @@ struct sp_handle {
     void *stage_hidden = nullptr; // host-entry staging [max_batch][d] w_dtype
     GemmPlanner gemm;
     // options
-    int opt_split = 0, opt_gemm = 0, opt_attn = 0, opt_profile = 0;
+    int opt_split = 0, opt_gemm = 0, opt_attn = 0, opt_profile = 0, opt_recursive = 0;
+    float *h2_all = nullptr;      // recursive probing: step outputs [k][max_batch][d] fp32
     int last_launches = 0;
     cudaEvent_t ev[SP_N_STAGES][2] = {};
     bool ev_used[SP_N_STAGES] = {};
@@ -373,7 +374,8 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
                             h->fused ? (size_t)c.max_batch * d * 4 : 0,  // xh
                             h->fused ? M * d * 4 : 0,                    // xrows
                             h->fused ? (size_t)k * d * 4 : 0,            // fc_prompt
-                            h->fused ? (size_t)c.max_batch * d * es : 0};  // stage hidden
+                            h->fused ? (size_t)c.max_batch * d * es : 0,  // stage hidden
+                            h->fused ? M * d * 4 : 0};                   // h2_all
     for (size_t sz : sizes) total += align256(sz);
     void *arena = nullptr;
     if ((st = dev_alloc(h, &arena, total)) != SP_OK) return cleanup(st);
@@ -400,6 +402,7 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     h->xrows = (float *)h->arena.take(sizes[18]);
     h->fc_prompt = (float *)h->arena.take(sizes[19]);
     h->stage_hidden = h->arena.take(sizes[20]);
+    h->h2_all = (float *)h->arena.take(sizes[21]);
     if (h->fused) init_act(h->xh, p_xh, c.max_batch, d, h->w_fc_h.tc);
     init_act(h->xn, p_xn, (int)M, d, h->w_qkv.tc);
     init_act(h->o, p_o_act, (int)M, hq * dh, h->w_o.tc);
@@ -478,6 +481,10 @@ sp_status sp_set_option(sp_handle *h, int key, int value) {
         if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad attention path");
         h->opt_attn = value;
         return SP_OK;
+    case SP_OPT_RECURSIVE:
+        if (value != 0 && value != 1) return fail(SP_ERR_INVALID_ARG, "bad recursion flag");
+        h->opt_recursive = value;
+        return SP_OK;
     case SP_OPT_PROFILE:
         if (value != 0 && value != 1) return fail(SP_ERR_INVALID_ARG, "bad profile flag");
         if (value && !h->ev[0][0]) {
@@ -505,6 +512,100 @@ sp_status sp_stage_times(sp_handle *h, float *ms, int n) {
     return SP_OK;
 }
 
+// Recursive probing SP-k (Sec. 3.2): k steps, each one layer pass of one row per
+// sequence.  Step i fuses the previous step's output (the base hidden state at
+// i = 0) with soft-prompt row i, sits at position L_b + i, appends its new key
+// and value to the k_new / v_new rows of the sequence and attends to the cache
+// and new rows 0..i.  Step outputs go to h2_all (step-major); the head reads
+// their pool.  The normalisation of a step's output for the next fusion is
+// fused into the kernel that forms it (residual + down projection).
+static sp_status recursive_impl(sp_handle *h, cudaStream_t st, int batch, const int *d_seq_ids,
+                                const int *d_seq_lens, int lens_by_batch, const sp_kv_cache *kv,
+                                const void *d_hidden, float *d_logits) {
+    const sp_config &c = h->cfg;
+    const int d = c.d_model, hq = c.n_q_heads, hkv = c.n_kv_heads, dh = c.head_dim, f = c.d_ff;
+    const int k = c.k_rows, C = c.n_classes, G = hq / hkv;
+    const int B = batch;
+    const int wb = c.w_dtype == SP_BF16;
+    const size_t Bd = (size_t)B * d;
+    int launches = 0;
+    sp_status s;
+    const bool tc_fc = h->gemm.use_tc(h->w_fc_h, h->xh, h->opt_gemm);
+    const bool tc_qkv = h->gemm.use_tc(h->w_qkv, h->xn, h->opt_gemm);
+    const bool tc_o = h->gemm.use_tc(h->w_o, h->o, h->opt_gemm);
+    const bool tc_gu = h->gemm.use_tc(h->w_gu, h->n, h->opt_gemm);
+    const bool tc_down = h->gemm.use_tc(h->w_down, h->a, h->opt_gemm);
+    for (bool &u : h->ev_used) u = false;
+    int ns = 1;
+    SP_CUDA(launch_rmsnorm_rows(wb, d_hidden, 0, h->g_h, c.rms_eps, B, d, h->xh.out(tc_fc), st));
+    ++launches;
+    // one split plan for every step: keys extend to L_b + k at the last step
+    int split_tokens = 0, n_splits = 0;
+    plan_attention(B, hkv, k, c.max_seq_len, h->opt_split, h->n_sm, &split_tokens, &n_splits);
+    for (int i = 0; i < k; ++i) {
+        // fusion: x_i = W_fc_h RMSNorm(prev; g_h) + fc_prompt[i]; x_hat = RMSNorm(x_i; g_in)
+        s = h->gemm.run(wb, h->opt_gemm, h->xh, h->w_fc_h, h->y, B, h->status, st, &launches, &ns);
+        if (s != SP_OK) return fail(s, "fusion projection launch failed");
+        SP_CUDA(launch_residual_norm(0, PartIn{h->y, ns, Bd}, h->fc_prompt + (size_t)i * d, 1, h->g_in,
+                                     c.rms_eps, B, d, h->xrows, h->xn.out(tc_qkv), st));
+        ++launches;
+        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, B, h->status, st, &launches, &ns);
+        if (s != SP_OK) return fail(s, "Q/K/V projection launch failed");
+        QkvRopeArgs r;
+        memset(&r, 0, sizeof r);
+        r.y = PartIn{h->y, ns, (size_t)B * h->nqkv};
+        r.shared = 0;
+        r.B = B; r.k = 1; r.Hq = hq; r.Hkv = hkv; r.dh = dh;
+        r.r0 = i; r.kn_stride = k;
+        r.seq_ids = d_seq_ids; r.seq_lens = d_seq_lens; r.lens_by_batch = lens_by_batch;
+        r.n_seqs = kv->n_seqs; r.max_seq_len = c.max_seq_len;
+        r.rope_cs = h->rope_cs;
+        r.q = h->q; r.k_new = h->k_new; r.v_new = h->v_new;
+        r.status = h->status;
+        r.zero_ints = attention_counters(h->attn_ws);
+        r.n_zero = B * hkv;
+        SP_CUDA(launch_qkv_rope(r, st));
+        ++launches;
+        AttnArgs a;
+        memset(&a, 0, sizeof a);
+        a.B = B; a.Hq = hq; a.Hkv = hkv; a.dh = dh; a.k = 1; a.G = G; a.R = G;
+        a.r0 = i; a.kn_stride = k;
+        a.kv_bf16 = c.kv_dtype == SP_BF16;
+        a.split_tokens = split_tokens;
+        a.n_splits = n_splits;
+        a.max_seq_len = c.max_seq_len;
+        a.seq_ids = d_seq_ids; a.seq_lens = d_seq_lens; a.lens_by_batch = lens_by_batch;
+        a.kv = to_dev(kv);
+        a.q = h->q; a.k_new = h->k_new; a.v_new = h->v_new;
+        a.status = h->status;
+        a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+        a.out = h->o.out(tc_o);
+        s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, h->n_sm, h->opt_split,
+                              &launches, st, true);
+        if (s != SP_OK) return s;
+        s = h->gemm.run(wb, h->opt_gemm, h->o, h->w_o, h->y, B, h->status, st, &launches, &ns);
+        if (s != SP_OK) return fail(s, "output projection launch failed");
+        SP_CUDA(launch_residual_norm(0, PartIn{h->y, ns, Bd}, h->xrows, 0, h->g_post, c.rms_eps, B, d,
+                                     h->h1, h->n.out(tc_gu), st));
+        ++launches;
+        s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, B, h->status, st, &launches, &ns);
+        if (s != SP_OK) return fail(s, "gate/up projection launch failed");
+        SP_CUDA(launch_swiglu(PartIn{h->y, ns, (size_t)B * 2 * f}, B, f, h->gu_blk, h->a.out(tc_down), st));
+        ++launches;
+        s = h->gemm.run(wb, h->opt_gemm, h->a, h->w_down, h->y, B, h->status, st, &launches, &ns);
+        if (s != SP_OK) return fail(s, "down projection launch failed");
+        // a_i = h1 + W_down a -> h2_all[i]; RMSNorm(a_i; g_h) is the next step's fusion input
+        SP_CUDA(launch_residual_norm(0, PartIn{h->y, ns, Bd}, h->h1, 0, h->g_h, c.rms_eps, B, d,
+                                     h->h2_all + (size_t)i * Bd, h->xh.out(tc_fc), st));
+        ++launches;
+    }
+    SP_CUDA(launch_readout(PartIn{nullptr, 0, 0}, h->h2_all, h->head_w, h->head_b, c.pool, B, k, d, C,
+                           h->readout_part, d_logits, st, (size_t)d, Bd));
+    launches += 2;
+    h->last_launches = launches;
+    return SP_OK;
+}
+
 static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const int *d_seq_ids,
                                const int *d_seq_lens, int lens_by_batch, const sp_kv_cache *kv,
                                const void *d_rows, float *d_logits, const void *d_hidden = nullptr) {
@@ -523,6 +624,9 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         return fail(SP_ERR_INVALID_ARG, "the handle was created without input fusion (w_fc)");
     if (d_hidden && ((uintptr_t)d_hidden & 15))
         return fail(SP_ERR_INVALID_ARG, "d_hidden must be 16-byte aligned");
+    if (d_hidden && h->opt_recursive)
+        return recursive_impl(h, st, batch, d_seq_ids, d_seq_lens, lens_by_batch, kv, d_hidden,
+                              d_logits);
 
     const int d = c.d_model, hq = c.n_q_heads, hkv = c.n_kv_heads, dh = c.head_dim, f = c.d_ff;
     const int k = c.k_rows, C = c.n_classes, G = hq / hkv;
@@ -578,6 +682,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         yqkv = PartIn{h->y, ns, stride_qkv};
     }
     QkvRopeArgs r;
+    memset(&r, 0, sizeof r);  // r0 = 0, kn_stride = 0 (= k): the parallel form
     r.y = yqkv;
     r.shared = (d_rows || d_hidden) ? 0 : 1;
     r.B = batch; r.k = k; r.Hq = hq; r.Hkv = hkv; r.dh = dh;

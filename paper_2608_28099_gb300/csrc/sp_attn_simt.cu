@@ -71,7 +71,8 @@ __global__ void __launch_bounds__(kThreads) attn_split_simt(AttnArgs a) {
     const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs, a.max_seq_len,
                                   (threadIdx.x == 0 && s == 0 && g == 0) ? a.status : nullptr);
     const int L = sq.len;
-    const int total = L + k;
+    const int total = L + a.r0 + k;
+    const int kns = a.kn_stride ? a.kn_stride : k;
     const int t_begin = s * a.split_tokens;
     if (t_begin >= total) return;  // the merge reads only units below ceil(total / split)
     const int t_end = min(total, t_begin + a.split_tokens);
@@ -109,7 +110,7 @@ __global__ void __launch_bounds__(kThreads) attn_split_simt(AttnArgs a) {
                             a.kv.page_table[(size_t)sq.sid * a.kv.max_pages + t / a.kv.page_size];
                 } else {
                     const int j = t - L;
-                    const size_t o = (((size_t)b * k + j) * a.Hkv + g) * DH + c;
+                    const size_t o = (((size_t)b * kns + j) * a.Hkv + g) * DH + c;
                     kv_k = a.k_new[o];
                     kv_v = a.v_new[o];
                 }
@@ -123,7 +124,7 @@ __global__ void __launch_bounds__(kThreads) attn_split_simt(AttnArgs a) {
             const int t = t0 + tt;
             const int r = rr % k;
             float sc = -INFINITY;
-            if (t < t_end && t <= L + r) {
+            if (t < t_end && t <= L + a.r0 + r) {
                 const float *qr = Qs + rr * DH;
                 const float *kr = Ks + tt * (DH + 1);
                 float acc = 0.f;
@@ -185,7 +186,7 @@ __global__ void attn_merge_kernel(AttnArgs a) {
     const int R = a.R, dh = a.dh, k = a.k;
     const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs,
                                   a.max_seq_len, nullptr);
-    const int n_valid = min(a.n_splits, ceil_div(sq.len + k, a.split_tokens)) * a.subs;
+    const int n_valid = min(a.n_splits, ceil_div(sq.len + a.r0 + k, a.split_tokens)) * a.subs;
     const size_t unit0 = ((size_t)b * a.Hkv + g) * a.n_splits * a.subs;
     const int c = threadIdx.x;
     float mmax = -INFINITY;

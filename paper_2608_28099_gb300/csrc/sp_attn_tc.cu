@@ -191,6 +191,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     volatile int *abort = &bars->abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int R = a.R, k = a.k, B = a.B, Hkv = a.Hkv;
+    const int kns = a.kn_stride ? a.kn_stride : k;  // rows per sequence of k_new / v_new
     const bool paged = a.kv.layout == SP_KV_PAGED;
     const int act_warps = (R + 31) / 32;  // softmax warps that own real query rows
     pdl_trigger();
@@ -205,7 +206,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int bb = b0; bb < b1; ++bb) {
             const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, bb, a.kv.n_seqs,
                                           a.max_seq_len, blockIdx.x == 0 ? a.status : nullptr);
-            const int v = ceil_div(sq.len + k, TT);
+            const int v = ceil_div(sq.len + a.r0 + k, TT);
             prefix[bb] = v;
             sum += v;
         }
@@ -300,7 +301,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int b = sg.b;
             const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs,
                                           a.max_seq_len, nullptr);
-            const int L = sq.len, total = L + k;
+            const int L = sq.len, total = L + a.r0 + k;
             const int *ptab = paged ? a.kv.page_table + (size_t)max(sq.sid, 0) * a.kv.max_pages : nullptr;
             for (int i = 0; i < sg.n; ++i, ++ci) {
                 const int st = ci % STG;
@@ -414,7 +415,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                             const int j = idx + u * pstride;
                             if (j < n_new * 16) {
                                 const int rr = (t0 + n_cache + (j >> 4)) - L, c16 = j & 15;
-                                const size_t o = (((size_t)b * k + rr) * Hkv + g) * DH + c16 * 8;
+                                const size_t o = (((size_t)b * kns + rr) * Hkv + g) * DH + c16 * 8;
                                 kf[u][0] = *(const float4 *)(a.k_new + o);
                                 kf[u][1] = *(const float4 *)(a.k_new + o + 4);
                                 vf[u][0] = *(const float4 *)(a.v_new + o);
@@ -585,8 +586,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                 n_tiles = sg.n;
                 const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, sg.b, a.kv.n_seqs,
                                               a.max_seq_len, nullptr);
-                // this row sees tokens t < min(L + k, L + r + 1); relative to the segment start:
-                lim_rel = min(sq.len + k, sq.len + r_soft + 1) - sg.t_a * TT;
+                // this row sees tokens t < L + r0 + r + 1; relative to the segment start:
+                lim_rel = sq.len + a.r0 + r_soft + 1 - sg.t_a * TT;
             }
             x += n_tiles;
             // this segment's queries are written, and the previous epilogue is complete
@@ -863,7 +864,7 @@ __global__ void __launch_bounds__(DH) attn_tc_merge_kernel(AttnArgs a) {
             prefix[bb] = run;
             const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, bb, a.kv.n_seqs,
                                           a.max_seq_len, nullptr);
-            run += ceil_div(sq.len + k, TT);
+            run += ceil_div(sq.len + a.r0 + k, TT);
         }
         prefix[B] = run;
     }

@@ -191,6 +191,9 @@ __device__ __forceinline__ SeqRef resolve_seq(const int *seq_ids, const int *seq
 // ---------------------------------------------------------------------------
 struct AttnArgs {
     int B, Hq, Hkv, dh, k, G, R;  // R = G * k query rows per (sequence, kv head)
+    int r0;                       // the pass's query row r is new row r0 + r (position
+                                  // L + r0 + r) and sees new keys 0..r0 + r
+    int kn_stride;                // rows per sequence of k_new / v_new (0 = k)
     int kv_bf16;                  // cache element type: 1 bf16, 0 fp32
     int split_tokens;             // tokens per work unit
     int n_splits;                 // work units per (sequence, kv head) in the grid
@@ -200,8 +203,8 @@ struct AttnArgs {
     int lens_by_batch;
     KVDev kv;
     const float *q;               // [B][k][Hq][dh], rotated
-    const float *k_new;           // [B][k][Hkv][dh], rotated
-    const float *v_new;           // [B][k][Hkv][dh]
+    const float *k_new;           // [B][kn_stride][Hkv][dh], rotated
+    const float *v_new;           // [B][kn_stride][Hkv][dh]
     int subs;                     // partials per work unit (1)
     int tc_ctas;                  // tensor-core kernel: persistent CTAs (one per SM)
     int tc_min_tiles;             // tensor-core kernel: fewest 64-token tiles per CTA
@@ -252,6 +255,8 @@ struct QkvRopeArgs {
     PartIn y;                // projections [rows][(Hq + 2 Hkv) dh]
     int shared;              // 1: row of m is m % k (shared soft prompt), 0: row m
     int B, k, Hq, Hkv, dh;
+    int r0;                  // row m = b k + r is new row r0 + r, at position L_b + r0 + r
+    int kn_stride;           // rows per sequence of k_new / v_new (0 = k)
     const int *seq_ids, *seq_lens;
     int lens_by_batch;
     int n_seqs, max_seq_len;
@@ -276,9 +281,11 @@ cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_
 // logits[b] = W_head pool_r(h1 + y) + bias, via per-chunk partial dot
 // products in `scratch` (readout_scratch_bytes); two launches.
 size_t readout_scratch_bytes(int B, int d, int C);
+// Row r of sequence b of (h1 + y) sits at b sb + r sr (0 = the dense [B][k][d]
+// strides k d and d).
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
                            int pool, int B, int k, int d, int C, float *scratch, float *logits,
-                           cudaStream_t st);
+                           cudaStream_t st, size_t sb = 0, size_t sr = 0);
 
 // ---------------------------------------------------------------------------
 // projections

@@ -80,19 +80,21 @@ __global__ void qkv_rope_kernel(QkvRopeArgs a) {
                            idx == 0 ? a.status : nullptr);
     const int nqkv = (a.Hq + 2 * a.Hkv) * dh;
     const size_t row = (size_t)(a.shared ? r : m) * nqkv;
+    const int kns = a.kn_stride ? a.kn_stride : a.k;
+    const size_t mn = (size_t)b * kns + a.r0 + r;  // row of k_new / v_new
     if (idx < nrot) {
-        const int pos = s.len + r;
+        const int pos = s.len + a.r0 + r;
         const int h = idx / half, i = idx - h * half;
         const float x0 = part_get(a.y, row + h * dh + i);
         const float x1 = part_get(a.y, row + h * dh + i + half);
         const float2 c = a.rope_cs[(size_t)pos * half + i];
         float *dst = h < a.Hq ? a.q + ((size_t)m * a.Hq + h) * dh
-                              : a.k_new + ((size_t)m * a.Hkv + (h - a.Hq)) * dh;
+                              : a.k_new + (mn * a.Hkv + (h - a.Hq)) * dh;
         dst[i] = x0 * c.x - x1 * c.y;
         dst[i + half] = x1 * c.x + x0 * c.y;
     } else {
         const int j = idx - nrot;
-        a.v_new[(size_t)m * nval + j] = part_get(a.y, row + (size_t)(a.Hq + a.Hkv) * dh + j);
+        a.v_new[mn * nval + j] = part_get(a.y, row + (size_t)(a.Hq + a.Hkv) * dh + j);
     }
 }
 
@@ -162,7 +164,7 @@ constexpr int kReadoutCols = 64;
 
 __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const float *__restrict__ h1,
                                        const float *__restrict__ head_w, int pool, int k, int d,
-                                       int C, float *__restrict__ part) {
+                                       int C, float *__restrict__ part, size_t sb, size_t sr) {
     pdl_trigger();
     pdl_wait();
     __shared__ float acc_s[4][kReadoutCols];
@@ -171,17 +173,17 @@ __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const fl
     const int chunk = blockIdx.x, b = blockIdx.y;
     const int c = threadIdx.x & (kReadoutCols - 1), rg = threadIdx.x / kReadoutCols;
     const int col = chunk * kReadoutCols + c;
-    const size_t base = (size_t)b * k * d;
+    const size_t base = (size_t)b * sb;
     float acc = 0.f;
     if (col < d) {
         if (pool == SP_POOL_LAST) {
             if (rg == 0) {
-                const size_t o = base + (size_t)(k - 1) * d + col;
+                const size_t o = base + (size_t)(k - 1) * sr + col;
                 acc = h1[o] + part_get(y, o);
             }
         } else {
             for (int r = rg; r < k; r += 4) {
-                const size_t o = base + (size_t)r * d + col;
+                const size_t o = base + (size_t)r * sr + col;
                 acc += h1[o] + part_get(y, o);
             }
         }
@@ -330,10 +332,12 @@ size_t readout_scratch_bytes(int B, int d, int C) {
 
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
                            int pool, int B, int k, int d, int C, float *scratch, float *logits,
-                           cudaStream_t st) {
+                           cudaStream_t st, size_t sb, size_t sr) {
     const int chunks = ceil_div(d, kReadoutCols);
+    if (!sb) sb = (size_t)k * d;
+    if (!sr) sr = d;
     cudaError_t e = launch_k(readout_partial_kernel, dim3(chunks, B), dim3(256), 0, st, y, h1,
-                             head_w, pool, k, d, C, scratch);
+                             head_w, pool, k, d, C, scratch, sb, sr);
     if (e != cudaSuccess) return e;
     return launch_k(readout_finish_kernel, dim3(B), dim3(64), 0, st, (const float *)scratch, chunks,
                     C, head_b, logits);

@@ -114,3 +114,56 @@ def test_hidden_entry_needs_fusion_weights():
                               run.cache.desc, hidden, out)
     assert e.value.status == sp.SP_ERR_INVALID_ARG
     run.close()
+
+
+# --------------------------------------------------------------------------- #
+# recursive probing SP-k (SP_OPT_RECURSIVE)
+# --------------------------------------------------------------------------- #
+REC_CASES = [
+    ("paged_k4", SMALL_BF16, [0, 17, 300, 1000, 64], wl.LAYOUT_PAGED, wl.POOL_MEAN),
+    ("contiguous_last", wl.Shape(256, 8, 2, 128, 512, 3, 2, pool=wl.POOL_LAST), [5, 129, 700],
+     wl.LAYOUT_CONTIGUOUS, wl.POOL_LAST),
+    ("k1", wl.Shape(256, 8, 2, 128, 512, 1, 2), [40, 2000], wl.LAYOUT_PAGED, wl.POOL_MEAN),
+    ("head_dim_64", wl.Shape(256, 8, 4, 64, 512, 5, 2), [90, 33, 250], wl.LAYOUT_PAGED,
+     wl.POOL_MEAN),
+]
+
+
+@pytest.mark.parametrize("name,shape,lens,layout,pool", REC_CASES, ids=[c[0] for c in REC_CASES])
+def test_recursive_probing_matches_oracle(name, shape, lens, layout, pool):
+    w = wl.with_fusion(wl.custom(shape, lens, layout, 211))
+    run = GpuRun(w, options={sp.SP_OPT_RECURSIVE: 1})
+    gpu = hidden_logits(run, w.hidden)
+    ref = so.classify_recursive(so.Layer(w.shape, w.weights), w.cache, w.seq_ids, w.hidden)
+    assert np.all(np.isfinite(gpu))
+    assert np.max(np.abs(ref)) > 0.05
+    compare(gpu, ref, label=f"recursive {name}")
+    # the parallel form of the same inputs differs for k > 1 (a real recursion ran)
+    if shape.k_rows > 1:
+        par = oracle_hidden(w)
+        assert np.max(np.abs(par - ref)) > 1e-3
+    run.close()
+
+
+def test_recursive_tiny_fp32_matches_oracle_tightly():
+    w = wl.generate(wl.named("tiny", fused=True))
+    run = GpuRun(w, options={sp.SP_OPT_RECURSIVE: 1})
+    gpu = hidden_logits(run, w.hidden)
+    ref = so.classify_recursive(so.Layer(w.shape, w.weights), w.cache, w.seq_ids, w.hidden)
+    scale = float(np.max(np.abs(ref)))
+    assert np.max(np.abs(gpu - ref)) <= 1e-5 * scale + 1e-7, (gpu, ref)
+    run.close()
+
+
+def test_recursive_then_parallel_on_one_handle():
+    # switching the option back restores the parallel form exactly
+    w = wl.with_fusion(wl.custom(SMALL_BF16, [80, 400], wl.LAYOUT_PAGED, 212))
+    run = GpuRun(w)
+    first = hidden_logits(run, w.hidden)
+    sp.sp_set_option(run.model.handle, sp.SP_OPT_RECURSIVE, 1)
+    rec = hidden_logits(run, w.hidden)
+    sp.sp_set_option(run.model.handle, sp.SP_OPT_RECURSIVE, 0)
+    again = hidden_logits(run, w.hidden)
+    assert np.array_equal(first, again)
+    assert np.max(np.abs(first - rec)) > 1e-3
+    run.close()
