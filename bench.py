@@ -63,6 +63,8 @@ def parse_args():
                         "shared: the soft prompt, whose Q/K/V projection is precomputed; "
                         "hidden: base hidden states through the MTP input fusion "
                         "(sp_classify_hidden)")
+    p.add_argument("--tasks", type=int, default=1,
+                   help="probes (soft prompt + head) sharing each pass over the cache")
     p.add_argument("--recursive", action="store_true",
                    help="with --rows hidden: recursive probing SP-k (k single-row steps)")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -87,8 +89,9 @@ def peaks():
 # --------------------------------------------------------------------------- #
 def work_model(w, per_seq_rows: bool, fused: bool = False, recursive: bool = False):
     sh = w.shape
-    B, k, d = len(w.seq_ids), sh.k_rows, sh.d_model
-    hq, hkv, dh, f, C = sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.d_ff, sh.n_classes
+    # T tasks stack T k rows per sequence and read T heads
+    B, k, d = len(w.seq_ids), sh.k_rows * sh.n_tasks, sh.d_model
+    hq, hkv, dh, f, C = sh.n_q_heads, sh.n_kv_heads, sh.head_dim, sh.d_ff, sh.n_classes * sh.n_tasks
     es = 2 if sh.w_dtype == 1 else 4
     kes = 2 if sh.kv_dtype == 1 else 4
     M = B * k
@@ -268,6 +271,7 @@ def workload_config(spec, w, args):
             "kv_layout": "paged16" if w.cache.layout == 1 else "contiguous",
             "rows": args.rows, "seed": spec.seed,
             "form": "recursive SP-k" if recursive_mode(args) else "parallel k rows",
+            "n_tasks": sh.n_tasks,
             "l2": "flushed between steps (256 MiB write)",
             "timing": ("CUDA events per step around a CUDA-graph replay of one "
                        + ("sp_classify_hidden" if w.hidden is not None else "sp_classify"))}
@@ -329,7 +333,8 @@ def run_ours(args, spec, w, rank, world):
     if fused:
         r = np.ascontiguousarray(w.hidden)
         hidden = torch.from_numpy(r.view(np.int16) if r.dtype == np.uint16 else r).cuda()
-    logits = torch.empty((B, w.shape.n_classes), dtype=torch.float32, device="cuda")
+    T = w.shape.n_tasks
+    logits = torch.empty((B, T, w.shape.n_classes), dtype=torch.float32, device="cuda")
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     stream = torch.cuda.current_stream()
 
@@ -403,7 +408,7 @@ def run_ours(args, spec, w, rank, world):
     h_lens = torch.from_numpy(np.ascontiguousarray(lens[w.seq_ids], dtype=np.int32)).pin_memory()
     h_rows = rows.cpu().pin_memory() if rows is not None else None
     h_hidden = hidden.cpu().pin_memory() if hidden is not None else None
-    h_logits = torch.empty((B, w.shape.n_classes), dtype=torch.float32).pin_memory()
+    h_logits = torch.empty((B, T, w.shape.n_classes), dtype=torch.float32).pin_memory()
     e2e_s = []
     for i in range(args.warmup + args.steps):
         flush.zero_()
@@ -627,7 +632,7 @@ def main():
             dist.init_process_group("nccl")
     from paper_2608_28099_gb300 import workloads as wl
     spec = shard_spec(wl.named(args.workload, rows_per_seq=(args.rows == "per-seq"),
-                               fused=(args.rows == "hidden")), rank)
+                               fused=(args.rows == "hidden"), n_tasks=max(1, args.tasks)), rank)
     w = wl.generate(spec)
     if args.impl == "reference":
         run_reference(args, spec, w, rank, world)

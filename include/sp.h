@@ -92,6 +92,14 @@ typedef struct sp_config {
     int kv_dtype;     /* SP_F32 or SP_BF16: cached keys/values                       */
     int max_batch;    /* largest batch passed to sp_classify (sizes the scratch)     */
     int max_seq_len;  /* largest cached length L_b (sizes the split plan)            */
+    int n_tasks;      /* T probes sharing one pass over the cache (Sec. 3.3: several
+                         classifiers with their own soft prompt and head on the same
+                         draft-head KV cache); 0 or 1 = one task.  Task t's k rows sit
+                         at positions L_b..L_b+k-1 and attend to the cache and to the
+                         task's own new rows only; the soft prompt is [T][k][d], the
+                         head [T][C][d] (+ bias [T][C]), per-sequence rows [B][T][k][d],
+                         logits [B][T][C].  G * T * k <= 128 keeps the tensor-core
+                         attention; recursive probing needs T = 1                  */
 } sp_config;
 
 /* Layer and probe parameters: HOST pointers, read once by sp_create and

@@ -46,6 +46,11 @@ Readings where the paper is silent (each is listed in the design notes):
    L + i - 1 whose attention sees the cache and the new keys/values of steps
    1..i (the KV caching of Fig. 2).  The head reads the pooled step outputs
    (reading 2: MEAN by default, LAST = the k-th step's output).
+11. several tasks over one cache (Sec. 3.3: classifiers with different soft
+   prompts and heads share the same draft-head KV cache): task t has its own k
+   soft-prompt rows and head; its rows sit at positions L..L+k-1 and attend to
+   the cache and to the task's own new rows only, so each task's logits are
+   those of a single-task classify with that task's prompt and head.
 """
 from __future__ import annotations
 
@@ -318,6 +323,27 @@ def classify_recursive(layer: Layer, cache, seq_ids, hidden, traces: list | None
             traces.append({"x": np.array(xs), "h2": h2})
         out.append(layer.readout(h2))
     return np.array(out).reshape(len(out), layer.head_w.shape[0])
+
+
+def classify_tasks(layer: Layer, cache, seq_ids, prompts, heads, biases=None, rows=None,
+                   hidden=None) -> np.ndarray:
+    """Logits [B, T, C] of T tasks (reading 11): one single-task classify per task.
+
+    prompts: stored soft prompts [T, k, d] (weight dtype); heads [T, C, d]
+    float; biases [T, C] or None; rows: per-sequence rows [B, T, k, d] or None;
+    hidden: base hidden states [B, d] fused with each task's prompt (reading 9)."""
+    T = len(prompts)
+    out = []
+    for t in range(T):
+        task = Layer.__new__(Layer)
+        task.__dict__.update(layer.__dict__)
+        task.soft_prompt = to_f64(prompts[t], layer.shape.w_dtype)
+        task.head_w = np.asarray(heads[t], dtype=np.float64)
+        task.head_b = (np.zeros(task.head_w.shape[0]) if biases is None
+                       else np.asarray(biases[t], dtype=np.float64))
+        out.append(classify(task, cache, seq_ids, None if rows is None else rows[:, t],
+                            hidden=hidden))
+    return np.stack(out, axis=1)
 
 
 def attention_step(shape, cache, seq_ids, q, k_new, v_new) -> np.ndarray:

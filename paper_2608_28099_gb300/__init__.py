@@ -35,7 +35,7 @@ class sp_config(C.Structure):
                 ("head_dim", C.c_int), ("d_ff", C.c_int), ("k_rows", C.c_int),
                 ("n_classes", C.c_int), ("rope_theta", C.c_float), ("rms_eps", C.c_float),
                 ("pool", C.c_int), ("w_dtype", C.c_int), ("kv_dtype", C.c_int),
-                ("max_batch", C.c_int), ("max_seq_len", C.c_int)]
+                ("max_batch", C.c_int), ("max_seq_len", C.c_int), ("n_tasks", C.c_int)]
 
 
 class sp_weights(C.Structure):
@@ -232,7 +232,8 @@ def sp_attend(stream, dims, batch, seq_ids, seq_lens, kv, q, k_new, v_new, out, 
 def make_config(shape, max_batch: int, max_seq_len: int) -> sp_config:
     return sp_config(shape.d_model, shape.n_q_heads, shape.n_kv_heads, shape.head_dim, shape.d_ff,
                      shape.k_rows, shape.n_classes, float(shape.rope_theta), float(shape.rms_eps),
-                     shape.pool, shape.w_dtype, shape.kv_dtype, int(max_batch), int(max_seq_len))
+                     shape.pool, shape.w_dtype, shape.kv_dtype, int(max_batch), int(max_seq_len),
+                     int(getattr(shape, "n_tasks", 1)))
 
 
 class Model:

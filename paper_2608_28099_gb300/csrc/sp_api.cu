@@ -89,6 +89,8 @@ struct sp_handle {
     GemmPlanner gemm;
     // options
     int opt_split = 0, opt_gemm = 0, opt_attn = 0, opt_profile = 0, opt_recursive = 0;
+    int T = 1;        // tasks sharing the pass; cfg.k_rows holds T * k_task rows per sequence
+    int k_task = 0;   // soft-prompt rows per task
     float *h2_all = nullptr;      // recursive probing: step outputs [k][max_batch][d] fp32
     int last_launches = 0;
     cudaEvent_t ev[SP_N_STAGES][2] = {};
@@ -126,6 +128,7 @@ sp_status check_config(const sp_config *c) {
         return fail(SP_ERR_UNSUPPORTED, "head_dim %d unsupported (32, 64, 128)", c->head_dim);
     if (c->d_ff <= 0 || c->d_ff % 8) return fail(SP_ERR_INVALID_ARG, "d_ff must be a positive multiple of 8");
     if (c->k_rows < 1 || c->k_rows > 32) return fail(SP_ERR_INVALID_ARG, "k_rows must be in 1..32");
+    if (c->n_tasks < 0 || c->n_tasks > 64) return fail(SP_ERR_INVALID_ARG, "n_tasks must be in 0..64");
     if (c->n_classes < 1) return fail(SP_ERR_INVALID_ARG, "n_classes must be >= 1");
     if (c->pool != SP_POOL_MEAN && c->pool != SP_POOL_LAST) return fail(SP_ERR_INVALID_ARG, "bad pool");
     if (c->w_dtype != SP_F32 && c->w_dtype != SP_BF16) return fail(SP_ERR_INVALID_ARG, "bad w_dtype");
@@ -133,7 +136,7 @@ sp_status check_config(const sp_config *c) {
     if (c->max_batch < 1) return fail(SP_ERR_INVALID_ARG, "max_batch must be >= 1");
     if (c->max_seq_len < 0) return fail(SP_ERR_INVALID_ARG, "max_seq_len must be >= 0");
     if (!(c->rope_theta > 0.f) || !(c->rms_eps >= 0.f)) return fail(SP_ERR_INVALID_ARG, "bad theta/eps");
-    const int R = (c->n_q_heads / c->n_kv_heads) * c->k_rows;
+    const int R = (c->n_q_heads / c->n_kv_heads) * c->k_rows * (c->n_tasks > 1 ? c->n_tasks : 1);
     if (R * c->head_dim > 128 * 128)
         return fail(SP_ERR_UNSUPPORTED, "query group x k_rows x head_dim too large (%d rows)", R);
     return SP_OK;
@@ -262,6 +265,11 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
 
     sp_handle *h = new sp_handle();
     h->cfg = *cfg;
+    // several tasks: their rows are stacked per sequence ([T][k] rows), so the
+    // layer runs on T k rows; k_task keeps the per-task row count
+    h->T = cfg->n_tasks > 1 ? cfg->n_tasks : 1;
+    h->k_task = cfg->k_rows;
+    h->cfg.k_rows = cfg->k_rows * h->T;
     const sp_config &c = h->cfg;
     cudaGetDevice(&h->device);
     h->n_sm = sm_count();
@@ -301,10 +309,10 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     if ((st = upload(h, (void **)&h->g_in, w->g_in, d * sizeof(float))) != SP_OK) return cleanup(st);
     if ((st = upload(h, (void **)&h->g_post, w->g_post, d * sizeof(float))) != SP_OK) return cleanup(st);
     if ((st = upload(h, &h->soft_prompt, w->soft_prompt, (size_t)k * d * es)) != SP_OK) return cleanup(st);
-    if ((st = upload(h, (void **)&h->head_w, w->head_w, (size_t)C * d * sizeof(float))) != SP_OK)
+    if ((st = upload(h, (void **)&h->head_w, w->head_w, (size_t)h->T * C * d * sizeof(float))) != SP_OK)
         return cleanup(st);
     if (w->head_b &&
-        (st = upload(h, (void **)&h->head_b, w->head_b, C * sizeof(float))) != SP_OK)
+        (st = upload(h, (void **)&h->head_b, w->head_b, (size_t)h->T * C * sizeof(float))) != SP_OK)
         return cleanup(st);
     // input fusion: W_fc [d][2d] split into its hidden-state half (a projection
     // of every call) and its embedding half (applied once to the soft prompt below)
@@ -368,9 +376,9 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
                             (size_t)c.max_batch * 4,    // stage ids
                             (size_t)c.max_batch * 4,    // stage lens
                             M * d * es,                 // stage rows
-                            (size_t)c.max_batch * C * 4,  // stage logits
+                            (size_t)c.max_batch * h->T * C * 4,  // stage logits
                             (size_t)k * h->nqkv * 4,    // qkv_shared
-                            readout_scratch_bytes(c.max_batch, d, C),   // readout partials
+                            readout_scratch_bytes(c.max_batch * h->T, d, C),  // readout partials
                             h->fused ? (size_t)c.max_batch * d * 4 : 0,  // xh
                             h->fused ? M * d * 4 : 0,                    // xrows
                             h->fused ? (size_t)k * d * 4 : 0,            // fc_prompt
@@ -522,6 +530,7 @@ sp_status sp_stage_times(sp_handle *h, float *ms, int n) {
 static sp_status recursive_impl(sp_handle *h, cudaStream_t st, int batch, const int *d_seq_ids,
                                 const int *d_seq_lens, int lens_by_batch, const sp_kv_cache *kv,
                                 const void *d_hidden, float *d_logits) {
+    if (h->T > 1) return fail(SP_ERR_UNSUPPORTED, "recursive probing runs one task per handle");
     const sp_config &c = h->cfg;
     const int d = c.d_model, hq = c.n_q_heads, hkv = c.n_kv_heads, dh = c.head_dim, f = c.d_ff;
     const int k = c.k_rows, C = c.n_classes, G = hq / hkv;
@@ -683,6 +692,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     }
     QkvRopeArgs r;
     memset(&r, 0, sizeof r);  // r0 = 0, kn_stride = 0 (= k): the parallel form
+    r.k_task = h->k_task;     // positions L_b .. L_b + k_task - 1 in every task
     r.y = yqkv;
     r.shared = (d_rows || d_hidden) ? 0 : 1;
     r.B = batch; r.k = k; r.Hq = hq; r.Hkv = hkv; r.dh = dh;
@@ -705,6 +715,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     AttnArgs a;
     memset(&a, 0, sizeof a);
     a.B = batch; a.Hq = hq; a.Hkv = hkv; a.dh = dh; a.k = k; a.G = G; a.R = G * k;
+    a.k_task = h->k_task;  // each task's rows see only that task's new rows
     a.kv_bf16 = c.kv_dtype == SP_BF16;
     a.split_tokens = split_tokens;
     a.n_splits = n_splits;
@@ -751,8 +762,10 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     mark(SP_STAGE_DOWN, 1);
     if (s != SP_OK) return fail(s, "down projection launch failed");
     mark(SP_STAGE_READOUT, 0);
+    // one pooled readout per (sequence, task): rows [B][T][k_task][d]
     SP_CUDA(launch_readout(PartIn{h->y, ns, (size_t)M * d}, h->h1, h->head_w, h->head_b, c.pool,
-                           batch, k, d, C, h->readout_part, d_logits, st));
+                           batch * h->T, h->k_task, d, C, h->readout_part, d_logits, st,
+                           (size_t)h->k_task * d, (size_t)d, h->T));
     mark(SP_STAGE_READOUT, 1);
     launches += 2;
     h->last_launches = launches;
@@ -784,7 +797,7 @@ sp_status sp_classify_host(sp_handle *h, sp_stream stream, int batch, const int 
     sp_status s = classify_impl(h, st, batch, h_seq_ids ? h->stage_ids : nullptr, h->stage_lens, 1,
                                 kv, h_rows ? h->stage_rows : nullptr, h->stage_logits);
     if (s != SP_OK) return s;
-    SP_CUDA(cudaMemcpyAsync(h_logits, h->stage_logits, (size_t)batch * c.n_classes * sizeof(float),
+    SP_CUDA(cudaMemcpyAsync(h_logits, h->stage_logits, (size_t)batch * h->T * c.n_classes * sizeof(float),
                             cudaMemcpyDeviceToHost, st));
     int bits = 0;
     return sp_check_status(h, stream, &bits);
@@ -817,7 +830,7 @@ sp_status sp_classify_hidden_host(sp_handle *h, sp_stream stream, int batch, con
     sp_status s = classify_impl(h, st, batch, h_seq_ids ? h->stage_ids : nullptr, h->stage_lens, 1,
                                 kv, nullptr, h->stage_logits, h->stage_hidden);
     if (s != SP_OK) return s;
-    SP_CUDA(cudaMemcpyAsync(h_logits, h->stage_logits, (size_t)batch * c.n_classes * sizeof(float),
+    SP_CUDA(cudaMemcpyAsync(h_logits, h->stage_logits, (size_t)batch * h->T * c.n_classes * sizeof(float),
                             cudaMemcpyDeviceToHost, st));
     int bits = 0;
     return sp_check_status(h, stream, &bits);

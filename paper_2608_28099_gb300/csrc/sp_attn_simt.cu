@@ -124,7 +124,8 @@ __global__ void __launch_bounds__(kThreads) attn_split_simt(AttnArgs a) {
             const int t = t0 + tt;
             const int r = rr % k;
             float sc = -INFINITY;
-            if (t < t_end && t <= L + a.r0 + r) {
+            const int lo = a.k_task ? (r / a.k_task) * a.k_task : 0;  // the task's first new row
+            if (t < t_end && t <= L + a.r0 + r && (t < L || t >= L + lo)) {
                 const float *qr = Qs + rr * DH;
                 const float *kr = Ks + tt * (DH + 1);
                 float acc = 0.f;

@@ -580,14 +580,17 @@ __global__ void __launch_bounds__(THREADS, 1)
         int k0 = 0, k1 = 0;  // tiles done so far by pipeline 0 / 1 (barrier phases)
         for (int x = x0; x < x1;) {
             const int xs = x;  // segment start (its other fields are recomputed after the tiles)
-            int n_tiles, lim_rel;
+            int n_tiles, lim_rel, lo_rel, new_rel;
             {
                 const Seg sg = seg_at(prefix, B, x, x1);
                 n_tiles = sg.n;
                 const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, sg.b, a.kv.n_seqs,
                                               a.max_seq_len, nullptr);
-                // this row sees tokens t < L + r0 + r + 1; relative to the segment start:
+                // this row sees tokens t < L + r0 + r + 1 except the new rows of
+                // other tasks before its own, [L, L + lo); relative to the segment start:
                 lim_rel = sq.len + a.r0 + r_soft + 1 - sg.t_a * TT;
+                lo_rel = sq.len + (a.k_task ? (r_soft / a.k_task) * a.k_task : 0) - sg.t_a * TT;
+                new_rel = sq.len - sg.t_a * TT;
             }
             x += n_tiles;
             // this segment's queries are written, and the previous epilogue is complete
@@ -614,10 +617,12 @@ __global__ void __launch_bounds__(THREADS, 1)
                     for (int jj = 0; jj < 32; ++jj) sv[32 + jj] = t32[jj];
                 }
                 const int t0 = i * TT;  // relative to the segment start
-                if (t0 + TT > lim_rel) {
+                if (t0 + TT > new_rel) {  // the tile holds new rows: causal and task masks
 #pragma unroll
-                    for (int jj = 0; jj < TT; ++jj)
-                        if (t0 + jj >= lim_rel) sv[jj] = -INFINITY;
+                    for (int jj = 0; jj < TT; ++jj) {
+                        const int t = t0 + jj;
+                        if (t >= lim_rel || (t >= new_rel && t < lo_rel)) sv[jj] = -INFINITY;
+                    }
                 }
                 // tile max as an 8-way tree
                 float mx[8];

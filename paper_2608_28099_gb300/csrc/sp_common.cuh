@@ -194,6 +194,8 @@ struct AttnArgs {
     int r0;                       // the pass's query row r is new row r0 + r (position
                                   // L + r0 + r) and sees new keys 0..r0 + r
     int kn_stride;                // rows per sequence of k_new / v_new (0 = k)
+    int k_task;                   // rows per task (0 = k): query row r belongs to task
+                                  // r / k_task and sees only that task's new rows
     int kv_bf16;                  // cache element type: 1 bf16, 0 fp32
     int split_tokens;             // tokens per work unit
     int n_splits;                 // work units per (sequence, kv head) in the grid
@@ -257,6 +259,7 @@ struct QkvRopeArgs {
     int B, k, Hq, Hkv, dh;
     int r0;                  // row m = b k + r is new row r0 + r, at position L_b + r0 + r
     int kn_stride;           // rows per sequence of k_new / v_new (0 = k)
+    int k_task;              // rows per task (0 = k): the position is L_b + r0 + r % k_task
     const int *seq_ids, *seq_lens;
     int lens_by_batch;
     int n_seqs, max_seq_len;
@@ -282,10 +285,11 @@ cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_
 // products in `scratch` (readout_scratch_bytes); two launches.
 size_t readout_scratch_bytes(int B, int d, int C);
 // Row r of sequence b of (h1 + y) sits at b sb + r sr (0 = the dense [B][k][d]
-// strides k d and d).
+// strides k d and d).  With n_tasks > 1, "sequence" b is (sequence b / n_tasks,
+// task b % n_tasks) and reads head [b % n_tasks] of head_w [n_tasks][C][d].
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
                            int pool, int B, int k, int d, int C, float *scratch, float *logits,
-                           cudaStream_t st, size_t sb = 0, size_t sr = 0);
+                           cudaStream_t st, size_t sb = 0, size_t sr = 0, int n_tasks = 1);
 
 // ---------------------------------------------------------------------------
 // projections

@@ -83,7 +83,7 @@ __global__ void qkv_rope_kernel(QkvRopeArgs a) {
     const int kns = a.kn_stride ? a.kn_stride : a.k;
     const size_t mn = (size_t)b * kns + a.r0 + r;  // row of k_new / v_new
     if (idx < nrot) {
-        const int pos = s.len + a.r0 + r;
+        const int pos = s.len + a.r0 + (a.k_task ? r % a.k_task : r);
         const int h = idx / half, i = idx - h * half;
         const float x0 = part_get(a.y, row + h * dh + i);
         const float x1 = part_get(a.y, row + h * dh + i + half);
@@ -164,7 +164,8 @@ constexpr int kReadoutCols = 64;
 
 __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const float *__restrict__ h1,
                                        const float *__restrict__ head_w, int pool, int k, int d,
-                                       int C, float *__restrict__ part, size_t sb, size_t sr) {
+                                       int C, float *__restrict__ part, size_t sb, size_t sr,
+                                       int n_tasks) {
     pdl_trigger();
     pdl_wait();
     __shared__ float acc_s[4][kReadoutCols];
@@ -174,6 +175,7 @@ __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const fl
     const int c = threadIdx.x & (kReadoutCols - 1), rg = threadIdx.x / kReadoutCols;
     const int col = chunk * kReadoutCols + c;
     const size_t base = (size_t)b * sb;
+    head_w += (size_t)(b % n_tasks) * C * d;  // this task's head
     float acc = 0.f;
     if (col < d) {
         if (pool == SP_POOL_LAST) {
@@ -212,10 +214,12 @@ __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const fl
 }
 
 __global__ void readout_finish_kernel(const float *__restrict__ part, int n_chunks, int C,
-                                      const float *__restrict__ head_b, float *__restrict__ logits) {
+                                      const float *__restrict__ head_b, float *__restrict__ logits,
+                                      int n_tasks) {
     pdl_trigger();
     pdl_wait();
     const int b = blockIdx.x;
+    if (head_b) head_b += (size_t)(b % n_tasks) * C;
     for (int c = threadIdx.x; c < C; c += blockDim.x) {
         float acc = head_b ? head_b[c] : 0.f;
         for (int j = 0; j < n_chunks; ++j) acc += part[((size_t)b * n_chunks + j) * C + c];
@@ -332,15 +336,16 @@ size_t readout_scratch_bytes(int B, int d, int C) {
 
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
                            int pool, int B, int k, int d, int C, float *scratch, float *logits,
-                           cudaStream_t st, size_t sb, size_t sr) {
+                           cudaStream_t st, size_t sb, size_t sr, int n_tasks) {
     const int chunks = ceil_div(d, kReadoutCols);
     if (!sb) sb = (size_t)k * d;
     if (!sr) sr = d;
+    if (n_tasks < 1) n_tasks = 1;
     cudaError_t e = launch_k(readout_partial_kernel, dim3(chunks, B), dim3(256), 0, st, y, h1,
-                             head_w, pool, k, d, C, scratch, sb, sr);
+                             head_w, pool, k, d, C, scratch, sb, sr, n_tasks);
     if (e != cudaSuccess) return e;
     return launch_k(readout_finish_kernel, dim3(B), dim3(64), 0, st, (const float *)scratch, chunks,
-                    C, head_b, logits);
+                    C, head_b, logits, n_tasks);
 }
 
 cudaError_t launch_to_act(const float *x, size_t n, ActOut out, cudaStream_t st) {

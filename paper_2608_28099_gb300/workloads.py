@@ -25,6 +25,8 @@ Sec. 6):
   [token][kv_head][head_dim].
 * input fusion (optional): a fifth stream draws W_fc [d][2d] N(0, 0.02), the
   two fusion norm gains 1 + N(0, 0.02) and base hidden states [B][d] N(0, 1).
+* several tasks (optional): a sixth stream draws the soft prompts, heads (and
+  rows) of tasks 1..T-1; task 0 keeps the single-task draws.
 """
 from __future__ import annotations
 
@@ -73,6 +75,7 @@ class Shape:
     kv_dtype: int = BF16
     pool: int = POOL_MEAN
     page_size: int = 16
+    n_tasks: int = 1         # probes (soft prompt + head) sharing one pass over the cache
 
     @property
     def group(self) -> int:
@@ -257,6 +260,45 @@ def draw_fusion(shape: Shape, seed: int, batch: int):
     return w_fc, g_h, g_e, hidden
 
 
+def with_tasks(w: "Workload", T: int) -> "Workload":
+    """The workload with T tasks: task 0 keeps the drawn soft prompt, head (and
+    rows); tasks 1..T-1 draw theirs from a sixth stream of the seed.  Stacked as
+    soft_prompt [T k][d], head_w [T C][d], head_b [T C], rows [B][T k][d]."""
+    sh = w.spec.shape
+    if T <= 1:
+        return w
+    rng = np.random.default_rng(np.random.SeedSequence(w.spec.seed).spawn(6)[5])
+    k, d, C, wd = sh.k_rows, sh.d_model, sh.n_classes, sh.w_dtype
+    prompts = [w.weights.soft_prompt] + [_normal(rng, (k, d), 0.02, wd) for _ in range(T - 1)]
+    heads = [w.weights.head_w] + [(0.02 * rng.standard_normal((C, d))).astype(np.float32)
+                                  for _ in range(T - 1)]
+    biases = None
+    if w.weights.head_b is not None:
+        biases = [w.weights.head_b] + [(0.02 * rng.standard_normal(C)).astype(np.float32)
+                                       for _ in range(T - 1)]
+    weights = dataclasses.replace(w.weights, soft_prompt=np.concatenate(prompts, axis=0),
+                                  head_w=np.concatenate(heads, axis=0),
+                                  head_b=None if biases is None else np.concatenate(biases))
+    rows = w.rows
+    if rows is not None:
+        B = rows.shape[0]
+        extra = [_normal(rng, (B, k, d), 0.02, wd) for _ in range(T - 1)]
+        rows = np.concatenate([rows] + extra, axis=1)
+    spec = dataclasses.replace(w.spec, shape=dataclasses.replace(sh, n_tasks=T))
+    return dataclasses.replace(w, spec=spec, weights=weights, rows=rows)
+
+
+def task_views(w: "Workload"):
+    """(prompts [T][k][d], heads [T][C][d], biases [T][C] or None, rows
+    [B][T][k][d] or None) of a stacked T-task workload."""
+    sh = w.spec.shape
+    T, k, d, C = sh.n_tasks, sh.k_rows, sh.d_model, sh.n_classes
+    wt = w.weights
+    rows = None if w.rows is None else w.rows.reshape(w.rows.shape[0], T, k, d)
+    return (wt.soft_prompt.reshape(T, k, d), wt.head_w.reshape(T, C, d),
+            None if wt.head_b is None else wt.head_b.reshape(T, C), rows)
+
+
 def with_fusion(w: "Workload") -> "Workload":
     """The same workload with fusion weights and hidden states attached."""
     w_fc, g_h, g_e, hidden = draw_fusion(w.spec.shape, w.spec.seed, len(w.seq_ids))
@@ -322,6 +364,9 @@ def generate(spec: WorkloadSpec) -> Workload:
                        sh.w_dtype)
     seq_ids = np.arange(spec.batch, dtype=np.int32)
     w = Workload(spec, weights, cache, seq_ids, rows)
+    if spec.shape.n_tasks > 1:
+        w = with_tasks(dataclasses.replace(w, spec=dataclasses.replace(
+            spec, shape=dataclasses.replace(spec.shape, n_tasks=1))), spec.shape.n_tasks)
     return with_fusion(w) if spec.fused else w
 
 

@@ -361,7 +361,44 @@ def check_recursive_embedding_only_is_the_row_path():
     np.testing.assert_allclose(a, b, rtol=1e-5, atol=1e-6)
 
 
-ALL_CHECKS = [check_recursive_k1_equals_parallel_fused,
+def _tasks(seed, T, sh):
+    rng = np.random.default_rng(seed)
+    prompts = f32(rng.standard_normal((T, sh.k_rows, sh.d_model)) * 0.4)
+    heads = f32(rng.standard_normal((T, sh.n_classes, sh.d_model)))
+    biases = f32(rng.standard_normal((T, sh.n_classes)))
+    return prompts, heads, biases
+
+
+def check_one_task_is_the_single_task_path():
+    sh, w = random_layer(50)
+    layer = so.Layer(sh, w)
+    cw = wl.custom(sh, [0, 9, 20], wl.LAYOUT_PAGED, 51)
+    got = so.classify_tasks(layer, cw.cache, cw.seq_ids, f32(w.soft_prompt[None]), f32(w.head_w[None]),
+                            f32(w.head_b[None]))
+    np.testing.assert_array_equal(got[:, 0], so.classify(layer, cw.cache, cw.seq_ids))
+
+
+def check_tasks_are_isolated_and_permutable():
+    sh, w = random_layer(52)
+    layer = so.Layer(sh, w)
+    cw = wl.custom(sh, [4, 13], wl.LAYOUT_CONTIGUOUS, 53)
+    prompts, heads, biases = _tasks(54, 3, sh)
+    a = so.classify_tasks(layer, cw.cache, cw.seq_ids, prompts, heads, biases)
+    # another task's prompt and head change nothing for task 0
+    p2, h2, b2 = prompts.copy(), heads.copy(), biases.copy()
+    p2[1] = p2[1][::-1] * 3
+    h2[2] = -h2[2]
+    b = so.classify_tasks(layer, cw.cache, cw.seq_ids, p2, h2, b2)
+    np.testing.assert_array_equal(a[:, 0], b[:, 0])
+    assert np.max(np.abs(a[:, 1] - b[:, 1])) > 1e-6
+    # permuting the tasks permutes the logits
+    perm = [2, 0, 1]
+    c = so.classify_tasks(layer, cw.cache, cw.seq_ids, prompts[perm], heads[perm], biases[perm])
+    np.testing.assert_array_equal(c, a[:, perm])
+
+
+ALL_CHECKS = [check_one_task_is_the_single_task_path, check_tasks_are_isolated_and_permutable,
+              check_recursive_k1_equals_parallel_fused,
               check_recursive_equals_stepwise_reconstruction,
               check_recursive_embedding_only_is_the_row_path,
               check_fusion_hand_example, check_fusion_with_embedding_only_is_the_row_path,
