@@ -51,6 +51,11 @@ Readings where the paper is silent (each is listed in the design notes):
    soft-prompt rows and head; its rows sit at positions L..L+k-1 and attend to
    the cache and to the task's own new rows only, so each task's logits are
    those of a single-task classify with that task's prompt and head.
+12. LM-head readout (Sec. 5 ablation "Classification head": the frozen lm_head's
+   yes/no token logits): the head rows are the label tokens' rows of the
+   frozen LM head and the pooled state first passes the head's final RMSNorm
+   (gain g_final, the layer's eps): logits = W_head RMSNorm(pool(h2); g_final)
+   (+ bias).  The yes/no difference is logits[yes] - logits[no].
 """
 from __future__ import annotations
 
@@ -163,6 +168,8 @@ class Layer:
         self.head_w = np.asarray(weights.head_w, dtype=np.float64)
         self.head_b = (np.zeros(self.head_w.shape[0]) if weights.head_b is None
                        else np.asarray(weights.head_b, dtype=np.float64))
+        gf = getattr(weights, "g_final", None)
+        self.g_final = None if gf is None else np.asarray(gf, dtype=np.float64)
         fc = getattr(weights, "w_fc", None)
         self.w_fc = None if fc is None else to_f64(fc, wd)
         self.g_h = None if fc is None else np.asarray(weights.g_h, dtype=np.float64)
@@ -204,8 +211,11 @@ class Layer:
         return h1 + a @ self.w_down.T
 
     def readout(self, h2: np.ndarray) -> np.ndarray:
-        """Linear head on the pooled soft-prompt outputs (reading 2, 7)."""
+        """Linear head on the pooled soft-prompt outputs (reading 2, 7), after
+        the final norm when the head is an LM head's rows (reading 12)."""
         pooled = h2.mean(axis=0) if self.shape.pool == POOL_MEAN else h2[-1]
+        if self.g_final is not None:
+            pooled = rms_norm(pooled, self.g_final, self.shape.rms_eps)
         return self.head_w @ pooled + self.head_b
 
     # -- the classify path: k rows against a resident cache ------------------

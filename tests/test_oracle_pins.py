@@ -34,6 +34,7 @@ class W:
     soft_prompt: np.ndarray
     head_w: np.ndarray
     head_b: np.ndarray = None
+    g_final: np.ndarray = None  # final norm before an LM-head readout (optional)
     w_fc: np.ndarray = None    # input fusion (optional)
     g_h: np.ndarray = None
     g_e: np.ndarray = None
@@ -397,7 +398,30 @@ def check_tasks_are_isolated_and_permutable():
     np.testing.assert_array_equal(c, a[:, perm])
 
 
-ALL_CHECKS = [check_one_task_is_the_single_task_path, check_tasks_are_isolated_and_permutable,
+def check_lm_head_readout_hand_example():
+    g = read_golden("lm_head_readout_d2.txt")
+    sh = wl.Shape(2, 1, 1, 2, 1, 2, 2, rms_eps=0.0, w_dtype=wl.F32, kv_dtype=wl.F32)
+    _, w = random_layer(60, d=2, hq=1, hkv=1, dh=2, f=1, k=2, C=2)
+    w = dataclasses.replace(w, head_w=np.eye(2), head_b=None, g_final=f32(g["g_final"]))
+    layer = so.Layer(sh, w)
+    z = layer.readout(np.reshape(g["h2"], (2, 2)))
+    np.testing.assert_allclose(z, g["logits"], atol=1e-9)
+    np.testing.assert_allclose(z[1] - z[0], g["yes_minus_no"][0], atol=1e-9)
+
+
+def check_lm_head_readout_is_scale_invariant():
+    # the final norm makes the logits blind to a positive scale of the outputs
+    sh, w = random_layer(61, eps=0.0)
+    w = dataclasses.replace(w, g_final=f32(1 + 0.1 * np.random.default_rng(62).standard_normal(16)))
+    layer = so.Layer(sh, w)
+    h2 = np.random.default_rng(63).standard_normal((sh.k_rows, sh.d_model))
+    np.testing.assert_allclose(layer.readout(h2 * 7.5), layer.readout(h2), rtol=1e-12, atol=1e-12)
+    plain = so.Layer(sh, dataclasses.replace(w, g_final=None))
+    assert np.max(np.abs(plain.readout(h2 * 7.5) - plain.readout(h2))) > 1e-3
+
+
+ALL_CHECKS = [check_lm_head_readout_hand_example, check_lm_head_readout_is_scale_invariant,
+              check_one_task_is_the_single_task_path, check_tasks_are_isolated_and_permutable,
               check_recursive_k1_equals_parallel_fused,
               check_recursive_equals_stepwise_reconstruction,
               check_recursive_embedding_only_is_the_row_path,
@@ -557,7 +581,26 @@ def _recursive_variant(feed_input=False, fixed_position=False, no_append=False, 
     return f
 
 
+def _readout_norm_before_pool(orig):
+    def f(self, h2):
+        if self.g_final is None:
+            return orig(self, h2)
+        n = so.rms_norm(h2, self.g_final, self.shape.rms_eps)
+        pooled = n.mean(axis=0) if self.shape.pool == so.POOL_MEAN else n[-1]
+        return self.head_w @ pooled + self.head_b
+    return f
+
+
+def _readout_final_norm_ignored(orig):
+    def f(self, h2):
+        pooled = h2.mean(axis=0) if self.shape.pool == so.POOL_MEAN else h2[-1]
+        return self.head_w @ pooled + self.head_b
+    return f
+
+
 MUTANTS = {
+    "lm_readout_norm_before_pool": (so.Layer, "readout", _readout_norm_before_pool),
+    "lm_readout_final_norm_ignored": (so.Layer, "readout", _readout_final_norm_ignored),
     "recursion_feeds_layer_input": (so, "classify_recursive",
                                     lambda orig: _recursive_variant(feed_input=True)),
     "recursion_fixed_position": (so, "classify_recursive",
