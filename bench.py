@@ -63,6 +63,8 @@ def parse_args():
                         "shared: the soft prompt, whose Q/K/V projection is precomputed; "
                         "hidden: base hidden states through the MTP input fusion "
                         "(sp_classify_hidden)")
+    p.add_argument("--head", default="linear", choices=["linear", "lm"],
+                   help="linear: trained linear head; lm: frozen LM-head rows after the final norm")
     p.add_argument("--tasks", type=int, default=1,
                    help="probes (soft prompt + head) sharing each pass over the cache")
     p.add_argument("--recursive", action="store_true",
@@ -271,7 +273,7 @@ def workload_config(spec, w, args):
             "kv_layout": "paged16" if w.cache.layout == 1 else "contiguous",
             "rows": args.rows, "seed": spec.seed,
             "form": "recursive SP-k" if recursive_mode(args) else "parallel k rows",
-            "n_tasks": sh.n_tasks,
+            "n_tasks": sh.n_tasks, "head": args.head,
             "l2": "flushed between steps (256 MiB write)",
             "timing": ("CUDA events per step around a CUDA-graph replay of one "
                        + ("sp_classify_hidden" if w.hidden is not None else "sp_classify"))}
@@ -634,6 +636,8 @@ def main():
     spec = shard_spec(wl.named(args.workload, rows_per_seq=(args.rows == "per-seq"),
                                fused=(args.rows == "hidden"), n_tasks=max(1, args.tasks)), rank)
     w = wl.generate(spec)
+    if args.head == "lm":
+        w = wl.with_lm_head(w)
     if args.impl == "reference":
         run_reference(args, spec, w, rank, world)
     else:

@@ -114,7 +114,12 @@ typedef struct sp_config {
  * projected by W_fc): w_fc [d][2d] (w_dtype; columns [0, d) act on the
  * normalised hidden state, [d, 2d) on the normalised embedding), g_h [d] and
  * g_e [d] (float) the two norm gains.  All three NULL: no fusion (then
- * sp_classify_hidden returns SP_ERR_INVALID_ARG). */
+ * sp_classify_hidden returns SP_ERR_INVALID_ARG).
+ * Optional LM-head readout (Sec. 5 ablation, "Classification head": the frozen
+ * lm_head read at label tokens such as yes/no): g_final [d] (float) is the
+ * head's final RMSNorm gain, applied to the pooled state before head_w, whose
+ * rows are then the label tokens' lm_head rows (logits[yes] - logits[no] is the
+ * binary logit).  NULL = the plain linear head. */
 typedef struct sp_weights {
     const void *w_q, *w_k, *w_v, *w_o, *w_gate, *w_up, *w_down;
     const float *g_in, *g_post;
@@ -122,6 +127,7 @@ typedef struct sp_weights {
     const float *head_w, *head_b;
     const void *w_fc;
     const float *g_h, *g_e;
+    const float *g_final;
 } sp_weights;
 
 /* A resident key/value cache (Sec. 3.3): DEVICE pointers, borrowed for the

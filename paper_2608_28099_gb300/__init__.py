@@ -41,7 +41,7 @@ class sp_config(C.Structure):
 class sp_weights(C.Structure):
     _fields_ = [(n, C.c_void_p) for n in ("w_q", "w_k", "w_v", "w_o", "w_gate", "w_up", "w_down",
                                            "g_in", "g_post", "soft_prompt", "head_w", "head_b",
-                                           "w_fc", "g_h", "g_e")]
+                                           "w_fc", "g_h", "g_e", "g_final")]
 
 
 class sp_kv_cache(C.Structure):
@@ -254,10 +254,12 @@ class Model:
         for name in ("g_h", "g_e"):
             arrs[name] = (None if fc is None
                           else np.ascontiguousarray(getattr(weights, name), dtype=np.float32))
+        gf = getattr(weights, "g_final", None)
+        arrs["g_final"] = None if gf is None else np.ascontiguousarray(gf, dtype=np.float32)
         self._arrs = arrs  # host copies stay alive for the handle's lifetime (read at create)
         w = sp_weights(*[None if arrs[n] is None else arrs[n].ctypes.data for n in (
             "w_q", "w_k", "w_v", "w_o", "w_gate", "w_up", "w_down", "g_in", "g_post",
-            "soft_prompt", "head_w", "head_b", "w_fc", "g_h", "g_e")])
+            "soft_prompt", "head_w", "head_b", "w_fc", "g_h", "g_e", "g_final")])
         self.cfg = make_config(shape, max_batch, max_seq_len)
         self.handle = sp_create(self.cfg, w)
 

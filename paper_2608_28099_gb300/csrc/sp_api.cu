@@ -61,6 +61,7 @@ struct sp_handle {
     // weights
     WeightMat w_qkv, w_o, w_gu, w_down;
     float *g_in = nullptr, *g_post = nullptr, *head_w = nullptr, *head_b = nullptr;
+    float *g_final = nullptr;     // LM-head readout: final RMSNorm gain (NULL: linear head)
     void *soft_prompt = nullptr;
     float *qkv_shared = nullptr;  // [k][nqkv] projections of the shared soft prompt
     float2 *rope_cs = nullptr;    // [max_seq_len + k][dh/2]
@@ -313,6 +314,9 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
         return cleanup(st);
     if (w->head_b &&
         (st = upload(h, (void **)&h->head_b, w->head_b, (size_t)h->T * C * sizeof(float))) != SP_OK)
+        return cleanup(st);
+    if (w->g_final &&
+        (st = upload(h, (void **)&h->g_final, w->g_final, d * sizeof(float))) != SP_OK)
         return cleanup(st);
     // input fusion: W_fc [d][2d] split into its hidden-state half (a projection
     // of every call) and its embedding half (applied once to the soft prompt below)
@@ -609,7 +613,7 @@ static sp_status recursive_impl(sp_handle *h, cudaStream_t st, int batch, const 
         ++launches;
     }
     SP_CUDA(launch_readout(PartIn{nullptr, 0, 0}, h->h2_all, h->head_w, h->head_b, c.pool, B, k, d, C,
-                           h->readout_part, d_logits, st, (size_t)d, Bd));
+                           h->readout_part, d_logits, st, (size_t)d, Bd, 1, h->g_final, c.rms_eps));
     launches += 2;
     h->last_launches = launches;
     return SP_OK;
@@ -765,7 +769,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     // one pooled readout per (sequence, task): rows [B][T][k_task][d]
     SP_CUDA(launch_readout(PartIn{h->y, ns, (size_t)M * d}, h->h1, h->head_w, h->head_b, c.pool,
                            batch * h->T, h->k_task, d, C, h->readout_part, d_logits, st,
-                           (size_t)h->k_task * d, (size_t)d, h->T));
+                           (size_t)h->k_task * d, (size_t)d, h->T, h->g_final, c.rms_eps));
     mark(SP_STAGE_READOUT, 1);
     launches += 2;
     h->last_launches = launches;

@@ -289,7 +289,8 @@ size_t readout_scratch_bytes(int B, int d, int C);
 // task b % n_tasks) and reads head [b % n_tasks] of head_w [n_tasks][C][d].
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
                            int pool, int B, int k, int d, int C, float *scratch, float *logits,
-                           cudaStream_t st, size_t sb = 0, size_t sr = 0, int n_tasks = 1);
+                           cudaStream_t st, size_t sb = 0, size_t sr = 0, int n_tasks = 1,
+                           const float *g_final = nullptr, float eps = 0.f);
 
 // ---------------------------------------------------------------------------
 // projections

@@ -165,7 +165,8 @@ constexpr int kReadoutCols = 64;
 __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const float *__restrict__ h1,
                                        const float *__restrict__ head_w, int pool, int k, int d,
                                        int C, float *__restrict__ part, size_t sb, size_t sr,
-                                       int n_tasks) {
+                                       int n_tasks, const float *__restrict__ g_final,
+                                       float *__restrict__ part_ss) {
     pdl_trigger();
     pdl_wait();
     __shared__ float acc_s[4][kReadoutCols];
@@ -194,9 +195,23 @@ __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const fl
     __syncthreads();
     if (threadIdx.x < kReadoutCols) {
         const float sum = (acc_s[0][c] + acc_s[1][c]) + (acc_s[2][c] + acc_s[3][c]);
-        pooled[c] = pool == SP_POOL_LAST ? sum : sum / (float)k;
+        const float p = pool == SP_POOL_LAST ? sum : sum / (float)k;
+        if (g_final) {
+            // LM-head readout: the chunk's share of the pooled row's square sum,
+            // and the pooled value times the final-norm gain (the 1/rms factor
+            // is applied to the finished dot products)
+            float sq = col < d ? p * p : 0.f;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+            if ((threadIdx.x & 31) == 0) red[3][4 + (threadIdx.x >> 5)] = sq;
+            pooled[c] = col < d ? p * g_final[col] : 0.f;
+        } else {
+            pooled[c] = p;
+        }
     }
     __syncthreads();
+    if (g_final && threadIdx.x == 0)
+        part_ss[(size_t)b * gridDim.x + chunk] = red[3][4] + red[3][5];
     // thread (group cg = tid / 64, column c): class c0 + cg
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     for (int c0 = 0; c0 < C; c0 += 4) {
@@ -215,15 +230,22 @@ __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const fl
 
 __global__ void readout_finish_kernel(const float *__restrict__ part, int n_chunks, int C,
                                       const float *__restrict__ head_b, float *__restrict__ logits,
-                                      int n_tasks) {
+                                      int n_tasks, const float *__restrict__ part_ss, int d,
+                                      float eps) {
     pdl_trigger();
     pdl_wait();
     const int b = blockIdx.x;
     if (head_b) head_b += (size_t)(b % n_tasks) * C;
+    float inv = 1.f;  // 1 / rms of the pooled row (LM-head readout)
+    if (part_ss) {
+        float ss = 0.f;
+        for (int j = 0; j < n_chunks; ++j) ss += part_ss[(size_t)b * n_chunks + j];
+        inv = rsqrtf(ss / (float)d + eps);
+    }
     for (int c = threadIdx.x; c < C; c += blockDim.x) {
-        float acc = head_b ? head_b[c] : 0.f;
+        float acc = 0.f;
         for (int j = 0; j < n_chunks; ++j) acc += part[((size_t)b * n_chunks + j) * C + c];
-        logits[(size_t)b * C + c] = acc;
+        logits[(size_t)b * C + c] = acc * inv + (head_b ? head_b[c] : 0.f);
     }
 }
 
@@ -331,21 +353,24 @@ cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_
 }
 
 size_t readout_scratch_bytes(int B, int d, int C) {
-    return (size_t)B * ceil_div(d, kReadoutCols) * C * sizeof(float);
+    // partial dot products [B][chunks][C], then square sums [B][chunks]
+    return (size_t)B * ceil_div(d, kReadoutCols) * (C + 1) * sizeof(float);
 }
 
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
                            int pool, int B, int k, int d, int C, float *scratch, float *logits,
-                           cudaStream_t st, size_t sb, size_t sr, int n_tasks) {
+                           cudaStream_t st, size_t sb, size_t sr, int n_tasks,
+                           const float *g_final, float eps) {
     const int chunks = ceil_div(d, kReadoutCols);
     if (!sb) sb = (size_t)k * d;
     if (!sr) sr = d;
     if (n_tasks < 1) n_tasks = 1;
+    float *ss = g_final ? scratch + (size_t)B * chunks * C : nullptr;
     cudaError_t e = launch_k(readout_partial_kernel, dim3(chunks, B), dim3(256), 0, st, y, h1,
-                             head_w, pool, k, d, C, scratch, sb, sr, n_tasks);
+                             head_w, pool, k, d, C, scratch, sb, sr, n_tasks, g_final, ss);
     if (e != cudaSuccess) return e;
     return launch_k(readout_finish_kernel, dim3(B), dim3(64), 0, st, (const float *)scratch, chunks,
-                    C, head_b, logits, n_tasks);
+                    C, head_b, logits, n_tasks, (const float *)ss, d, eps);
 }
 
 cudaError_t launch_to_act(const float *x, size_t n, ActOut out, cudaStream_t st) {

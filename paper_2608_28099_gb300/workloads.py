@@ -169,6 +169,8 @@ class Weights:
     w_fc: Optional[np.ndarray] = None
     g_h: Optional[np.ndarray] = None
     g_e: Optional[np.ndarray] = None
+    # LM-head readout: final RMSNorm gain float32 [d] applied before the head
+    g_final: Optional[np.ndarray] = None
 
 
 @dataclasses.dataclass
@@ -297,6 +299,18 @@ def task_views(w: "Workload"):
     rows = None if w.rows is None else w.rows.reshape(w.rows.shape[0], T, k, d)
     return (wt.soft_prompt.reshape(T, k, d), wt.head_w.reshape(T, C, d),
             None if wt.head_b is None else wt.head_b.reshape(T, C), rows)
+
+
+def with_lm_head(w: "Workload") -> "Workload":
+    """The workload read out through a frozen LM head: a final-norm gain
+    1 + N(0, 0.02) and head rows standing in for the label tokens' lm_head rows
+    (N(0, 0.02) per task, no bias), from a seventh stream of the seed."""
+    sh = w.spec.shape
+    rng = np.random.default_rng(np.random.SeedSequence(w.spec.seed).spawn(7)[6])
+    g_final = (1.0 + 0.02 * rng.standard_normal(sh.d_model)).astype(np.float32)
+    head = (0.02 * rng.standard_normal(w.weights.head_w.shape)).astype(np.float32)
+    weights = dataclasses.replace(w.weights, g_final=g_final, head_w=head, head_b=None)
+    return dataclasses.replace(w, weights=weights)
 
 
 def with_fusion(w: "Workload") -> "Workload":
