@@ -285,28 +285,40 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
         return s;
     };
 
-    // weights: [W_q; W_k; W_v] and [W_gate; W_up] concatenated along the output dim
-    void *p_qkv = nullptr, *p_gu = nullptr, *p_o = nullptr, *p_down = nullptr;
+    // weights: [W_q; W_k; W_v] and [W_gate; W_up] concatenated along the output
+    // dim; bf16 matrices the tensor cores take are stored in 16 KB (tile,
+    // k-block) blocks (block_weights_layout), the rest row-major
+    const int wb = c.w_dtype == SP_BF16;
+    auto upload_weight = [&](WeightMat &wm, const char *src, int N, int K) -> sp_status {
+        const size_t bytes = (size_t)N * K * es;
+        const bool blocked = wb && tc_supported(N, K);
+        std::vector<char> blk;
+        if (blocked) {
+            blk.resize(bytes);
+            block_weights_layout(src, blk.data(), N, K, es);
+            src = blk.data();
+        }
+        void *p = nullptr;
+        sp_status s2 = upload(h, &p, src, bytes);
+        if (s2 != SP_OK) return s2;
+        init_weight(wm, p, N, K, wb, blocked);
+        return SP_OK;
+    };
     {
         std::vector<char> buf((size_t)h->nqkv * d * es);
         memcpy(buf.data(), w->w_q, (size_t)hq * dh * d * es);
         memcpy(buf.data() + (size_t)hq * dh * d * es, w->w_k, (size_t)hkv * dh * d * es);
         memcpy(buf.data() + (size_t)(hq + hkv) * dh * d * es, w->w_v, (size_t)hkv * dh * d * es);
-        if ((st = upload(h, &p_qkv, buf.data(), buf.size())) != SP_OK) return cleanup(st);
+        if ((st = upload_weight(h->w_qkv, buf.data(), h->nqkv, d)) != SP_OK) return cleanup(st);
     }
     {
         std::vector<char> buf((size_t)2 * f * d * es);
         memcpy(buf.data(), w->w_gate, (size_t)f * d * es);
         memcpy(buf.data() + (size_t)f * d * es, w->w_up, (size_t)f * d * es);
-        if ((st = upload(h, &p_gu, buf.data(), buf.size())) != SP_OK) return cleanup(st);
+        if ((st = upload_weight(h->w_gu, buf.data(), 2 * f, d)) != SP_OK) return cleanup(st);
     }
-    if ((st = upload(h, &p_o, w->w_o, (size_t)d * hq * dh * es)) != SP_OK) return cleanup(st);
-    if ((st = upload(h, &p_down, w->w_down, (size_t)d * f * es)) != SP_OK) return cleanup(st);
-    const int wb = c.w_dtype == SP_BF16;
-    init_weight(h->w_qkv, p_qkv, h->nqkv, d, wb);
-    init_weight(h->w_o, p_o, d, hq * dh, wb);
-    init_weight(h->w_gu, p_gu, 2 * f, d, wb);
-    init_weight(h->w_down, p_down, d, f, wb);
+    if ((st = upload_weight(h->w_o, (const char *)w->w_o, d, hq * dh)) != SP_OK) return cleanup(st);
+    if ((st = upload_weight(h->w_down, (const char *)w->w_down, d, f)) != SP_OK) return cleanup(st);
     if ((st = upload(h, (void **)&h->g_in, w->g_in, d * sizeof(float))) != SP_OK) return cleanup(st);
     if ((st = upload(h, (void **)&h->g_post, w->g_post, d * sizeof(float))) != SP_OK) return cleanup(st);
     if ((st = upload(h, &h->soft_prompt, w->soft_prompt, (size_t)k * d * es)) != SP_OK) return cleanup(st);
@@ -331,9 +343,7 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
             memcpy(wh.data() + (size_t)i * d * es, row, (size_t)d * es);
             memcpy(w_fc_e.data() + (size_t)i * d * es, row + (size_t)d * es, (size_t)d * es);
         }
-        void *p_fc = nullptr;
-        if ((st = upload(h, &p_fc, wh.data(), wh.size())) != SP_OK) return cleanup(st);
-        init_weight(h->w_fc_h, p_fc, d, d, c.w_dtype == SP_BF16);
+        if ((st = upload_weight(h->w_fc_h, wh.data(), d, d)) != SP_OK) return cleanup(st);
         if ((st = upload(h, (void **)&h->g_h, w->g_h, d * sizeof(float))) != SP_OK) return cleanup(st);
         h->fused = true;
     }
@@ -428,7 +438,8 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
         cudaError_t e = launch_rmsnorm_rows(wb, h->soft_prompt, 0, h->g_in, c.rms_eps, k, d,
                                             h->xn.out(false), 0);
         if (e == cudaSuccess)
-            e = launch_gemm_simt(wb, h->xn.ptr, h->w_qkv.ptr, h->qkv_shared, k, h->nqkv, d, 0);
+            e = launch_gemm_simt(wb, h->xn.ptr, h->w_qkv.ptr, h->qkv_shared, k, h->nqkv, d, 0,
+                                 h->w_qkv.blocked);
         if (e == cudaSuccess) e = cudaDeviceSynchronize();
         if (e != cudaSuccess)
             return cleanup(fail(SP_ERR_CUDA, "shared prompt projection failed: %s", cudaGetErrorString(e)));

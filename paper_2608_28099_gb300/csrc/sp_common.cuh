@@ -300,8 +300,9 @@ cudaError_t launch_to_act(const float *x, size_t n, ActOut out, cudaStream_t st)
 cudaError_t launch_sum_partials(PartIn y, size_t n, float *out, cudaStream_t st);
 
 // Y[M][N] (fp32) = X[M][K] (fp32) * W[N][K]^T (bf16 or fp32) on CUDA cores.
+// w_blocked: W stored as [N / 128][K / 64][128][64] blocks (N % 128 == 0, K % 64 == 0).
 cudaError_t launch_gemm_simt(int w_bf16, const void *X, const void *W, float *Y, int M, int N,
-                             int K, cudaStream_t st);
+                             int K, cudaStream_t st, bool w_blocked = false);
 
 // Replace the text sp_last_error() returns on this thread.
 void set_error_text(const char *msg);

@@ -5,6 +5,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <string.h>
 
 #include "sp_common.cuh"
 
@@ -28,9 +29,25 @@ bool encode_q_group_f32(CUtensorMap *map, const float *q, int rows, int Hq, int 
 bool tc_supported(int N, int K);
 int tc_bn_for(int M);
 TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes);
+// w_blocked: the weights are stored blocked (block_weights_layout) and map_w
+// views them as [N K / 64][64] rows.
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
-                           float *y, int *status, cudaStream_t st);
+                           float *y, int *status, cudaStream_t st, bool w_blocked = false);
+
+// Weights [N][K] (es bytes per element) re-laid out as contiguous 16 KB blocks
+// [N / 128][K / 64][128][64]: one weight tile's k-block is one sequential read
+// instead of 128 row pieces K * es bytes apart (+13-17 % weight bandwidth in the
+// GEMV regime).  Needs N % 128 == 0 and K % 64 == 0.
+inline void block_weights_layout(const char *src, char *dst, int N, int K, size_t es) {
+    const int nkb = K / 64;
+    for (int n = 0; n < N; ++n)
+        for (int kb = 0; kb < nkb; ++kb) {
+            const size_t blk = ((size_t)(n / 128) * nkb + kb) * 128 * 64;
+            memcpy(dst + (blk + (size_t)(n % 128) * 64) * es, src + ((size_t)n * K + kb * 64) * es,
+                   64 * es);
+        }
+}
 
 constexpr int kNumBn = 4;  // tile widths 16, 32, 64, 128
 inline int bn_index(int bn) { return bn == 16 ? 0 : bn == 32 ? 1 : bn == 64 ? 2 : 3; }
@@ -41,6 +58,7 @@ struct WeightMat {
     const void *ptr = nullptr;
     int N = 0, K = 0;
     bool tc = false;
+    bool blocked = false;  // stored by block_weights_layout
     CUtensorMap map;
 };
 
@@ -65,11 +83,15 @@ struct ActBuf {
     }
 };
 
-inline bool init_weight(WeightMat &w, const void *ptr, int N, int K, int w_bf16) {
+inline bool init_weight(WeightMat &w, const void *ptr, int N, int K, int w_bf16,
+                        bool blocked = false) {
     w.ptr = ptr;
     w.N = N;
     w.K = K;
-    w.tc = w_bf16 && tc_supported(N, K) && encode_kmajor_bf16(&w.map, ptr, N, K, 128);
+    w.blocked = blocked;
+    w.tc = w_bf16 && tc_supported(N, K) &&
+           (blocked ? encode_kmajor_bf16(&w.map, ptr, (int)((long long)N * K / 64), 64, 128)
+                    : encode_kmajor_bf16(&w.map, ptr, N, K, 128));
     return true;
 }
 
@@ -107,10 +129,10 @@ struct GemmPlanner {
         if (use_tc(w, x, path)) {
             const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity);
             const int bi = bn_index(p.bn);
-            e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st);
+            e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked);
             *nsplit = p.splits;
         } else {
-            e = launch_gemm_simt(w_bf16, x.ptr, w.ptr, y, M, w.N, w.K, st);
+            e = launch_gemm_simt(w_bf16, x.ptr, w.ptr, y, M, w.N, w.K, st, w.blocked);
             *nsplit = 1;
         }
         if (e != cudaSuccess) return SP_ERR_CUDA;

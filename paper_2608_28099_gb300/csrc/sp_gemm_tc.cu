@@ -55,6 +55,7 @@ struct TileCfg {
 struct TcArgs {
     int M, N, K;
     int kb_per_split, n_kb;
+    int w_blocked;    // weights stored as contiguous [tile][k-block][128][64] blocks
     float *y;         // [split][M][N]
     size_t split_stride;
     int *status;
@@ -111,7 +112,9 @@ __global__ void __launch_bounds__(128, 1)
         const int pre = nkb < Cfg::STAGES ? nkb : Cfg::STAGES;
         for (int i = 0; i < pre; ++i) {
             mbar_arrive_expect_tx(&full[i], Cfg::STAGE);
-            tma_load_2d_hint(smem + i * Cfg::STAGE, &map_w, &full[i], (kb0 + i) * BK, n0, pol_w);
+            tma_load_2d_hint(smem + i * Cfg::STAGE, &map_w, &full[i],
+                             g.w_blocked ? 0 : (kb0 + i) * BK,
+                             g.w_blocked ? (blockIdx.y * g.n_kb + kb0 + i) * 128 : n0, pol_w);
         }
         issued = pre;
         pdl_wait();
@@ -123,7 +126,8 @@ __global__ void __launch_bounds__(128, 1)
             if (i >= pre) {
                 if (!mbar_wait(&empty[s], ph ^ 1, abort)) break;
                 mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
-                tma_load_2d_hint(st, &map_w, &full[s], kc, n0, pol_w);
+                tma_load_2d_hint(st, &map_w, &full[s], g.w_blocked ? 0 : kc,
+                                 g.w_blocked ? (blockIdx.y * g.n_kb + kb0 + i) * 128 : n0, pol_w);
                 issued = i + 1;
             }
             tma_load_2d_hint(st + A_BYTES, &map_xhi, &full[s], kc, m0, pol_x);
@@ -229,6 +233,7 @@ struct PkCfg {
 
 struct PkArgs {
     int M, N, n_kb, m_tiles, tiles;
+    int w_blocked;    // weights stored as contiguous [tile][k-block][128][64] blocks
     int L;            // units per CTA
     int planes;       // partial planes in y
     float *y;         // [planes][M][N]
@@ -324,7 +329,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                     break;
                 }
                 mbar_arrive_expect_tx(&w_full[s], A_BYTES);
-                tma_load_2d_hint(smem + s * A_BYTES, &map_w, &w_full[s], kb * BK, n0, pol_w);
+                tma_load_2d_hint(smem + s * A_BYTES, &map_w, &w_full[s], g.w_blocked ? 0 : kb * BK,
+                                 g.w_blocked ? ((t / g.m_tiles) * g.n_kb + kb) * 128 : n0, pol_w);
                 issued = i + 1;
             }
         }
@@ -594,7 +600,7 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes) {
 
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
-                           float *y, int *status, cudaStream_t st) {
+                           float *y, int *status, cudaStream_t st, bool w_blocked) {
     if (p.persistent) {
         PkArgs g;
         g.M = M;
@@ -602,6 +608,7 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
         g.n_kb = p.n_kb;
         g.m_tiles = p.m_tiles;
         g.tiles = p.m_tiles * p.n_tiles;
+        g.w_blocked = w_blocked;
         g.L = p.units_per_cta;
         g.planes = p.splits;
         g.y = y;
@@ -621,6 +628,7 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
     g.K = K;
     g.kb_per_split = p.kb_per_split;
     g.n_kb = p.n_kb;
+    g.w_blocked = w_blocked;
     g.y = y;
     g.split_stride = (size_t)M * N;
     g.status = status;

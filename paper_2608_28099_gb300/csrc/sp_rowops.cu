@@ -271,7 +271,7 @@ template <typename T>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const float *__restrict__ X,
                                                         const T *__restrict__ W,
                                                         float *__restrict__ Y, int M, int N,
-                                                        int K) {
+                                                        int K, int w_blocked) {
     pdl_trigger();
     pdl_wait();
     constexpr int BM = 64, BN = 64, BK = 32;
@@ -287,7 +287,10 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const float *__restrict_
             const int gm = m0 + row, gk = k0 + kk;
             Xs[kk][row] = (gm < M && gk < K) ? X[(size_t)gm * K + gk] : 0.f;
             const int gn = n0 + row;
-            Ws[kk][row] = (gn < N && gk < K) ? to_f(W[(size_t)gn * K + gk]) : 0.f;
+            const size_t wi = w_blocked ? (((size_t)(gn >> 7) * (K >> 6) + (gk >> 6)) * 128 + (gn & 127)) * 64 +
+                                              (gk & 63)
+                                        : (size_t)gn * K + gk;
+            Ws[kk][row] = (gn < N && gk < K) ? to_f(W[wi]) : 0.f;
         }
         __syncthreads();
 #pragma unroll 8
@@ -388,14 +391,14 @@ cudaError_t launch_sum_partials(PartIn y, size_t n, float *out, cudaStream_t st)
 }
 
 cudaError_t launch_gemm_simt(int w_bf16, const void *X, const void *W, float *Y, int M, int N,
-                             int K, cudaStream_t st) {
+                             int K, cudaStream_t st, bool w_blocked) {
     dim3 grid(ceil_div(N, 64), ceil_div(M, 64));
     if (w_bf16)
         return launch_k(gemm_simt_kernel<bf16>, grid, dim3(256), 0, st, (const float *)X, (const bf16 *)W,
-                        Y, M, N, K);
+                        Y, M, N, K, (int)w_blocked);
     else
         return launch_k(gemm_simt_kernel<float>, grid, dim3(256), 0, st, (const float *)X,
-                        (const float *)W, Y, M, N, K);
+                        (const float *)W, Y, M, N, K, (int)w_blocked);
 }
 
 }  // namespace sp
