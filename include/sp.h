@@ -301,6 +301,8 @@ SP_API size_t sp_attend_workspace_bytes(const sp_attn_dims *dims, int batch);
  *   d_k_new [batch][k][Hkv][dh] float device (already rotated), d_v_new same
  *   d_out   [batch][k][Hq][dh], float (out_dtype SP_F32) or bf16 (SP_BF16)
  * Row r of sequence b sees the L_b cached tokens and new tokens 0..r.
+ * d_q, d_k_new, d_v_new and d_out must be 16-byte aligned (SP_ERR_INVALID_ARG
+ * otherwise): the kernels move whole 16-byte vectors.
  * d_workspace: caller-allocated, >= sp_attend_workspace_bytes(dims, batch).
  * d_status: optional device int (OR-ed SP_DEV_* bits), NULL = not recorded.
  * d_gathered_pages: optional device int32 [batch][kv->max_pages_per_seq]

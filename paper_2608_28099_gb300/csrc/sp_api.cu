@@ -898,6 +898,8 @@ sp_status sp_attend(sp_stream stream, const sp_attn_dims *dm, int batch, const i
     if (!d_seq_lens || !d_q || !d_k_new || !d_v_new || !d_out || !d_workspace)
         return fail(SP_ERR_INVALID_ARG, "a required pointer is NULL");
     if (((uintptr_t)d_workspace) & 255) return fail(SP_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    if ((((uintptr_t)d_q) | ((uintptr_t)d_k_new) | ((uintptr_t)d_v_new) | ((uintptr_t)d_out)) & 15)
+        return fail(SP_ERR_INVALID_ARG, "queries, new keys/values and the output must be 16-byte aligned");
     sp_status s = check_kv(kv, dm->kv_dtype);
     if (s != SP_OK) return s;
     if (!d_seq_ids && batch > kv->n_seqs)

@@ -78,8 +78,9 @@ constexpr int OFF_PREFIX = OFF_KV + STG * KV_STAGE;
 constexpr int MAX_GRP = 256;                   // groups (cuts table in smem)
 constexpr int OFF_CUTS = OFF_PREFIX + (MAX_B + 4) * 4;
 constexpr int OFF_BAR = OFF_CUTS + (MAX_GRP + 4) * 4;
-constexpr int OFF_ML = OFF_BAR + 512;           // warpgroup 1's (max, sum) per row; merge scales
-constexpr int SMEM_BYTES = OFF_ML + 1024 + 1024;
+constexpr int OFF_ML = OFF_BAR + 512;           // both warpgroups' (max, sum) per row, 2 KB
+// + 1 KB: the kernel rounds the dynamic shared window's start up to 1024 bytes
+constexpr int SMEM_BYTES = OFF_ML + 2048 + 1024;
 constexpr int THREADS = 384;                   // 2 softmax warpgroups, 2 producers, 2 MMA
 constexpr int PRODUCER_WARP = 8, MMA_WARP = 9, MMA_WARP1 = 10, PRODUCER_WARP1 = 11;
 constexpr float RESCALE_LOG2 = 8.f;            // tolerate p <= 2^8 before rescaling O
@@ -676,30 +677,27 @@ __global__ void __launch_bounds__(THREADS, 1)
             k0 += n0;
             k1 += n1;
 
-            // ---- epilogue: warpgroup 1 hands its (max, sum) to warpgroup 0 through
-            // shared memory and loads half of the next segment's queries; warpgroup 0
-            // combines (max, sum, O) of both, writes the pair's output (whole pair in
-            // this CTA's share) or this segment's partial, and loads the other half
+            // ---- epilogue, shared by the two warpgroups: each hands its (max, sum)
+            // to the other through shared memory, combines (max, sum, O) of both
+            // pipelines over its half of the columns, writes the pair's output
+            // (whole pair in this CTA's share) or this segment's partial, and loads
+            // its half of the next segment's queries
             const Seg sg = seg_at(prefix, B, xs, x1);
             const int b = sg.b;
             const int j_first = group_of(cuts, n_grp, sg.xp);
             const int j_last = group_of(cuts, n_grp, sg.xp + sg.nt - 1);
             const bool whole = j_first == j_last;
-            if (wg == 1) {
-                sm_ml[row] = n1 > 0 ? m : -INFINITY;
-                sm_ml[128 + row] = n1 > 0 ? l : 0.f;
-            }
+            const bool mine = wg == 0 || n1 > 0;  // pipeline 0 has >= 1 tile, pipeline 1 may have none
+            sm_ml[wg * 256 + row] = mine ? m : -INFINITY;
+            sm_ml[wg * 256 + 128 + row] = mine ? l : 0.f;
             // both warpgroups are past their last S of the segment: Q may be rewritten
             named_sync(BAR_EPI, n_cons);
-            if (wg == 1) {
-                if (x < x1) load_q(seg_at(prefix, B, x, x1).b);
-                continue;
-            }
-            const float m1 = sm_ml[row], l1 = sm_ml[128 + row];
-            const float mc = fmaxf(m, m1);
-            const float a0 = (m == -INFINITY) ? 0.f : fast_exp2(m - mc);
+            const float m0 = sm_ml[row], l0 = sm_ml[128 + row];
+            const float m1 = sm_ml[256 + row], l1 = sm_ml[384 + row];
+            const float mc = fmaxf(m0, m1);
+            const float a0 = (m0 == -INFINITY) ? 0.f : fast_exp2(m0 - mc);
             const float a1 = (m1 == -INFINITY) ? 0.f : fast_exp2(m1 - mc);
-            const float lsum = a0 * l + a1 * l1;
+            const float lsum = a0 * l0 + a1 * l1;
             bool have = ok && mbar_wait(&bars->pv_done[0], (uint32_t)((k0 - 1) & 1), abort);
             if (have && n1 > 0) have = mbar_wait(&bars->pv_done[1], (uint32_t)((k1 - 1) & 1), abort);
             have = __all_sync(0xffffffffu, have);  // the TMEM loads below are warp-collective
@@ -712,7 +710,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (have) {
                 tc_fence_after();
 #pragma unroll 1
-                for (int c0 = 0; c0 < DH; c0 += 32) {
+                for (int c0 = wg * (DH / 2); c0 < (wg + 1) * (DH / 2); c0 += 32) {
                     float o0[32], o1[32];
                     tmem_ld32(lane_base + O_COL + c0, o0);
                     if (n1 > 0) {
@@ -738,7 +736,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                                             a0 * o0[jj + 3] + a1 * o1[jj + 3]);
                     }
                 }
-                if (active && !whole) {
+                if (active && !whole && wg == 0) {
                     a.part_ml[(slot * R + row) * 2] = mc;
                     a.part_ml[(slot * R + row) * 2 + 1] = lsum;
                 }
@@ -756,7 +754,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     // every MMA must be finished before TMEM and shared memory go away
     mbar_wait_drain(&bars->fin, 0);
-    if (warp < 4) __threadfence();  // the partials are visible device-wide before they are counted
+    if (warp < 8) __threadfence();  // the partials are visible device-wide before they are counted
     tc_fence_before();
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -777,79 +775,97 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
 
     // ---- merges, by the whole CTA: every segment of pair (b, g) has written its
-    // partial (slots (j + b) Hkv + g, j = j0 .. j1).  One pass per (row, 4
-    // columns), the partials' loads issued together in chunks of MCH with an
-    // online rescale between chunks, and MIT items in flight per thread.
-    constexpr int MCH = 4, MIT = 2;
-    for (int t = 0; t < bars->n_merge; ++t) {
-        const int b = bars->m_b[t], j0 = bars->m_j0[t], ns = bars->m_j1[t] - j0 + 1;
-        const size_t slot0 = ((size_t)j0 + b) * Hkv + g;  // slot of segment j0 + e: slot0 + e Hkv
-        const int items = R * (DH / 4);
-        for (int i0 = threadIdx.x; i0 < items; i0 += THREADS * MIT) {
-            float mm[MIT], ls[MIT];
-            float4 o[MIT];
+    // partial (slots (j + b) Hkv + g, j = j0 .. j1).  One item per (pair, row, 8
+    // columns), the items of all of this CTA's pairs (at most 2) in one pass: the
+    // partials' loads issued together MCH segments at a time with an online
+    // rescale between chunks, MIT items in flight per thread.
+    constexpr int MCH = 2, MIT = 3, CPI = 8;  // columns per item
+    const int items = R * (DH / CPI), n_merge = bars->n_merge;
+    const int n_items = n_merge * items;
+    for (int i0 = threadIdx.x; i0 < n_items; i0 += THREADS * MIT) {
+        float mm[MIT], ls[MIT];
+        float4 o[MIT][2];
+        int nsu[MIT], rru[MIT], cqu[MIT], bu[MIT];
+        size_t s0u[MIT];  // slot of segment j0 + e of the item's pair: s0u + e Hkv
+        int ns_max = 0;
+#pragma unroll
+        for (int u = 0; u < MIT; ++u) {
+            mm[u] = -INFINITY;
+            ls[u] = 0.f;
+            o[u][0] = o[u][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+            const int ia = i0 + u * THREADS;
+            const int t = min(ia / items, n_merge - 1);  // items past the end: no loads, no store
+            const int idx = ia - t * items;
+            const int j0 = bars->m_j0[t];
+            bu[u] = bars->m_b[t];
+            nsu[u] = ia < n_items ? bars->m_j1[t] - j0 + 1 : 0;
+            s0u[u] = ((size_t)j0 + bu[u]) * Hkv + g;
+            rru[u] = idx / (DH / CPI);
+            cqu[u] = (idx % (DH / CPI)) * CPI;
+            ns_max = max(ns_max, nsu[u]);
+        }
+        for (int e0 = 0; e0 < ns_max; e0 += MCH) {
+            float mv[MIT][MCH], lv[MIT][MCH];
+            float4 ov[MIT][MCH][2];
 #pragma unroll
             for (int u = 0; u < MIT; ++u) {
-                mm[u] = -INFINITY;
-                ls[u] = 0.f;
-                o[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-            }
-            for (int e0 = 0; e0 < ns; e0 += MCH) {
-                float mv[MIT][MCH], lv[MIT][MCH];
-                float4 ov[MIT][MCH];
 #pragma unroll
-                for (int u = 0; u < MIT; ++u) {
-                    const int idx = i0 + u * THREADS;
-                    const int rr = idx / (DH / 4), cq = (idx % (DH / 4)) * 4;
-#pragma unroll
-                    for (int e = 0; e < MCH; ++e) {
-                        const bool in = idx < items && e0 + e < ns;
-                        const size_t sl = slot0 + (size_t)(e0 + e) * Hkv;
-                        const float2 ml = in ? __ldcg((const float2 *)(a.part_ml + (sl * R + rr) * 2))
-                                             : make_float2(-INFINITY, 0.f);
-                        mv[u][e] = ml.x;
-                        lv[u][e] = ml.y;
-                        ov[u][e] = in ? __ldcg((const float4 *)(a.part_o + (sl * R + rr) * DH + cq))
-                                      : make_float4(0.f, 0.f, 0.f, 0.f);
-                    }
-                }
-#pragma unroll
-                for (int u = 0; u < MIT; ++u) {
-                    float mn = mm[u];
-#pragma unroll
-                    for (int e = 0; e < MCH; ++e) mn = fmaxf(mn, mv[u][e]);
-                    if (mn == -INFINITY) continue;
-                    const float al = mm[u] == -INFINITY ? 0.f : exp2f(mm[u] - mn);
-                    ls[u] *= al;
-                    o[u].x *= al;
-                    o[u].y *= al;
-                    o[u].z *= al;
-                    o[u].w *= al;
-#pragma unroll
-                    for (int e = 0; e < MCH; ++e) {
-                        const float wgt = mv[u][e] == -INFINITY ? 0.f : exp2f(mv[u][e] - mn);
-                        ls[u] += wgt * lv[u][e];
-                        o[u].x += wgt * ov[u][e].x;
-                        o[u].y += wgt * ov[u][e].y;
-                        o[u].z += wgt * ov[u][e].z;
-                        o[u].w += wgt * ov[u][e].w;
-                    }
-                    mm[u] = mn;
+                for (int e = 0; e < MCH; ++e) {
+                    const bool in = e0 + e < nsu[u];
+                    const size_t sl = s0u[u] + (size_t)(e0 + e) * Hkv;
+                    const float2 ml = in ? __ldcg((const float2 *)(a.part_ml + (sl * R + rru[u]) * 2))
+                                         : make_float2(-INFINITY, 0.f);
+                    mv[u][e] = ml.x;
+                    lv[u][e] = ml.y;
+                    const float4 *src = (const float4 *)(a.part_o + (sl * R + rru[u]) * DH + cqu[u]);
+                    ov[u][e][0] = in ? __ldcg(src) : make_float4(0.f, 0.f, 0.f, 0.f);
+                    ov[u][e][1] = in ? __ldcg(src + 1) : make_float4(0.f, 0.f, 0.f, 0.f);
                 }
             }
 #pragma unroll
             for (int u = 0; u < MIT; ++u) {
-                const int idx = i0 + u * THREADS;
-                if (idx >= items) continue;
-                const int rr = idx / (DH / 4), cq = (idx % (DH / 4)) * 4;
-                const float inv = ls[u] > 0.f ? 1.f / ls[u] : 0.f;
-                const int hl = rr / k, r = rr - hl * k;
-                act_store4(a.out, (((size_t)b * k + r) * a.Hq + g * a.G + hl) * DH + cq,
-                           make_float4(o[u].x * inv, o[u].y * inv, o[u].z * inv, o[u].w * inv));
+                float mn = mm[u];
+#pragma unroll
+                for (int e = 0; e < MCH; ++e) mn = fmaxf(mn, mv[u][e]);
+                if (mn == -INFINITY) continue;
+                const float al = mm[u] == -INFINITY ? 0.f : exp2f(mm[u] - mn);
+                ls[u] *= al;
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    o[u][h].x *= al;
+                    o[u][h].y *= al;
+                    o[u][h].z *= al;
+                    o[u][h].w *= al;
+                }
+#pragma unroll
+                for (int e = 0; e < MCH; ++e) {
+                    const float wgt = mv[u][e] == -INFINITY ? 0.f : exp2f(mv[u][e] - mn);
+                    ls[u] += wgt * lv[u][e];
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        o[u][h].x += wgt * ov[u][e][h].x;
+                        o[u][h].y += wgt * ov[u][e][h].y;
+                        o[u][h].z += wgt * ov[u][e][h].z;
+                        o[u][h].w += wgt * ov[u][e][h].w;
+                    }
+                }
+                mm[u] = mn;
             }
         }
-        if (threadIdx.x == 0) a.counters[b * Hkv + g] = 0;  // ready for a launch that does not clear it
+#pragma unroll
+        for (int u = 0; u < MIT; ++u) {
+            if (i0 + u * THREADS >= n_items) continue;
+            const float inv = ls[u] > 0.f ? 1.f / ls[u] : 0.f;
+            const int hl = rru[u] / k, r = rru[u] - hl * k;
+            const size_t dst = (((size_t)bu[u] * k + r) * a.Hq + g * a.G + hl) * DH + cqu[u];
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+                act_store4(a.out, dst + 4 * h,
+                           make_float4(o[u][h].x * inv, o[u][h].y * inv, o[u][h].z * inv, o[u][h].w * inv));
+        }
     }
+    // ready for a launch that does not clear them
+    if (threadIdx.x < n_merge) a.counters[bars->m_b[threadIdx.x] * Hkv + g] = 0;
 }
 
 // Merge of the partial segments for small batches (a few long sequences, each
