@@ -43,12 +43,10 @@ UNIT = "sequences/s"
 FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS = 6800.0, 1900.0
 FLUSH_BYTES = 256 << 20
 
-# DRAM traffic per launch of the dominant kernel from an ncu capture of the same
-# kernel build (profiles/); None until one is taken for the current kernel.
 # DRAM read + write per launch of the dominant kernel, from one ncu capture of
 # the current kernel on the same workload (profiles/attn_tc_kernel_*.md); a
 # workload or kernel without a capture reports null.
-TRAFFIC_BYTES = {("4b", "attention"): 78501120, ("27b_long", "attention"): 1086287872}
+TRAFFIC_BYTES = {("4b", "attention"): 78714112}
 
 
 def parse_args():
