@@ -79,8 +79,11 @@ constexpr int MAX_GRP = 256;                   // groups (cuts table in smem)
 constexpr int OFF_CUTS = OFF_PREFIX + (MAX_B + 4) * 4;
 constexpr int OFF_BAR = OFF_CUTS + (MAX_GRP + 4) * 4;
 constexpr int OFF_ML = OFF_BAR + 512;           // both warpgroups' (max, sum) per row, 2 KB
+// each sequence's cache id and length, resolved once at the start (the segment
+// loops then make no global round trip for them)
+constexpr int OFF_SEQ = OFF_ML + 2048;
 // + 1 KB: the kernel rounds the dynamic shared window's start up to 1024 bytes
-constexpr int SMEM_BYTES = OFF_ML + 2048 + 1024;
+constexpr int SMEM_BYTES = OFF_SEQ + MAX_B * 8 + 1024;
 constexpr int THREADS = 384;                   // 2 softmax warpgroups, 2 producers, 2 MMA
 constexpr int PRODUCER_WARP = 8, MMA_WARP = 9, MMA_WARP1 = 10, PRODUCER_WARP1 = 11;
 constexpr float RESCALE_LOG2 = 8.f;            // tolerate p <= 2^8 before rescaling O
@@ -200,6 +203,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     // ---- the tile list: prefix[b] = sum_{b' < b} ceil((L_b' + k) / TT).
     // Lengths and ids come from the caller, not from the previous kernel, so
     // this runs before pdl_wait.
+    int2 *seqs = (int2 *)(smem + OFF_SEQ);  // (sid, len) of sequence b
     {
         const int per = (B + THREADS - 1) / THREADS;
         const int b0 = min(B, (int)threadIdx.x * per), b1 = min(B, b0 + per);
@@ -207,6 +211,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int bb = b0; bb < b1; ++bb) {
             const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, bb, a.kv.n_seqs,
                                           a.max_seq_len, blockIdx.x == 0 ? a.status : nullptr);
+            seqs[bb] = make_int2(sq.sid, sq.len);
             const int v = ceil_div(sq.len + a.r0 + k, TT);
             prefix[bb] = v;
             sum += v;
@@ -300,8 +305,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             const Seg sg = seg_at(prefix, B, x, x1);
             x += sg.n;
             const int b = sg.b;
-            const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.kv.n_seqs,
-                                          a.max_seq_len, nullptr);
+            const int2 sq2 = seqs[b];
+            const SeqRef sq = {sq2.x, sq2.y};
             const int L = sq.len, total = L + a.r0 + k;
             const int *ptab = paged ? a.kv.page_table + (size_t)max(sq.sid, 0) * a.kv.max_pages : nullptr;
             for (int i = 0; i < sg.n; ++i, ++ci) {
@@ -585,8 +590,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             {
                 const Seg sg = seg_at(prefix, B, x, x1);
                 n_tiles = sg.n;
-                const SeqRef sq = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, sg.b, a.kv.n_seqs,
-                                              a.max_seq_len, nullptr);
+                const int2 sq2 = seqs[sg.b];
+                const SeqRef sq = {sq2.x, sq2.y};
                 // this row sees tokens t < L + r0 + r + 1 except the new rows of
                 // other tasks before its own, [L, L + lo); relative to the segment start:
                 lim_rel = sq.len + a.r0 + r_soft + 1 - sg.t_a * TT;
