@@ -46,7 +46,7 @@ FLUSH_BYTES = 256 << 20
 # DRAM read + write per launch of the dominant kernel, from one ncu capture of
 # the current kernel on the same workload (profiles/attn_tc_kernel_*.md); a
 # workload or kernel without a capture reports null.
-TRAFFIC_BYTES = {("4b", "attention"): 78714112}
+TRAFFIC_BYTES = {("4b", "attention"): 77519616}
 
 
 def parse_args():
