@@ -88,3 +88,18 @@ def test_attend_rejects_bad_dims_on_host(lib):
     assert st == sp.SP_ERR_INVALID_ARG
     dims = sp.sp_attn_dims(4, 2, 32, 4, sp.SP_F32, 64, 100)   # split not a multiple of 64
     assert lib.sp_attend_workspace_bytes(C.byref(dims), 1) == 0
+
+
+@pytest.mark.parametrize("bad", ["q", "k_new", "v_new", "out"])
+def test_attend_rejects_misaligned_vectors_on_host(lib, bad):
+    # the kernels move whole 16-byte vectors: a pointer off by 4 bytes is refused
+    # before any launch (the fake addresses are never dereferenced)
+    kv = sp.sp_kv_cache()
+    dims = sp.sp_attn_dims(4, 2, 128, 4, sp.SP_BF16, 64, 0)
+    ptr = {n: C.c_void_p(0x100000 * (i + 1)) for i, n in enumerate(["q", "k_new", "v_new", "out"])}
+    ptr[bad] = C.c_void_p(ptr[bad].value + 4)
+    lens, ws = C.c_void_p(0x900000), C.c_void_p(0xA00000)
+    st = lib.sp_attend(None, C.byref(dims), 1, None, lens, C.byref(kv), ptr["q"], ptr["k_new"],
+                       ptr["v_new"], ptr["out"], sp.SP_F32, ws, 1 << 20, None, None)
+    assert st == sp.SP_ERR_INVALID_ARG
+    assert "16-byte aligned" in sp.sp_last_error()
