@@ -31,9 +31,10 @@
 //   O_w  += P_i V_i           P written as bf16 over the first half of S_w (A
 //                             operand from TMEM), V read in place from shared
 //                             memory as an MN-major B operand
-// At the end of a segment warpgroup 0 folds warpgroup 1's state into its own
-// (both O accumulators sit on the same TMEM lanes), writes the output or the
-// partial, and loads the next segment's queries into TMEM.  The even and odd
+// At the end of a segment the two warpgroups swap their (max, sum) through
+// shared memory; each then combines both O accumulators (they sit on the same
+// TMEM lanes) over half of the columns, writes that half of the output or the
+// partial, and loads half of the next segment's queries into TMEM.  The even and odd
 // tiles form two independent pipelines, each with its own MMA issuing warp:
 // one thread issuing small-N MMAs back to back leaves the tensor pipe idle
 // between them, two keep it busy.
