@@ -157,19 +157,19 @@ __global__ void swiglu_kernel(PartIn y, int M, int f, int blk, ActOut a) {
 }
 
 // Pooling and the linear head, column-parallel: block (chunk, b) pools 64
-// hidden columns of sequence b (h2 = h1 + y summed over the k rows by four
+// hidden columns of sequence b (h2 = h1 + y summed over the k rows by two
 // row groups, then mean or last) and writes its partial dot products with
-// every head row to part[b][chunk][C]; four classes are reduced at a time.
+// every head row to part[b][chunk][C]; two classes are reduced at a time.
 constexpr int kReadoutCols = 64;
+constexpr int kReadoutGroups = 2;  // row groups of a block (threads = 64 x 2)
 
-__global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const float *__restrict__ h1,
-                                       const float *__restrict__ head_w, int pool, int k, int d,
-                                       int C, float *__restrict__ part, size_t sb, size_t sr,
-                                       int n_tasks, const float *__restrict__ g_final,
-                                       float *__restrict__ part_ss) {
+// six blocks per SM: all blocks of a 4b-sized call in one wave
+__global__ void __launch_bounds__(kReadoutCols * kReadoutGroups, 6)
+readout_partial_kernel(PartIn y, const float *__restrict__ h1, const float *__restrict__ head_w,
+                       int pool, int k, int d, int C, float *__restrict__ part, size_t sb, size_t sr,
+                       int n_tasks, const float *__restrict__ g_final, float *__restrict__ part_ss) {
     pdl_trigger();
-    pdl_wait();
-    __shared__ float acc_s[4][kReadoutCols];
+    __shared__ float acc_s[kReadoutGroups][kReadoutCols];
     __shared__ float pooled[kReadoutCols];
     __shared__ float red[4][8];
     const int chunk = blockIdx.x, b = blockIdx.y;
@@ -177,6 +177,10 @@ __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const fl
     const int col = chunk * kReadoutCols + c;
     const size_t base = (size_t)b * sb;
     head_w += (size_t)(b % n_tasks) * C * d;  // this task's head
+    // the head is a constant of the handle, not an output of the previous
+    // kernel: the first classes' weights are fetched before the wait
+    const float hw0 = (rg < C && col < d) ? head_w[(size_t)rg * d + col] : 0.f;
+    pdl_wait();
     float acc = 0.f;
     if (col < d) {
         if (pool == SP_POOL_LAST) {
@@ -185,16 +189,41 @@ __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const fl
                 acc = h1[o] + part_get(y, o);
             }
         } else {
-            for (int r = rg; r < k; r += 4) {
-                const size_t o = base + (size_t)r * sr + col;
-                acc += h1[o] + part_get(y, o);
+            // rows rg, rg + G, ... (G row groups), four at a time with the loads
+            // of all their partials issued together
+            for (int r0 = rg; r0 < k; r0 += 4 * kReadoutGroups) {
+                size_t o[4];
+                bool in[4];
+                float v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int r = r0 + u * kReadoutGroups;
+                    in[u] = r < k;
+                    o[u] = base + (size_t)(in[u] ? r : r0) * sr + col;
+                    v[u] = in[u] ? h1[o[u]] : 0.f;
+                }
+                for (int i0 = 0; i0 < y.n; i0 += 8) {
+                    float pv[4][8];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+#pragma unroll
+                        for (int jj = 0; jj < 8; ++jj)
+                            pv[u][jj] = (in[u] && i0 + jj < y.n) ? y.y[(size_t)(i0 + jj) * y.stride + o[u]] : 0.f;
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+#pragma unroll
+                        for (int jj = 0; jj < 8; ++jj) v[u] += pv[u][jj];
+                }
+                acc += (v[0] + v[1]) + (v[2] + v[3]);
             }
         }
     }
     acc_s[rg][c] = acc;
     __syncthreads();
     if (threadIdx.x < kReadoutCols) {
-        const float sum = (acc_s[0][c] + acc_s[1][c]) + (acc_s[2][c] + acc_s[3][c]);
+        float sum = 0.f;
+#pragma unroll
+        for (int q = 0; q < kReadoutGroups; ++q) sum += acc_s[q][c];
         const float p = pool == SP_POOL_LAST ? sum : sum / (float)k;
         if (g_final) {
             // LM-head readout: the chunk's share of the pooled row's square sum,
@@ -212,16 +241,18 @@ __global__ void __launch_bounds__(256) readout_partial_kernel(PartIn y, const fl
     __syncthreads();
     if (g_final && threadIdx.x == 0)
         part_ss[(size_t)b * gridDim.x + chunk] = red[3][4] + red[3][5];
-    // thread (group cg = tid / 64, column c): class c0 + cg
+    // row group rg takes class c0 + rg; its two warps hold the chunk's 64 columns
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int c0 = 0; c0 < C; c0 += 4) {
+    for (int c0 = 0; c0 < C; c0 += kReadoutGroups) {
         const int cls = c0 + rg;
-        float v = (cls < C && col < d) ? head_w[(size_t)cls * d + col] * pooled[c] : 0.f;
+        const bool use = cls < C && col < d;
+        const float hw = c0 == 0 ? hw0 : (use ? head_w[(size_t)cls * d + col] : 0.f);
+        float v = use ? hw * pooled[c] : 0.f;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
         if (lane == 0) red[w >> 1][w & 1] = v;
         __syncthreads();
-        if (threadIdx.x < 4 && c0 + (int)threadIdx.x < C)
+        if (threadIdx.x < kReadoutGroups && c0 + (int)threadIdx.x < C)
             part[((size_t)b * gridDim.x + chunk) * C + c0 + threadIdx.x] =
                 red[threadIdx.x][0] + red[threadIdx.x][1];
         __syncthreads();
@@ -369,7 +400,7 @@ cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const
     if (!sr) sr = d;
     if (n_tasks < 1) n_tasks = 1;
     float *ss = g_final ? scratch + (size_t)B * chunks * C : nullptr;
-    cudaError_t e = launch_k(readout_partial_kernel, dim3(chunks, B), dim3(256), 0, st, y, h1,
+    cudaError_t e = launch_k(readout_partial_kernel, dim3(chunks, B), dim3(kReadoutCols * kReadoutGroups), 0, st, y, h1,
                              head_w, pool, k, d, C, scratch, sb, sr, n_tasks, g_final, ss);
     if (e != cudaSuccess) return e;
     return launch_k(readout_finish_kernel, dim3(B), dim3(64), 0, st, (const float *)scratch, chunks,
