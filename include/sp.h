@@ -345,7 +345,8 @@ SP_API sp_status sp_attend_static(sp_stream stream, const sp_attn_dims *dims, in
 SP_API size_t sp_project_workspace_bytes(int M, int N, int K);
 
 /* Y[M][N] = X[M][K] W[N][K]^T with X and Y fp32 row-major and W bf16 row-major
- * [N][K] (raw 16-bit patterns), all DEVICE pointers (X, W 16-byte aligned).
+ * [N][K] (raw 16-bit patterns), all DEVICE pointers (X, W 16-byte aligned,
+ * SP_ERR_INVALID_ARG otherwise).
  * path: 1 = CUDA cores, 2 = tensor cores (needs N % 128 == 0 and K % 64 == 0;
  * SP_ERR_UNSUPPORTED otherwise), 0 = tensor cores when supported.  The tensor
  * path splits X into bf16 hi + lo parts and may split K across CTAs; both live

@@ -942,6 +942,8 @@ sp_status sp_project(sp_stream stream, int M, int N, int K, const float *d_x, co
                      float *d_y, int path, void *d_workspace, size_t workspace_bytes) {
     if (M < 1 || N < 1 || K < 1) return fail(SP_ERR_INVALID_ARG, "M, N, K must be >= 1");
     if (!d_x || !d_w || !d_y) return fail(SP_ERR_INVALID_ARG, "a required pointer is NULL");
+    if ((((uintptr_t)d_x) | ((uintptr_t)d_w)) & 15)
+        return fail(SP_ERR_INVALID_ARG, "X and W must be 16-byte aligned");
     if (path < 0 || path > 2) return fail(SP_ERR_INVALID_ARG, "bad path");
     cudaStream_t st = (cudaStream_t)stream;
     const bool tc_ok = tc_supported(N, K);

@@ -103,3 +103,16 @@ def test_attend_rejects_misaligned_vectors_on_host(lib, bad):
                        ptr["v_new"], ptr["out"], sp.SP_F32, ws, 1 << 20, None, None)
     assert st == sp.SP_ERR_INVALID_ARG
     assert "16-byte aligned" in sp.sp_last_error()
+
+
+@pytest.mark.parametrize("bad", ["x", "w"])
+def test_project_rejects_misaligned_operands_on_host(lib, bad):
+    # X and W are read by TMA when the tensor path runs: 16-byte aligned or refused
+    x, w, y = C.c_void_p(0x100000), C.c_void_p(0x200000), C.c_void_p(0x300000)
+    if bad == "x":
+        x = C.c_void_p(x.value + 8)
+    else:
+        w = C.c_void_p(w.value + 8)
+    st = lib.sp_project(None, 128, 256, 128, x, w, y, 0, C.c_void_p(0x400000), 1 << 24)
+    assert st == sp.SP_ERR_INVALID_ARG
+    assert "16-byte aligned" in sp.sp_last_error()
