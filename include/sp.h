@@ -143,7 +143,11 @@ typedef struct sp_weights {
  *    max_pages_per_seq pages is reported as SP_DEV_BAD_PAGE and the excess is
  *    masked.  page_size: 16, 32 or 64.
  *  A contiguous buffer must hold min(L_s, max_seq_len) tokens: its size is not
- *  known to the library, so a length beyond it cannot be detected. */
+ *  known to the library, so a length beyond it cannot be detected.
+ *  Every sequence pointer and both pools must be 16-byte aligned: the kernels
+ *  copy 16-byte vectors.  The pools are checked on the host
+ *  (SP_ERR_INVALID_ARG); the per-sequence pointers live in device memory and
+ *  are the caller's to get right. */
 typedef struct sp_kv_cache {
     int layout;
     const void *const *k_seq;

@@ -152,6 +152,8 @@ sp_status check_kv(const sp_kv_cache *kv, int kv_dtype) {
     } else if (kv->layout == SP_KV_PAGED) {
         if (!kv->k_pool || !kv->v_pool || !kv->page_table)
             return fail(SP_ERR_INVALID_ARG, "paged cache needs k_pool, v_pool and page_table");
+        if ((((uintptr_t)kv->k_pool) | ((uintptr_t)kv->v_pool)) & 15)
+            return fail(SP_ERR_INVALID_ARG, "k_pool and v_pool must be 16-byte aligned");
         if (kv->page_size != 16 && kv->page_size != 32 && kv->page_size != 64)
             return fail(SP_ERR_UNSUPPORTED, "page_size %d unsupported (16, 32, 64)", kv->page_size);
         if (kv->n_pages < 1 || kv->max_pages_per_seq < 1)

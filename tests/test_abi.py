@@ -116,3 +116,13 @@ def test_project_rejects_misaligned_operands_on_host(lib, bad):
     st = lib.sp_project(None, 128, 256, 128, x, w, y, 0, C.c_void_p(0x400000), 1 << 24)
     assert st == sp.SP_ERR_INVALID_ARG
     assert "16-byte aligned" in sp.sp_last_error()
+
+
+def test_attend_rejects_misaligned_pools_on_host(lib):
+    kv = sp.sp_kv_cache(sp.SP_KV_PAGED, None, None, 0x600008, 0x700000, 0x500000, 16, 4, 4, 1)
+    dims = sp.sp_attn_dims(4, 2, 128, 4, sp.SP_BF16, 64, 0)
+    q, kn, vn, out = (C.c_void_p(0x100000 * i) for i in range(1, 5))
+    st = lib.sp_attend(None, C.byref(dims), 1, None, C.c_void_p(0x900000), C.byref(kv), q, kn, vn,
+                       out, sp.SP_F32, C.c_void_p(0xA00000), 1 << 20, None, None)
+    assert st == sp.SP_ERR_INVALID_ARG
+    assert "k_pool and v_pool" in sp.sp_last_error()
