@@ -420,7 +420,68 @@ def check_lm_head_readout_is_scale_invariant():
     assert np.max(np.abs(plain.readout(h2 * 7.5) - plain.readout(h2))) > 1e-3
 
 
-ALL_CHECKS = [check_lm_head_readout_hand_example, check_lm_head_readout_is_scale_invariant,
+def check_bf16_decode_fixed_patterns():
+    # bf16 is the upper half of an IEEE binary32: these bit patterns have fixed values
+    bits = np.array([0x3F80, 0xC020, 0x0001, 0x7F80, 0x8000, 0x4049, 0x0080], dtype=np.uint16)
+    v = so.to_f64(bits, so.BF16)
+    assert v.dtype == np.float64
+    assert v[0] == 1.0 and v[1] == -2.5
+    assert v[2] == 2.0 ** -133                     # smallest bf16 subnormal
+    assert np.isposinf(v[3])
+    assert v[4] == 0.0 and np.signbit(v[4])        # negative zero keeps its sign
+    assert v[5] == 3.140625                        # 0x4049: 1.5703125 * 2
+    assert v[6] == 2.0 ** -126                     # smallest normal
+
+
+def _attention_step_case(seed, lens, kr=3):
+    sh = wl.Shape(16, 4, 2, 8, 24, kr, 3, rope_theta=100.0, w_dtype=wl.F32, kv_dtype=wl.F32)
+    w = wl.custom(sh, lens, wl.LAYOUT_PAGED, seed)
+    _, lw = random_layer(seed + 1, k=kr)
+    layer = so.Layer(sh, lw)
+    rng = np.random.default_rng(seed + 2)
+    x = rng.standard_normal((len(lens), kr, 16)) * 0.5
+    return sh, w, layer, x
+
+
+def check_attention_step_matches_the_layer_trace():
+    # the step-level checker must agree with the attention inside the layer
+    # pass, whose mask and positions the full causal recompute pins
+    sh, w, layer, x = _attention_step_case(70, [0, 1, 5, 16, 23])
+    q, kn, vn, want = [], [], [], []
+    for i, sid in enumerate(w.seq_ids):
+        kc, vc = so.sequence_kv(w.cache, int(sid))
+        tr = {}
+        layer.rows_with_cache(x[i], kc, vc, trace=tr)
+        q.append(tr["q"]); kn.append(tr["k_new"]); vn.append(tr["v_new"]); want.append(tr["o"])
+    got = so.attention_step(sh, w.cache, w.seq_ids, np.array(q), np.array(kn), np.array(vn))
+    np.testing.assert_allclose(got, np.array(want), rtol=1e-12, atol=1e-12)
+
+
+def check_attention_step_uniform_keys_closed_form():
+    # equal keys everywhere: row r averages the values of the L + r + 1 tokens it sees
+    sh, w, _, _ = _attention_step_case(71, [0, 3, 17])
+    rng = np.random.default_rng(72)
+    B, kr, hq, hkv, dh = 3, sh.k_rows, sh.n_q_heads, sh.n_kv_heads, sh.head_dim
+    key = rng.standard_normal((hkv, dh)).astype(np.float32).astype(np.float64)  # exact in the cache
+    cache = dataclasses.replace(w.cache, k_pool=np.broadcast_to(
+        key[None, :, None, :].astype(np.float32), w.cache.k_pool.shape).copy())
+    q = rng.standard_normal((B, kr, hq, dh))
+    kn = np.broadcast_to(key, (B, kr, hkv, dh)).copy()
+    vn = rng.standard_normal((B, kr, hkv, dh))
+    o = so.attention_step(sh, cache, w.seq_ids, q, kn, vn)
+    for i, sid in enumerate(w.seq_ids):
+        _, vc = so.sequence_kv(cache, int(sid))
+        vals = np.concatenate([vc, vn[i]], axis=0)
+        L = vc.shape[0]
+        for r in range(kr):
+            for h in range(hq):
+                np.testing.assert_allclose(o[i, r, h], vals[:L + r + 1, h // sh.group].mean(axis=0),
+                                           rtol=1e-12, atol=1e-12)
+
+
+ALL_CHECKS = [check_bf16_decode_fixed_patterns, check_attention_step_matches_the_layer_trace,
+              check_attention_step_uniform_keys_closed_form,
+              check_lm_head_readout_hand_example, check_lm_head_readout_is_scale_invariant,
               check_one_task_is_the_single_task_path, check_tasks_are_isolated_and_permutable,
               check_recursive_k1_equals_parallel_fused,
               check_recursive_equals_stepwise_reconstruction,
@@ -598,7 +659,34 @@ def _readout_final_norm_ignored(orig):
     return f
 
 
+def _bf16_low_half(orig):
+    def f(arr, dtype_code):
+        a = np.asarray(arr)
+        if dtype_code == so.BF16:
+            return a.astype(np.uint32).view(np.float32).astype(np.float64)
+        return orig(arr, dtype_code)
+    return f
+
+
+def _attention_step_mask_off_by_one(orig):
+    def f(shape, cache, seq_ids, q, k_new, v_new):
+        kr = q.shape[1]
+        out = np.zeros_like(q, dtype=np.float64)
+        for i, sid in enumerate(np.asarray(seq_ids)):
+            kc, vc = so.sequence_kv(cache, int(sid))
+            L = kc.shape[0]
+            keys = np.concatenate([kc, k_new[i]], axis=0)
+            values = np.concatenate([vc, v_new[i]], axis=0)
+            # row r also sees new token r + 1 (one position into its future)
+            visible = np.arange(L + kr)[None, :] <= (L + np.arange(kr))[:, None] + 1
+            out[i] = so.attention(q[i], keys, values, visible, shape.group)
+        return out
+    return f
+
+
 MUTANTS = {
+    "bf16_decoded_from_low_half": (so, "to_f64", _bf16_low_half),
+    "attention_step_mask_off_by_one": (so, "attention_step", _attention_step_mask_off_by_one),
     "lm_readout_norm_before_pool": (so.Layer, "readout", _readout_norm_before_pool),
     "lm_readout_final_norm_ignored": (so.Layer, "readout", _readout_final_norm_ignored),
     "recursion_feeds_layer_input": (so, "classify_recursive",
