@@ -330,8 +330,13 @@ SP_API sp_status sp_attend(sp_stream stream, const sp_attn_dims *dims, int batch
  *  - A batch whose scratch (sp_attend_workspace_bytes) exceeds 32 MiB is
  *    rejected with SP_ERR_INVALID_ARG before any launch.
  *  - The first call on each device looks up the array's device address, with
- *    that device current, and caches it; make that first call before any
- *    stream capture.
+ *    that device current, and caches it.  With lazy module loading (CUDA's
+ *    default) that first call also loads the module holding the array, which
+ *    commits its 32 MiB on the device: make the first call at set-up time,
+ *    before any stream capture.  Later calls allocate nothing.  The cached
+ *    address does not survive cudaDeviceReset.
+ *  - Invalid dims or batch (those sp_attend_workspace_bytes rejects) return
+ *    SP_ERR_INVALID_ARG.
  *  - Every call shares the one array and leaves its contents behind: calls
  *    whose work overlaps on the GPU (other streams, other threads) race on it
  *    and must be serialised by the caller.  Nothing in it needs clearing: each

@@ -896,6 +896,7 @@ sp_status sp_attend(sp_stream stream, const sp_attn_dims *dm, int batch, const i
     if (out_dtype != SP_F32 && out_dtype != SP_BF16) return fail(SP_ERR_INVALID_ARG, "bad out_dtype");
     if (dm->split_tokens < 0 || dm->split_tokens % 64)
         return fail(SP_ERR_INVALID_ARG, "split_tokens must be a multiple of 64");
+    if (dm->max_seq_len < 0) return fail(SP_ERR_INVALID_ARG, "max_seq_len must be >= 0");
     if (batch < 1) return fail(SP_ERR_INVALID_ARG, "batch must be >= 1");
     if (!d_seq_lens || !d_q || !d_k_new || !d_v_new || !d_out || !d_workspace)
         return fail(SP_ERR_INVALID_ARG, "a required pointer is NULL");

@@ -14,7 +14,12 @@
 // GPU that loads the library holds it until the process exits.  Host code
 // cannot use the array's name as a device address, so the first call on each
 // device looks the address up with cudaGetSymbolAddress (with that device
-// current) and caches it; make that first call before any stream capture.
+// current) and caches it.  Under CUDA's lazy module loading that first call
+// also loads this file's module, which is when the array's memory is committed
+// on the device (an allocation, and possibly a synchronisation): make the first
+// call on each device at set-up time, before any stream capture and before the
+// decoding loop it must not disturb.  The cached address belongs to the
+// device's primary context; it is not valid across cudaDeviceReset.
 // All calls share the one array: calls whose work overlaps on the GPU (other
 // streams, other host threads) race on it and must be serialised by the
 // caller.  Nothing in it needs to start at zero: every partial the merge reads
@@ -63,9 +68,13 @@ sp_status sp_attend_static(sp_stream stream, const sp_attn_dims *dims, int batch
                            const float *d_q, const float *d_k_new, const float *d_v_new,
                            void *d_out, int out_dtype, int *d_status, int *d_gathered_pages) {
     const size_t need = sp_attend_workspace_bytes(dims, batch);
-    if (need == 0)
-        return sp_attend(stream, dims, batch, d_seq_ids, d_seq_lens, kv, d_q, d_k_new, d_v_new,
-                         d_out, out_dtype, nullptr, 0, d_status, d_gathered_pages);
+    if (need == 0) {
+        snprintf(g_msg, sizeof g_msg,
+                 "sp_attend_static: invalid attention dims or batch (heads, k_rows, "
+                 "max_seq_len or split_tokens out of range)");
+        sp::set_error_text(g_msg);
+        return SP_ERR_INVALID_ARG;
+    }
     if (need > kStaticScratchBytes) {
         snprintf(g_msg, sizeof g_msg,
                  "sp_attend_static: this batch needs %zu bytes of scratch, more than the "

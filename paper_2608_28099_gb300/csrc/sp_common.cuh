@@ -179,7 +179,7 @@ __device__ __forceinline__ SeqRef resolve_seq(const int *seq_ids, const int *seq
     int L = seq_lens[lens_by_batch ? b : sid];
     if (L < 0 || L > max_seq_len) {
         if (status) atomicOr(status, SP_DEV_BAD_LENGTH);
-        L = L < 0 ? 0 : max_seq_len;
+        L = L < 0 ? 0 : max(max_seq_len, 0);  // a negative bound never yields a negative length
     }
     r.sid = sid;
     r.len = L;

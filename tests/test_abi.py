@@ -126,3 +126,25 @@ def test_attend_rejects_misaligned_pools_on_host(lib):
                        out, sp.SP_F32, C.c_void_p(0xA00000), 1 << 20, None, None)
     assert st == sp.SP_ERR_INVALID_ARG
     assert "k_pool and v_pool" in sp.sp_last_error()
+
+
+def test_attend_rejects_negative_max_seq_len_on_host(lib):
+    # a negative bound would clamp lengths to a negative value on the device
+    kv = sp.sp_kv_cache(sp.SP_KV_PAGED, None, None, 0x600000, 0x700000, 0x500000, 16, 4, 4, 1)
+    dims = sp.sp_attn_dims(4, 2, 128, 4, sp.SP_BF16, -1, 0)
+    q, kn, vn, out = (C.c_void_p(0x100000 * i) for i in range(1, 5))
+    st = lib.sp_attend(None, C.byref(dims), 1, None, C.c_void_p(0x900000), C.byref(kv), q, kn, vn,
+                       out, sp.SP_F32, C.c_void_p(0xA00000), 1 << 20, None, None)
+    assert st == sp.SP_ERR_INVALID_ARG
+    assert "max_seq_len" in sp.sp_last_error()
+    assert lib.sp_attend_workspace_bytes(C.byref(dims), 1) == 0
+
+
+def test_attend_static_rejects_invalid_dims_on_host(lib):
+    kv = sp.sp_kv_cache(sp.SP_KV_PAGED, None, None, 0x600000, 0x700000, 0x500000, 16, 4, 4, 1)
+    dims = sp.sp_attn_dims(4, 2, 128, 4, sp.SP_BF16, -1, 0)
+    q, kn, vn, out = (C.c_void_p(0x100000 * i) for i in range(1, 5))
+    st = lib.sp_attend_static(None, C.byref(dims), 1, None, C.c_void_p(0x900000), C.byref(kv), q,
+                              kn, vn, out, sp.SP_F32, None, None)
+    assert st == sp.SP_ERR_INVALID_ARG
+    assert "invalid attention dims" in sp.sp_last_error()

@@ -72,3 +72,27 @@ def test_static_scratch_rejects_batches_that_do_not_fit():
                             torch.empty_like(q), sp.SP_F32)
     assert e.value.status == sp.SP_ERR_INVALID_ARG
     assert "static" in sp.sp_last_error()
+
+
+def test_static_scratch_calls_after_the_first_allocate_nothing():
+    torch = torch_dev()
+    ensure_built()
+    shape, cache, dims, q, kn, vn = _inputs(torch, [300, 1200, 5], 14)
+    out = torch.empty(q.shape, dtype=torch.float32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+
+    def call():
+        sp.sp_attend_static(torch.cuda.current_stream(), dims, q.shape[0], None, cache.seq_lens,
+                            cache.desc, q, kn, vn, out, sp.SP_F32, status)
+
+    call()  # the first call on the device may load the module holding the array
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    alloc0 = torch.cuda.memory_allocated()
+    for _ in range(3):
+        call()
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert torch.cuda.memory_allocated() == alloc0
+    assert free1 == free0
+    assert int(status.item()) == 0
