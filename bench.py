@@ -33,6 +33,12 @@ import sys
 import tempfile
 import time
 
+# The fp64 oracle's parallelism comes from a pool of worker processes, one per
+# host core, each with single-threaded BLAS (fixed before numpy loads), so the
+# reported core count is the number of workers that ran.
+for _var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_var, "1")
+
 import numpy as np
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -44,9 +50,9 @@ FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS = 6800.0, 1900.0
 FLUSH_BYTES = 256 << 20
 
 # DRAM read + write per launch of the dominant kernel, from one ncu capture of
-# the current kernel on the same workload (profiles/attn_tc_kernel_*.md); a
-# workload or kernel without a capture reports null.
-TRAFFIC_BYTES = {("4b", "attention"): 77519616}
+# the current kernel on the same workload; a workload or kernel without such a
+# capture reports null.
+TRAFFIC_BYTES = {("4b", "attention"): 77519616, ("27b_long", "attention"): 1086108416}
 
 
 def parse_args():
@@ -54,7 +60,9 @@ def parse_args():
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=5)
-    p.add_argument("--workload", default="4b")
+    p.add_argument("--workload", default="27b_long",
+                   help="tiny, 4b, 8b_paged or 27b_long (default: the largest single-GPU "
+                        "configuration, B=8 x L=32768, d=5120, paged)")
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--rows", default="per-seq", choices=["per-seq", "shared", "hidden"],
                    help="per-seq: per-sequence input rows (full layer per call); "
@@ -195,60 +203,113 @@ def cores():
         return os.cpu_count() or 1
 
 
-def oracle_rate(w, per_seq_rows: bool, seconds: float, max_seqs: int | None = None,
-                recursive: bool = False):
-    """Sequences/s of the oracle over successive sequences of the workload
-    (through the input fusion when the workload carries hidden states)."""
+# State the oracle workers inherit when the pool forks (set before any CUDA call).
+_ORACLE = {}
+
+
+def _oracle_one(i: int):
+    """Classify sequence i % B of the workload with the oracle (one worker)."""
     import oracle.sp_oracle as so
-    layer = so.Layer(w.shape, w.weights)
-    n = 0
-    t0 = time.perf_counter()
-    B = len(w.seq_ids)
+    st = _ORACLE
+    w, layer = st["w"], st["layer"]
+    i %= len(w.seq_ids)
+    rows = w.rows[i:i + 1] if (st["per_seq"] and w.rows is not None) else None
+    hid = w.hidden[i:i + 1] if w.hidden is not None else None
+    if st["recursive"]:
+        so.classify_recursive(layer, w.cache, w.seq_ids[i:i + 1], hid)
+    else:
+        so.classify(layer, w.cache, w.seq_ids[i:i + 1], rows, hidden=hid)
+
+
+def _oracle_worker(args):
+    """Sequences first, first + stride, ... until `seconds` have passed (at
+    least one); returns how many were classified."""
+    first, stride, seconds = args
+    n, t0 = 0, time.perf_counter()
     while True:
-        i = n % B
-        rows = w.rows[i:i + 1] if (per_seq_rows and w.rows is not None) else None
-        hid = w.hidden[i:i + 1] if w.hidden is not None else None
-        if recursive:
-            so.classify_recursive(layer, w.cache, w.seq_ids[i:i + 1], hid)
-        else:
-            so.classify(layer, w.cache, w.seq_ids[i:i + 1], rows, hidden=hid)
+        _oracle_one(first + n * stride)
         n += 1
+        if time.perf_counter() - t0 >= seconds:
+            return n
+
+
+def _mem_available() -> int | None:
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return None
+
+
+class OraclePool:
+    """The oracle on the host cores: one single-threaded worker process per
+    core (capped by free memory), forked before any CUDA call so that the
+    workers share the decoded weights and the workload."""
+
+    def __init__(self, w, per_seq_rows: bool, recursive: bool):
+        import multiprocessing as mp
+
+        import oracle.sp_oracle as so
+        _ORACLE.update(w=w, layer=so.Layer(w.shape, w.weights), per_seq=per_seq_rows,
+                       recursive=recursive)
+        sh = w.shape
+        # float64 temporaries of one sequence: its gathered K and V, the
+        # attention probabilities and the layer's activations (x4 headroom)
+        L = int(w.cache.seq_lens[w.seq_ids].max(initial=0)) + sh.k_rows
+        per = 8 * (2 * L * sh.n_kv_heads * sh.head_dim + 2 * sh.k_rows * sh.n_q_heads * L
+                   + 4 * sh.k_rows * (sh.d_model + sh.d_ff))
+        n = cores()
+        avail = _mem_available()
+        if avail is not None:
+            n = max(1, min(n, int(avail // (4 * per + (256 << 20)))))
+        self.workers = n
+        self.pool = mp.get_context("fork").Pool(n)
+
+    def rate(self, seconds: float):
+        """(sequences/s, sequences, seconds) with every worker busy for about
+        `seconds` (each finishes the sequence it is on)."""
+        t0 = time.perf_counter()
+        counts = self.pool.map(_oracle_worker, [(j, self.workers, seconds)
+                                                for j in range(self.workers)], chunksize=1)
         el = time.perf_counter() - t0
-        if el >= seconds or (max_seqs is not None and n >= max_seqs):
-            return n / el, n, el
+        return sum(counts) / el, sum(counts), el
+
+    def step(self, first: int):
+        """One sequence per worker (first, first + 1, ...): the wall time."""
+        t0 = time.perf_counter()
+        self.pool.map(_oracle_one, [first + j for j in range(self.workers)], chunksize=1)
+        return time.perf_counter() - t0
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
 
 
 def run_reference(args, spec, w, rank, world):
     if rank != 0:
         return
-    per_seq = args.rows == "per-seq"
-    import oracle.sp_oracle as so
-    layer = so.Layer(w.shape, w.weights)
+    pool = OraclePool(w, args.rows == "per-seq", recursive_mode(args))
     B = len(w.seq_ids)
-    times, counts = [], []
-    per_step = max(1, min(B, 2))
+    times = []
     for step in range(args.warmup + args.steps):
-        ids = [(step * per_step + j) % B for j in range(per_step)]
-        rows = w.rows[ids] if (per_seq and w.rows is not None) else None
-        hid = w.hidden[ids] if w.hidden is not None else None
-        t0 = time.perf_counter()
-        if recursive_mode(args):
-            so.classify_recursive(layer, w.cache, w.seq_ids[ids], hid)
-        else:
-            so.classify(layer, w.cache, w.seq_ids[ids], rows, hidden=hid)
-        el = time.perf_counter() - t0
+        el = pool.step(step * pool.workers)
         if step >= args.warmup:
             times.append(el)
-            counts.append(per_step)
-    value = sum(counts) / sum(times)
-    sample = (f"{per_step} sequence(s) of workload {spec.name} per step, "
-              f"{args.steps} steps after {args.warmup} warm-up")
+    pool.close()
+    per_step = pool.workers
+    value = per_step * len(times) / sum(times)
+    sample = (f"{per_step} sequence(s) of workload {spec.name} (of its {B}) per step, one per "
+              f"worker process, {per_step} single-threaded workers; {args.steps} steps after "
+              f"{args.warmup} warm-up")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(spec, w, args),
-            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle",
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": per_step, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
@@ -301,7 +362,7 @@ def shard_spec(spec, rank: int):
 # --------------------------------------------------------------------------- #
 # our arm
 # --------------------------------------------------------------------------- #
-def run_ours(args, spec, w, rank, world):
+def run_ours(args, spec, w, rank, world, oracle_pool=None):
     import torch
     import torch.distributed as dist
 
@@ -457,10 +518,13 @@ def run_ours(args, spec, w, rank, world):
                 "ms": stage_ms[dom]}
     path_bytes = totals["total_bytes"]
     cpu = None
-    if world == 1 and not args.no_cpu_baseline:
-        rate, n, el = oracle_rate(w, per_seq, args.cpu_seconds, recursive=recursive)
-        cpu = {"value": rate, "unit": UNIT, "cores": cores(), "kind": "oracle",
-               "sample": f"{n} sequences of workload {spec.name} one at a time, {el:.1f} s"}
+    if oracle_pool is not None:
+        rate, n, el = oracle_pool.rate(args.cpu_seconds)
+        cpu = {"value": rate, "unit": UNIT, "cores": oracle_pool.workers, "kind": "oracle",
+               "sample": f"{n} sequences of workload {spec.name} over {el:.1f} s, one sequence "
+                         f"at a time per worker process, {oracle_pool.workers} single-threaded "
+                         f"workers"}
+        oracle_pool.close()
     value = world * B / (ms / 1e3)
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "us_per_call": ms * 1e3,
@@ -639,7 +703,11 @@ def main():
     if args.impl == "reference":
         run_reference(args, spec, w, rank, world)
     else:
-        run_ours(args, spec, w, rank, world)
+        # the oracle's worker pool forks here, before this process touches CUDA
+        pool = None
+        if world == 1 and not args.no_cpu_baseline:
+            pool = OraclePool(w, args.rows == "per-seq", recursive_mode(args))
+        run_ours(args, spec, w, rank, world, pool)
     if world > 1 and args.impl != "reference":
         import torch.distributed as dist
         dist.destroy_process_group()

@@ -3,6 +3,8 @@ memory (a monitor on the decoding hot path must not call cudaMalloc, which can
 synchronise the device; some serving frameworks give a library no device memory
 of its own).  It must give the same result as sp_attend with a caller-provided
 workspace, call after call, although every call reuses one static array."""
+import gc
+
 import numpy as np
 import pytest
 
@@ -87,12 +89,14 @@ def test_static_scratch_calls_after_the_first_allocate_nothing():
 
     call()  # the first call on the device may load the module holding the array
     torch.cuda.synchronize()
+    gc.collect()  # tensors of earlier tests must not be freed inside the window
     free0, _ = torch.cuda.mem_get_info()
     alloc0 = torch.cuda.memory_allocated()
     for _ in range(3):
         call()
     torch.cuda.synchronize()
     free1, _ = torch.cuda.mem_get_info()
-    assert torch.cuda.memory_allocated() == alloc0
-    assert free1 == free0
+    # neither torch's allocator nor the driver gave out memory for these calls
+    assert torch.cuda.memory_allocated() <= alloc0
+    assert free1 >= free0
     assert int(status.item()) == 0
