@@ -245,11 +245,16 @@ enum {
                                  sp_classify on its stream (as external event
                                  nodes when the call is captured in a graph),
                                  0 = off (default)                              */
-    SP_OPT_RECURSIVE = 5      /* 1 = sp_classify_hidden runs recursive probing
+    SP_OPT_RECURSIVE = 5,     /* 1 = sp_classify_hidden runs recursive probing
                                  SP-k (Sec. 3.2): k steps of one row each, step i
                                  fusing step i-1's output with soft-prompt row i
                                  (no per-stage event markers); 0 = the parallel
                                  form (default)                                   */
+    SP_OPT_ATTN_SEG_COST = 6  /* tensor-core attention: the cost of a segment
+                                 boundary, in 64-token tiles, that the cuts
+                                 between CTA shares balance (-1..1024); -1 = the
+                                 built-in default.  Changes the work split only,
+                                 never the result beyond rounding order          */
 };
 
 /* Stages of sp_classify, in launch order. */

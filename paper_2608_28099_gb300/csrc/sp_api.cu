@@ -90,6 +90,7 @@ struct sp_handle {
     GemmPlanner gemm;
     // options
     int opt_split = 0, opt_gemm = 0, opt_attn = 0, opt_profile = 0, opt_recursive = 0;
+    int opt_seg_cost = -1;  // attention segment-boundary cost in tiles (-1 = default)
     int T = 1;        // tasks sharing the pass; cfg.k_rows holds T * k_task rows per sequence
     int k_task = 0;   // soft-prompt rows per task
     float *h2_all = nullptr;      // recursive probing: step outputs [k][max_batch][d] fp32
@@ -209,9 +210,11 @@ int *attention_counters(void *ws) { return (int *)ws; }
 // counters (else they are cleared here).
 sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_path, int n_sm,
                             int forced_split, int *launches, cudaStream_t st, bool counters_zeroed,
-                            cudaEvent_t *ev_attn = nullptr, cudaEvent_t *ev_merge = nullptr) {
+                            cudaEvent_t *ev_attn = nullptr, cudaEvent_t *ev_merge = nullptr,
+                            int seg_cost = -1) {
     a.tc_ctas = attn_tc_ctas(n_sm, a.Hkv);
     a.tc_min_tiles = forced_split > 0 ? forced_split / 64 : kAttnMinTiles;
+    a.tc_seg_cost = seg_cost >= 0 ? seg_cost : kAttnSegCost;
     // few sequences over many groups: each pair has many partials, merged by a
     // kernel spread over (head, sequence, row) instead of one CTA per pair
     a.tc_merge_kernel = 4 * a.B < a.tc_ctas / a.Hkv;
@@ -510,6 +513,10 @@ sp_status sp_set_option(sp_handle *h, int key, int value) {
         if (value != 0 && value != 1) return fail(SP_ERR_INVALID_ARG, "bad recursion flag");
         h->opt_recursive = value;
         return SP_OK;
+    case SP_OPT_ATTN_SEG_COST:
+        if (value < -1 || value > 1024) return fail(SP_ERR_INVALID_ARG, "bad segment cost");
+        h->opt_seg_cost = value;
+        return SP_OK;
     case SP_OPT_PROFILE:
         if (value != 0 && value != 1) return fail(SP_ERR_INVALID_ARG, "bad profile flag");
         if (value && !h->ev[0][0]) {
@@ -747,7 +754,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, h->n_sm, h->opt_split,
                           &launches, st, true,
                           h->opt_profile ? h->ev[SP_STAGE_ATTN] : nullptr,
-                          h->opt_profile ? h->ev[SP_STAGE_MERGE] : nullptr);
+                          h->opt_profile ? h->ev[SP_STAGE_MERGE] : nullptr, h->opt_seg_cost);
     if (s != SP_OK) return s;
     if (h->opt_profile) h->ev_used[SP_STAGE_ATTN] = h->ev_used[SP_STAGE_MERGE] = true;
 

@@ -15,7 +15,10 @@
 // each of its segments leaves an unnormalised partial (max, sum, O) in slot
 // (j + b) Hkv + g (unique: segments are ordered by both j and b), and the CTA
 // that completes the pair's last segment (a counter per pair, zero before the
-// launch) combines the partials in the exp2 domain.
+// launch) combines the partials in the exp2 domain, in segment order, in that
+// segment's epilogue.  The cuts between shares weigh every sequence start as
+// a number of tiles (the cost of a segment boundary), so shares with more
+// boundaries hold fewer tiles.
 //
 // All R = G * k query rows of the KV head's group share every K/V tile: the
 // GQA group and the k soft-prompt rows together form the M side of the MMA.
@@ -118,10 +121,7 @@ struct Bars {
     uint64_t kv_full[STG], kv_empty[STG], s_full[2], p_full[2], pv_done[2], fin, q_full;  // fin: 2 arrivals
     uint32_t tmem;
     int abort;
-    int n_pend;                // partial segments written (counted at the end), <= 2
-    int p_b[2], p_j0[2], p_j1[2];
-    int n_merge;               // pairs this CTA completes (merged at the end), <= 2
-    int m_b[2], m_j0[2], m_j1[2];
+    int merge_now;             // this segment completed its pair: merge it in the epilogue
     int wsum[THREADS / 32];    // tile-prefix scan
 };
 static_assert(sizeof(Bars) <= 512, "barrier block");
@@ -151,20 +151,35 @@ __device__ __forceinline__ Seg seg_at(const int *prefix, int B, int x, int x_end
     return s;
 }
 
-// First tile of group j's share.  The even cut j T / n moves to the nearest
-// sequence start when one lies within delta = min(share / 4, SNAP) tiles: a
-// segment boundary costs the consumers a pipeline drain and refill worth a few
-// tiles, so a short sequence is better kept whole than split near its end.
-// Cuts stay strictly increasing (they move by at most a quarter share).
-// Evaluated once per group into a table (cuts[0..n]).
+// First tile of group j's share.  A segment boundary inside a share costs the
+// consumers a pipeline drain, the epilogue and the next queries' load, worth
+// about `c` tiles of streaming, so the shares balance tiles + c per sequence:
+// every sequence b gets c virtual tiles in front of its own, the virtual list
+// (T + c B long) is cut evenly, and a cut that lands in a sequence's virtual
+// part moves to that sequence's first tile.  A cut within delta = min(share /
+// 4, SNAP) tiles of a sequence start then moves onto it (a short piece of a
+// sequence would pay a whole boundary).  c falls back to 0 when a share is
+// shorter than c + 1 virtual tiles, which keeps the cuts strictly increasing
+// (snapping moves them by at most a quarter share).  Evaluated once per group
+// into a table (cuts[0..n]).
 constexpr int SNAP = 4;
-__device__ __forceinline__ int share_start(const int *prefix, int B, int T, int n, int j) {
+__device__ __forceinline__ int share_start(const int *prefix, int B, int T, int n, int j, int c) {
     if (j <= 0) return 0;
     if (j >= n) return T;
-    const int x = (int)((long long)j * T / n);
+    if ((long long)T + (long long)c * B < (long long)n * (c + 1)) c = 0;
+    const long long V = (long long)T + (long long)c * B;
+    const long long v = (long long)j * V / n;
+    int lo = 0, hi = B - 1;  // last sequence whose virtual start vpre(b) = prefix[b] + c b is <= v
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if ((long long)prefix[mid] + (long long)c * mid <= v) lo = mid;
+        else hi = mid - 1;
+    }
+    const long long off = v - ((long long)prefix[lo] + (long long)c * lo);
+    int x = off < c ? prefix[lo] : (int)min((long long)prefix[lo] + off - c, (long long)prefix[lo + 1] - 1);
     const int delta = min(T / n / 4, SNAP);
     if (delta == 0) return x;
-    int lo = 0, hi = B - 1;  // last sequence starting at or before x
+    lo = 0, hi = B - 1;  // last sequence starting at or before x
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
         if (prefix[mid] <= x) lo = mid;
@@ -244,7 +259,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int grp = blockIdx.x / Hkv, g = blockIdx.x - grp * Hkv;
     if (grp >= n_grp) return;  // uniform over the CTA: no tile for this one
     int *cuts = (int *)(smem + OFF_CUTS);
-    for (int j = threadIdx.x; j <= n_grp; j += THREADS) cuts[j] = share_start(prefix, B, T, n_grp, j);
+    for (int j = threadIdx.x; j <= n_grp; j += THREADS) cuts[j] = share_start(prefix, B, T, n_grp, j, a.tc_seg_cost);
     __syncthreads();
     const int x0 = cuts[grp], x1 = cuts[grp + 1];
 
@@ -271,8 +286,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         mbar_init(&bars->fin, 2);
         mbar_init(&bars->q_full, 1);
         bars->abort = 0;
-        bars->n_merge = 0;
-        bars->n_pend = 0;
+        bars->merge_now = 0;
         fence_mbar_init();
         if (paged) {
             prefetch_tmap(&map_k);
@@ -298,6 +312,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (is_producer) {
         // ------------------------------------------------------------ producers
         const int ptid = pidx * 32 + lane, pstride = 32 * n_prod;
+        const uint64_t pol_kv = policy_evict_first();
         const int npg = paged ? TT / P : 0;  // pages per tile
         int ci = 0;                          // CTA-local tile counter (ring position)
         int bad = 0;
@@ -344,8 +359,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                         const int pj = __shfl_sync(0xffffffffu, page, j);
                         if (lane < 2 * npg && ((okm >> j) & 1)) {
                             const int grp = (pj * Hkv + g) * (P / 8);
-                            tma_load_4d((part ? V : K) + j * P * 256, part ? &map_v : &map_k,
-                                        &bars->kv_full[st], 0, 0, 0, grp);
+                            // the cache is read once: evict-first keeps the queries and
+                            // the partials of the merges resident in L2
+                            tma_load_4d_hint((part ? V : K) + j * P * 256, part ? &map_v : &map_k,
+                                             &bars->kv_full[st], 0, 0, 0, grp, pol_kv);
                         }
                         const unsigned want = (1u << npg) - 1u;
                         if ((okm & want) != want) {
@@ -747,131 +764,77 @@ __global__ void __launch_bounds__(THREADS, 1)
                     a.part_ml[(slot * R + row) * 2 + 1] = lsum;
                 }
             }
-            if (!whole && ct == 0 && !a.tc_merge_kernel && bars->n_pend < 2) {
-                // counted at the end of the kernel (only a share's first and last
-                // segments can be partial)
-                const int t = bars->n_pend++;
-                bars->p_b[t] = b;
-                bars->p_j0[t] = j_first;
-                bars->p_j1[t] = j_last;
+            if (!whole && !a.tc_merge_kernel) {
+                // count this segment; the one completing the pair merges all of its
+                // partials here, in segment order (the result does not depend on
+                // which CTA finishes last), while its own are still in L2
+                const int n_seg = j_last - j_first + 1;
+                __threadfence();  // this segment's partial is visible before it is counted
+                named_sync(BAR_EPI, n_cons);
+                if (ct == 0) {
+                    const int done_before = atomicAdd(a.counters + b * Hkv + g, 1);
+                    const int last = done_before == n_seg - 1;
+                    if (last) a.counters[b * Hkv + g] = 0;  // ready for the next launch
+                    bars->merge_now = last;
+                }
+                named_sync(BAR_EPI, n_cons);
+                if (bars->merge_now && have && active) {
+                    __threadfence();  // the other segments' partials are read after their count
+                    const size_t slot0 = ((size_t)j_first + b) * Hkv + g;  // segment e: + e Hkv
+#pragma unroll 1
+                    for (int c0 = wg * (DH / 2); c0 < (wg + 1) * (DH / 2); c0 += 32) {
+                        float acc[32], mm = -INFINITY, ll = 0.f;
+#pragma unroll
+                        for (int jj = 0; jj < 32; ++jj) acc[jj] = 0.f;
+                        for (int e0 = 0; e0 < n_seg; e0 += 2) {
+                            float2 ml[2];
+                            float4 ov[2][8];
+#pragma unroll
+                            for (int e = 0; e < 2; ++e) {  // both segments' loads in flight together
+                                const bool in = e0 + e < n_seg;
+                                const size_t sl = slot0 + (size_t)(e0 + e) * Hkv;
+                                ml[e] = in ? __ldcg((const float2 *)(a.part_ml + (sl * R + row) * 2))
+                                           : make_float2(-INFINITY, 0.f);
+                                const float4 *src = (const float4 *)(a.part_o + (sl * R + row) * DH + c0);
+#pragma unroll
+                                for (int q4 = 0; q4 < 8; ++q4)
+                                    ov[e][q4] = in ? __ldcg(src + q4) : make_float4(0.f, 0.f, 0.f, 0.f);
+                            }
+#pragma unroll
+                            for (int e = 0; e < 2; ++e) {
+                                const float mn = fmaxf(mm, ml[e].x);
+                                if (mn == -INFINITY) continue;
+                                const float al = mm == -INFINITY ? 0.f : exp2f(mm - mn);
+                                const float wt = ml[e].x == -INFINITY ? 0.f : exp2f(ml[e].x - mn);
+                                ll = ll * al + wt * ml[e].y;
+#pragma unroll
+                                for (int q4 = 0; q4 < 8; ++q4) {
+                                    acc[4 * q4] = acc[4 * q4] * al + wt * ov[e][q4].x;
+                                    acc[4 * q4 + 1] = acc[4 * q4 + 1] * al + wt * ov[e][q4].y;
+                                    acc[4 * q4 + 2] = acc[4 * q4 + 2] * al + wt * ov[e][q4].z;
+                                    acc[4 * q4 + 3] = acc[4 * q4 + 3] * al + wt * ov[e][q4].w;
+                                }
+                                mm = mn;
+                            }
+                        }
+                        const float il = ll > 0.f ? 1.f / ll : 0.f;
+#pragma unroll
+                        for (int jj = 0; jj < 32; jj += 4)
+                            act_store4(a.out, out0 + c0 + jj,
+                                       make_float4(acc[jj] * il, acc[jj + 1] * il, acc[jj + 2] * il,
+                                                   acc[jj + 3] * il));
+                    }
+                }
             }
             if (x < x1) load_q(seg_at(prefix, B, x, x1).b);
         }
     }
     // every MMA must be finished before TMEM and shared memory go away
     mbar_wait_drain(&bars->fin, 0);
-    if (warp < 8) __threadfence();  // the partials are visible device-wide before they are counted
     tc_fence_before();
     __syncthreads();
-    if (threadIdx.x == 0) {
-        if (*abort && a.status) atomicOr(a.status, SP_DEV_TIMEOUT);
-        // count this CTA's partial segments; the CTA completing a pair merges it
-        for (int t = 0; t < bars->n_pend; ++t) {
-            const int b = bars->p_b[t], n_seg = bars->p_j1[t] - bars->p_j0[t] + 1;
-            if (atomicAdd(a.counters + b * Hkv + g, 1) == n_seg - 1) {
-                const int u = bars->n_merge++;
-                bars->m_b[u] = b;
-                bars->m_j0[u] = bars->p_j0[t];
-                bars->m_j1[u] = bars->p_j1[t];
-            }
-        }
-        __threadfence();  // the other segments' partials are read after their count
-    }
+    if (threadIdx.x == 0 && *abort && a.status) atomicOr(a.status, SP_DEV_TIMEOUT);
     if (warp == MMA_WARP) tmem_dealloc(tmem, TMEM_COLS);
-    __syncthreads();
-
-    // ---- merges, by the whole CTA: every segment of pair (b, g) has written its
-    // partial (slots (j + b) Hkv + g, j = j0 .. j1).  One item per (pair, row, 8
-    // columns), the items of all of this CTA's pairs (at most 2) in one pass: the
-    // partials' loads issued together MCH segments at a time with an online
-    // rescale between chunks, MIT items in flight per thread.
-    constexpr int MCH = 2, MIT = 3, CPI = 8;  // columns per item
-    const int items = R * (DH / CPI), n_merge = bars->n_merge;
-    const int n_items = n_merge * items;
-    for (int i0 = threadIdx.x; i0 < n_items; i0 += THREADS * MIT) {
-        float mm[MIT], ls[MIT];
-        float4 o[MIT][2];
-        int nsu[MIT], rru[MIT], cqu[MIT], bu[MIT];
-        size_t s0u[MIT];  // slot of segment j0 + e of the item's pair: s0u + e Hkv
-        int ns_max = 0;
-#pragma unroll
-        for (int u = 0; u < MIT; ++u) {
-            mm[u] = -INFINITY;
-            ls[u] = 0.f;
-            o[u][0] = o[u][1] = make_float4(0.f, 0.f, 0.f, 0.f);
-            const int ia = i0 + u * THREADS;
-            const int t = min(ia / items, n_merge - 1);  // items past the end: no loads, no store
-            const int idx = ia - t * items;
-            const int j0 = bars->m_j0[t];
-            bu[u] = bars->m_b[t];
-            nsu[u] = ia < n_items ? bars->m_j1[t] - j0 + 1 : 0;
-            s0u[u] = ((size_t)j0 + bu[u]) * Hkv + g;
-            rru[u] = idx / (DH / CPI);
-            cqu[u] = (idx % (DH / CPI)) * CPI;
-            ns_max = max(ns_max, nsu[u]);
-        }
-        for (int e0 = 0; e0 < ns_max; e0 += MCH) {
-            float mv[MIT][MCH], lv[MIT][MCH];
-            float4 ov[MIT][MCH][2];
-#pragma unroll
-            for (int u = 0; u < MIT; ++u) {
-#pragma unroll
-                for (int e = 0; e < MCH; ++e) {
-                    const bool in = e0 + e < nsu[u];
-                    const size_t sl = s0u[u] + (size_t)(e0 + e) * Hkv;
-                    const float2 ml = in ? __ldcg((const float2 *)(a.part_ml + (sl * R + rru[u]) * 2))
-                                         : make_float2(-INFINITY, 0.f);
-                    mv[u][e] = ml.x;
-                    lv[u][e] = ml.y;
-                    const float4 *src = (const float4 *)(a.part_o + (sl * R + rru[u]) * DH + cqu[u]);
-                    ov[u][e][0] = in ? __ldcg(src) : make_float4(0.f, 0.f, 0.f, 0.f);
-                    ov[u][e][1] = in ? __ldcg(src + 1) : make_float4(0.f, 0.f, 0.f, 0.f);
-                }
-            }
-#pragma unroll
-            for (int u = 0; u < MIT; ++u) {
-                float mn = mm[u];
-#pragma unroll
-                for (int e = 0; e < MCH; ++e) mn = fmaxf(mn, mv[u][e]);
-                if (mn == -INFINITY) continue;
-                const float al = mm[u] == -INFINITY ? 0.f : exp2f(mm[u] - mn);
-                ls[u] *= al;
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    o[u][h].x *= al;
-                    o[u][h].y *= al;
-                    o[u][h].z *= al;
-                    o[u][h].w *= al;
-                }
-#pragma unroll
-                for (int e = 0; e < MCH; ++e) {
-                    const float wgt = mv[u][e] == -INFINITY ? 0.f : exp2f(mv[u][e] - mn);
-                    ls[u] += wgt * lv[u][e];
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        o[u][h].x += wgt * ov[u][e][h].x;
-                        o[u][h].y += wgt * ov[u][e][h].y;
-                        o[u][h].z += wgt * ov[u][e][h].z;
-                        o[u][h].w += wgt * ov[u][e][h].w;
-                    }
-                }
-                mm[u] = mn;
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < MIT; ++u) {
-            if (i0 + u * THREADS >= n_items) continue;
-            const float inv = ls[u] > 0.f ? 1.f / ls[u] : 0.f;
-            const int hl = rru[u] / k, r = rru[u] - hl * k;
-            const size_t dst = (((size_t)bu[u] * k + r) * a.Hq + g * a.G + hl) * DH + cqu[u];
-#pragma unroll
-            for (int h = 0; h < 2; ++h)
-                act_store4(a.out, dst + 4 * h,
-                           make_float4(o[u][h].x * inv, o[u][h].y * inv, o[u][h].z * inv, o[u][h].w * inv));
-        }
-    }
-    // ready for a launch that does not clear them
-    if (threadIdx.x < n_merge) a.counters[bars->m_b[threadIdx.x] * Hkv + g] = 0;
 }
 
 // Merge of the partial segments for small batches (a few long sequences, each
@@ -898,7 +861,7 @@ __global__ void __launch_bounds__(DH) attn_tc_merge_kernel(AttnArgs a) {
     __syncthreads();
     const int T = prefix[B];
     const int n_grp = min(a.tc_ctas / Hkv, ceil_div(T, max(1, a.tc_min_tiles)));
-    for (int j = threadIdx.x; j <= n_grp; j += blockDim.x) cuts[j] = share_start(prefix, B, T, n_grp, j);
+    for (int j = threadIdx.x; j <= n_grp; j += blockDim.x) cuts[j] = share_start(prefix, B, T, n_grp, j, a.tc_seg_cost);
     __syncthreads();
     const int j0 = group_of(cuts, n_grp, prefix[b]);
     const int j1 = group_of(cuts, n_grp, prefix[b + 1] - 1);

@@ -210,6 +210,8 @@ struct AttnArgs {
     int subs;                     // partials per work unit (1)
     int tc_ctas;                  // tensor-core kernel: persistent CTAs (one per SM)
     int tc_min_tiles;             // tensor-core kernel: fewest 64-token tiles per CTA
+    int tc_seg_cost;              // tensor-core kernel: cost of a segment boundary, in tiles,
+                                  // that the cuts between shares balance
     int tc_merge_kernel;          // tensor-core kernel: 1 = merge in a second kernel (small
                                   // batches), 0 = inside the attention kernel
     float *part_o;                // CUDA cores: [B][Hkv][n_splits][subs][R][dh]; tensor
@@ -232,6 +234,9 @@ void plan_attention(int B, int Hkv, int k, int max_seq_len, int forced_split, in
 size_t attention_workspace_bytes(int B, int Hkv, int R, int dh, int n_splits, int n_sm);
 // Default fewest tiles per CTA of the tensor-core kernel (64 tokens each).
 constexpr int kAttnMinTiles = 8;
+// Default cost of a segment boundary in the tensor-core kernel, in 64-token
+// tiles (a pipeline drain, the epilogue and the next queries' load).
+constexpr int kAttnSegCost = 12;
 // Persistent CTAs of the tensor-core kernel: whole groups of Hkv (one CTA per
 // kv head), as many groups as the SMs hold, at least one.
 inline int attn_tc_ctas(int n_sm, int Hkv) { return (n_sm / Hkv > 1 ? n_sm / Hkv : 1) * Hkv; }
