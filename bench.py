@@ -52,7 +52,7 @@ FLUSH_BYTES = 256 << 20
 # DRAM read + write per launch of the dominant kernel, from one ncu capture of
 # the current kernel on the same workload; a workload or kernel without such a
 # capture reports null.
-TRAFFIC_BYTES = {("4b", "attention"): 77519616, ("27b_long", "attention"): 1086108416}
+TRAFFIC_BYTES = {}
 
 
 def parse_args():

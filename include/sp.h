@@ -250,11 +250,18 @@ enum {
                                  fusing step i-1's output with soft-prompt row i
                                  (no per-stage event markers); 0 = the parallel
                                  form (default)                                   */
-    SP_OPT_ATTN_SEG_COST = 6  /* tensor-core attention: the cost of a segment
+    SP_OPT_ATTN_SEG_COST = 6, /* tensor-core attention: the cost of a segment
                                  boundary, in 64-token tiles, that the cuts
                                  between CTA shares balance (-1..1024); -1 = the
                                  built-in default.  Changes the work split only,
                                  never the result beyond rounding order          */
+    SP_OPT_ACT_PRECISION = 7  /* activations fed to the tensor-core MLP
+                                 projections (gate/up and down): 0 = automatic
+                                 (plain bf16 when pool is SP_POOL_MEAN and at
+                                 least 8 rows per task are pooled, else bf16
+                                 hi + lo planes, ~16 mantissa bits), 1 = hi + lo
+                                 always, 2 = plain bf16 always.  The Q/K/V and
+                                 output projections always take hi + lo        */
 };
 
 /* Stages of sp_classify, in launch order. */

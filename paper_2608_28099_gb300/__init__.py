@@ -22,6 +22,7 @@ SP_DEV_BAD_SEQ_ID, SP_DEV_BAD_LENGTH, SP_DEV_BAD_PAGE = 1, 2, 4
 SP_OPT_SPLIT_TOKENS, SP_OPT_GEMM_PATH, SP_OPT_ATTN_PATH, SP_OPT_PROFILE = 1, 2, 3, 4
 SP_OPT_RECURSIVE = 5
 SP_OPT_ATTN_SEG_COST = 6
+SP_OPT_ACT_PRECISION = 7
 STAGES = ["input_norm", "qkv", "rope", "attention", "merge", "o_proj", "post_norm", "gate_up",
           "swiglu", "down", "readout", "fusion"]
 

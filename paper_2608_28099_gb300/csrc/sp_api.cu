@@ -91,6 +91,7 @@ struct sp_handle {
     // options
     int opt_split = 0, opt_gemm = 0, opt_attn = 0, opt_profile = 0, opt_recursive = 0;
     int opt_seg_cost = -1;  // attention segment-boundary cost in tiles (-1 = default)
+    int opt_prec = 0;       // activation precision of the MLP inputs (SP_OPT_ACT_PRECISION)
     int T = 1;        // tasks sharing the pass; cfg.k_rows holds T * k_task rows per sequence
     int k_task = 0;   // soft-prompt rows per task
     float *h2_all = nullptr;      // recursive probing: step outputs [k][max_batch][d] fp32
@@ -513,6 +514,10 @@ sp_status sp_set_option(sp_handle *h, int key, int value) {
         if (value != 0 && value != 1) return fail(SP_ERR_INVALID_ARG, "bad recursion flag");
         h->opt_recursive = value;
         return SP_OK;
+    case SP_OPT_ACT_PRECISION:
+        if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad activation precision");
+        h->opt_prec = value;
+        return SP_OK;
     case SP_OPT_ATTN_SEG_COST:
         if (value < -1 || value > 1024) return fail(SP_ERR_INVALID_ARG, "bad segment cost");
         h->opt_seg_cost = value;
@@ -679,6 +684,12 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     const bool tc_gu = h->gemm.use_tc(h->w_gu, h->n, h->opt_gemm);
     const bool tc_down = h->gemm.use_tc(h->w_down, h->a, h->opt_gemm);
     int ns = 1;
+    // The MLP inputs (the post-norm n and the SwiGLU output a) go to the tensor
+    // cores as plain bf16 when the head averages at least 8 rows per pooled
+    // state (their rounding errors average out in the mean; the measured budget
+    // is in the design notes), else as hi + lo planes.  The Q/K/V and output
+    // projections always take hi + lo.
+    const bool mlp_lo = h->opt_prec == 1 || (h->opt_prec == 0 && !(c.pool == SP_POOL_MEAN && h->k_task >= 8));
 
     // a1-a2: pre-norm, Q/K/V projection, rotation at positions L_b + r
     PartIn yqkv = {h->qkv_shared, 1, 0};
@@ -768,21 +779,21 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     if (s != SP_OK) return fail(s, "output projection launch failed");
     mark(SP_STAGE_POST_NORM, 0);
     SP_CUDA(launch_residual_norm(x_bf16, PartIn{h->y, ns, (size_t)M * d}, x, row_mod, h->g_post,
-                                 c.rms_eps, M, d, h->h1, h->n.out(tc_gu), st));
+                                 c.rms_eps, M, d, h->h1, h->n.out(tc_gu, mlp_lo), st));
     mark(SP_STAGE_POST_NORM, 1);
     ++launches;
     // a5: gate/up + SwiGLU
     mark(SP_STAGE_GATE_UP, 0);
-    s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, M, h->status, st, &launches, &ns);
+    s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, M, h->status, st, &launches, &ns, mlp_lo);
     mark(SP_STAGE_GATE_UP, 1);
     if (s != SP_OK) return fail(s, "gate/up projection launch failed");
     mark(SP_STAGE_SWIGLU, 0);
-    SP_CUDA(launch_swiglu(PartIn{h->y, ns, (size_t)M * 2 * f}, M, f, h->gu_blk, h->a.out(tc_down), st));
+    SP_CUDA(launch_swiglu(PartIn{h->y, ns, (size_t)M * 2 * f}, M, f, h->gu_blk, h->a.out(tc_down, mlp_lo), st));
     mark(SP_STAGE_SWIGLU, 1);
     ++launches;
     // a6-a7: down projection + residual, pooling, linear head
     mark(SP_STAGE_DOWN, 0);
-    s = h->gemm.run(wb, h->opt_gemm, h->a, h->w_down, h->y, M, h->status, st, &launches, &ns);
+    s = h->gemm.run(wb, h->opt_gemm, h->a, h->w_down, h->y, M, h->status, st, &launches, &ns, mlp_lo);
     mark(SP_STAGE_DOWN, 1);
     if (s != SP_OK) return fail(s, "down projection launch failed");
     mark(SP_STAGE_READOUT, 0);

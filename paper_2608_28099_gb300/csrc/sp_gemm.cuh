@@ -33,7 +33,8 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes);
 // views them as [N K / 64][64] rows.
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
-                           float *y, int *status, cudaStream_t st, bool w_blocked = false);
+                           float *y, int *status, cudaStream_t st, bool w_blocked = false,
+                           bool lo = true);
 
 // Weights [N][K] (es bytes per element) re-laid out as contiguous 16 KB blocks
 // [N / 128][K / 64][128][64]: one weight tile's k-block is one sequential read
@@ -69,12 +70,14 @@ struct ActBuf {
     int K = 0, rows_max = 0;
     bool maps = false;
     CUtensorMap hi[kNumBn], lo[kNumBn];
-    ActOut out(bool hilo) const {
+    // tc: the consumer is a tensor-core projection (bf16 planes), else fp32;
+    // lo: with the lo plane (hi + lo ~ 16 mantissa bits), else plain bf16
+    ActOut out(bool tc, bool lo = true) const {
         ActOut o;
-        if (hilo) {
+        if (tc) {
             o.f32 = nullptr;
             o.hi = (bf16 *)ptr;
-            o.lo = (bf16 *)ptr + (size_t)rows_max * K;
+            o.lo = lo ? (bf16 *)ptr + (size_t)rows_max * K : nullptr;
         } else {
             o.f32 = (float *)ptr;
             o.hi = o.lo = nullptr;
@@ -124,12 +127,12 @@ struct GemmPlanner {
     }
     // Enqueue the projection; *nsplit receives the number of partials in y.
     sp_status run(int w_bf16, int path, const ActBuf &x, const WeightMat &w, float *y, int M,
-                  int *status, cudaStream_t st, int *launches, int *nsplit) const {
+                  int *status, cudaStream_t st, int *launches, int *nsplit, bool lo = true) const {
         cudaError_t e;
         if (use_tc(w, x, path)) {
             const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity);
             const int bi = bn_index(p.bn);
-            e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked);
+            e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked, lo);
             *nsplit = p.splits;
         } else {
             e = launch_gemm_simt(w_bf16, x.ptr, w.ptr, y, M, w.N, w.K, st, w.blocked);

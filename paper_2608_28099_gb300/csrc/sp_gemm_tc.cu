@@ -12,6 +12,8 @@
 // one MMA of N = 2 BN per 16-wide k-step reads the weight tile once and leaves
 // W hi^T in TMEM columns [0, BN) and W lo^T in [BN, 2 BN); the epilogue adds
 // the halves.  The product carries ~16 bits of the activation's mantissa.
+// Without the lo plane (template flag LO = false) the activations are plain
+// bf16: half the MMA work and activation traffic, a deeper ring.
 //
 // Two schedules, fp32 partials in planes of Y that the consumers add:
 //  * tile kernel: one CTA per (tile, K split); split-K when the tiles alone
@@ -43,12 +45,15 @@ constexpr int BK = 64;               // bf16 elements per 128-byte swizzle row
 constexpr int A_BYTES = 128 * BK * 2;
 
 // ---------------------------------------------------------------- tile kernel
-template <int BN>
+// LO: the activations come as hi and lo planes (the MMA's N side is [hi; lo],
+// 2 BN rows), else as plain bf16 (N = BN).
+template <int BN, bool LO>
 struct TileCfg {
     static constexpr int B_BYTES = BN * BK * 2;
-    static constexpr int STAGE = A_BYTES + 2 * B_BYTES;
-    static constexpr int STAGES = (BN <= 32) ? 8 : (BN == 64 ? 6 : 4);
-    static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;  // hi and lo halves
+    static constexpr int NB = (LO ? 2 : 1) * BN;                 // MMA N
+    static constexpr int STAGE = A_BYTES + (LO ? 2 : 1) * B_BYTES;
+    static constexpr int STAGES = 196608 / STAGE < 10 ? 196608 / STAGE : 10;  // 192 KB ring
+    static constexpr int TMEM_COLS = NB < 32 ? 32 : NB;          // hi and lo halves
     static constexpr int SMEM = STAGES * STAGE + 1024 /*align*/ + 256 /*barriers*/;
 };
 
@@ -61,12 +66,12 @@ struct TcArgs {
     int *status;
 };
 
-template <int BN>
+template <int BN, bool LO>
 __global__ void __launch_bounds__(128, 1)
     gemm_tile_kernel(const __grid_constant__ CUtensorMap map_w,
                    const __grid_constant__ CUtensorMap map_xhi,
                    const __grid_constant__ CUtensorMap map_xlo, TcArgs g) {
-    using Cfg = TileCfg<BN>;
+    using Cfg = TileCfg<BN, LO>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t *full = (uint64_t *)(smem + Cfg::STAGES * Cfg::STAGE);
@@ -131,11 +136,11 @@ __global__ void __launch_bounds__(128, 1)
                 issued = i + 1;
             }
             tma_load_2d_hint(st + A_BYTES, &map_xhi, &full[s], kc, m0, pol_x);
-            tma_load_2d_hint(st + A_BYTES + Cfg::B_BYTES, &map_xlo, &full[s], kc, m0, pol_x);
+            if (LO) tma_load_2d_hint(st + A_BYTES + Cfg::B_BYTES, &map_xlo, &full[s], kc, m0, pol_x);
         }
     } else if (warp == 1 && lane == 0) {
         // MMA issuer
-        constexpr uint32_t idesc = idesc_bf16_f32(128, 2 * BN);
+        constexpr uint32_t idesc = idesc_bf16_f32(128, Cfg::NB);
         for (int i = 0; i < nkb; ++i) {
             const int s = i % Cfg::STAGES;
             const uint32_t ph = (i / Cfg::STAGES) & 1;
@@ -164,9 +169,9 @@ __global__ void __launch_bounds__(128, 1)
         float *y = g.y + (size_t)blockIdx.z * g.split_stride;
         const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
         if constexpr (BN == 16) {
-            float v[16], u[16];
+            float v[16], u[16] = {};
             tmem_ld16(trow, v);
-            tmem_ld16(trow + 16, u);
+            if (LO) tmem_ld16(trow + 16, u);
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
                 const int m = m0 + j;
@@ -175,9 +180,9 @@ __global__ void __launch_bounds__(128, 1)
         } else {
 #pragma unroll 1
             for (int c0 = 0; c0 < BN; c0 += 32) {
-                float v[32], u[32];
+                float v[32], u[32] = {};
                 tmem_ld32(trow + c0, v);
-                tmem_ld32(trow + BN + c0, u);
+                if (LO) tmem_ld32(trow + BN + c0, u);
 #pragma unroll
                 for (int j = 0; j < 32; ++j) {
                     const int m = m0 + c0 + j;
@@ -197,18 +202,18 @@ __global__ void __launch_bounds__(128, 1)
     if (warp == 2) tmem_dealloc(tmem, Cfg::TMEM_COLS);
 }
 
-template <int BN>
+template <int BN, bool LO>
 cudaError_t launch_tile(const CUtensorMap &mw, const CUtensorMap &mh, const CUtensorMap &ml,
                       const TcArgs &g, dim3 grid, cudaStream_t st) {
-    const int smem = TileCfg<BN>::SMEM;
+    const int smem = TileCfg<BN, LO>::SMEM;
     static bool attr_set = false;  // per device process-wide (one device per process here)
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_tile_kernel<BN>,
+        cudaError_t e = cudaFuncSetAttribute(gemm_tile_kernel<BN, LO>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    return launch_k(gemm_tile_kernel<BN>, grid, dim3(128), (size_t)smem, st, mw, mh, ml, g);
+    return launch_k(gemm_tile_kernel<BN, LO>, grid, dim3(128), (size_t)smem, st, mw, mh, ml, g);
 }
 
 
@@ -216,13 +221,14 @@ cudaError_t launch_tile(const CUtensorMap &mw, const CUtensorMap &mh, const CUte
 constexpr int GEMM_THREADS = 224;
 constexpr int W_WARP = 4, X_WARP = 5, MMA_WARP_G = 6;
 
-template <int BN>
+template <int BN, bool LO>
 struct PkCfg {
     static constexpr int B_BYTES = BN * BK * 2;       // one activation plane of a k-block
-    static constexpr int X_STAGE = 2 * B_BYTES;       // hi + lo
-    static constexpr int W_STAGES = BN <= 32 ? 8 : (BN == 64 ? 6 : 5);
-    static constexpr int X_STAGES = BN <= 32 ? 4 : 3;
-    static constexpr int ACC_COLS = 2 * BN < 32 ? 32 : 2 * BN;  // hi and lo halves
+    static constexpr int NB = (LO ? 2 : 1) * BN;      // MMA N
+    static constexpr int X_STAGE = (LO ? 2 : 1) * B_BYTES;  // hi (+ lo)
+    static constexpr int W_STAGES = BN <= 32 ? 8 : (BN == 64 ? 6 : (LO ? 5 : 6));
+    static constexpr int X_STAGES = BN <= 32 ? 4 : (LO ? 3 : 4);
+    static constexpr int ACC_COLS = NB < 32 ? 32 : NB;     // hi and lo halves
     static constexpr int TMEM_COLS = 2 * ACC_COLS;              // double-buffered
     static constexpr int OFF_X = W_STAGES * A_BYTES;
     static constexpr int OFF_BAR = OFF_X + X_STAGES * X_STAGE;
@@ -254,12 +260,12 @@ __device__ __forceinline__ Seg segment(const PkArgs &g, long long u0, long long 
     return s;
 }
 
-template <int BN>
+template <int BN, bool LO>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_pk_kernel(const __grid_constant__ CUtensorMap map_w,
                    const __grid_constant__ CUtensorMap map_xhi,
                    const __grid_constant__ CUtensorMap map_xlo, PkArgs g) {
-    using Cfg = PkCfg<BN>;
+    using Cfg = PkCfg<BN, LO>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t *w_full = (uint64_t *)(smem + Cfg::OFF_BAR);
@@ -352,12 +358,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                 uint8_t *st = smem + Cfg::OFF_X + s * Cfg::X_STAGE;
                 mbar_arrive_expect_tx(&x_full[s], Cfg::X_STAGE);
                 tma_load_2d_hint(st, &map_xhi, &x_full[s], kb * BK, m0, pol_x);
-                tma_load_2d_hint(st + Cfg::B_BYTES, &map_xlo, &x_full[s], kb * BK, m0, pol_x);
+                if (LO) tma_load_2d_hint(st + Cfg::B_BYTES, &map_xlo, &x_full[s], kb * BK, m0, pol_x);
                 issued = i + 1;
             }
         }
     } else if (warp == MMA_WARP_G && lane == 0) {
-        constexpr uint32_t idesc = idesc_bf16_f32(128, 2 * BN);
+        constexpr uint32_t idesc = idesc_bf16_f32(128, Cfg::NB);
         int i = 0, sgi = 0;
         bool ok = true;
         for (int t = t_first; ok && t <= t_last; ++t, ++sgi) {
@@ -406,9 +412,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             float *y = g.y + (size_t)plane * g.plane_stride;
             const uint32_t ta = trow + (uint32_t)(buf * Cfg::ACC_COLS);
             if constexpr (BN == 16) {
-                float v[16], u[16];
+                float v[16], u[16] = {};
                 tmem_ld16(ta, v);
-                tmem_ld16(ta + 16, u);
+                if (LO) tmem_ld16(ta + 16, u);
 #pragma unroll
                 for (int j = 0; j < 16; ++j) {
                     const int m = m0 + j;
@@ -417,9 +423,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             } else {
 #pragma unroll 1
                 for (int c0 = 0; c0 < BN; c0 += 32) {
-                    float v[32], u[32];
+                    float v[32], u[32] = {};
                     tmem_ld32(ta + c0, v);
-                    tmem_ld32(ta + BN + c0, u);
+                    if (LO) tmem_ld32(ta + BN + c0, u);
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
                         const int m = m0 + c0 + j;
@@ -456,18 +462,18 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     if (warp == MMA_WARP_G) tmem_dealloc(tmem, Cfg::TMEM_COLS);
 }
 
-template <int BN>
+template <int BN, bool LO>
 cudaError_t launch_pk(const CUtensorMap &mw, const CUtensorMap &mh, const CUtensorMap &ml,
                       const PkArgs &g, int grid, cudaStream_t st) {
-    const int smem = PkCfg<BN>::SMEM;
+    const int smem = PkCfg<BN, LO>::SMEM;
     static bool attr_set = false;  // per device process-wide (one device per process here)
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_pk_kernel<BN>,
+        cudaError_t e = cudaFuncSetAttribute(gemm_pk_kernel<BN, LO>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    return launch_k(gemm_pk_kernel<BN>, dim3(grid), dim3(GEMM_THREADS), (size_t)smem, st, mw, mh, ml,
+    return launch_k(gemm_pk_kernel<BN, LO>, dim3(grid), dim3(GEMM_THREADS), (size_t)smem, st, mw, mh, ml,
                     g);
 }
 
@@ -600,7 +606,7 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes) {
 
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
-                           float *y, int *status, cudaStream_t st, bool w_blocked) {
+                           float *y, int *status, cudaStream_t st, bool w_blocked, bool lo) {
     if (p.persistent) {
         PkArgs g;
         g.M = M;
@@ -615,10 +621,14 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
         g.plane_stride = (size_t)M * N;
         g.status = status;
         switch (p.bn) {
-        case 16: return launch_pk<16>(map_w, map_xhi, map_xlo, g, p.grid, st);
-        case 32: return launch_pk<32>(map_w, map_xhi, map_xlo, g, p.grid, st);
-        case 64: return launch_pk<64>(map_w, map_xhi, map_xlo, g, p.grid, st);
-        case 128: return launch_pk<128>(map_w, map_xhi, map_xlo, g, p.grid, st);
+        case 16: return lo ? launch_pk<16, true>(map_w, map_xhi, map_xlo, g, p.grid, st)
+                        : launch_pk<16, false>(map_w, map_xhi, map_xlo, g, p.grid, st);
+        case 32: return lo ? launch_pk<32, true>(map_w, map_xhi, map_xlo, g, p.grid, st)
+                        : launch_pk<32, false>(map_w, map_xhi, map_xlo, g, p.grid, st);
+        case 64: return lo ? launch_pk<64, true>(map_w, map_xhi, map_xlo, g, p.grid, st)
+                        : launch_pk<64, false>(map_w, map_xhi, map_xlo, g, p.grid, st);
+        case 128: return lo ? launch_pk<128, true>(map_w, map_xhi, map_xlo, g, p.grid, st)
+                        : launch_pk<128, false>(map_w, map_xhi, map_xlo, g, p.grid, st);
         default: return cudaErrorInvalidValue;
         }
     }
@@ -634,10 +644,14 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
     g.status = status;
     dim3 grid(p.m_tiles, p.n_tiles, p.splits);
     switch (p.bn) {
-    case 16: return launch_tile<16>(map_w, map_xhi, map_xlo, g, grid, st);
-    case 32: return launch_tile<32>(map_w, map_xhi, map_xlo, g, grid, st);
-    case 64: return launch_tile<64>(map_w, map_xhi, map_xlo, g, grid, st);
-    case 128: return launch_tile<128>(map_w, map_xhi, map_xlo, g, grid, st);
+    case 16: return lo ? launch_tile<16, true>(map_w, map_xhi, map_xlo, g, grid, st)
+                    : launch_tile<16, false>(map_w, map_xhi, map_xlo, g, grid, st);
+    case 32: return lo ? launch_tile<32, true>(map_w, map_xhi, map_xlo, g, grid, st)
+                    : launch_tile<32, false>(map_w, map_xhi, map_xlo, g, grid, st);
+    case 64: return lo ? launch_tile<64, true>(map_w, map_xhi, map_xlo, g, grid, st)
+                    : launch_tile<64, false>(map_w, map_xhi, map_xlo, g, grid, st);
+    case 128: return lo ? launch_tile<128, true>(map_w, map_xhi, map_xlo, g, grid, st)
+                    : launch_tile<128, false>(map_w, map_xhi, map_xlo, g, grid, st);
     default: return cudaErrorInvalidValue;
     }
 }
