@@ -255,13 +255,23 @@ enum {
                                  between CTA shares balance (-1..1024); -1 = the
                                  built-in default.  Changes the work split only,
                                  never the result beyond rounding order          */
-    SP_OPT_ACT_PRECISION = 7  /* activations fed to the tensor-core MLP
+    SP_OPT_ACT_PRECISION = 7, /* activations fed to the tensor-core MLP
                                  projections (gate/up and down): 0 = automatic
                                  (plain bf16 when pool is SP_POOL_MEAN and at
                                  least 8 rows per task are pooled, else bf16
                                  hi + lo planes, ~16 mantissa bits), 1 = hi + lo
                                  always, 2 = plain bf16 always.  The Q/K/V and
                                  output projections always take hi + lo        */
+    SP_OPT_DEBUG_STALL = 8    /* test of the failure path: 1 = in the next
+                                 sp_classify only, the first CTA of the output
+                                 projection (when it runs on the one-CTA-per-tile
+                                 schedule) never loads its first k-block, so its
+                                 tensor-core wait runs out; that launch's waits
+                                 give up after 1 ms, the kernel drains its copies,
+                                 frees TMEM and returns, and sp_check_status
+                                 reports SP_DEV_TIMEOUT (that call's logits are
+                                 invalid, the handle stays usable).  Resets
+                                 itself after that call                          */
 };
 
 /* Stages of sp_classify, in launch order. */
@@ -290,6 +300,17 @@ SP_API sp_status sp_set_option(sp_handle *h, int key, int value);
 
 /* Number of kernel launches the last sp_classify enqueued. */
 SP_API int sp_last_launch_count(const sp_handle *h);
+
+/* Test hook: record the physical page ids the attention step of every later
+ * sp_classify / sp_classify_hidden reads (paged caches only).  d_out is a
+ * DEVICE int32 buffer of `capacity` entries, caller-owned, laid out
+ * [batch][kv->max_pages_per_seq]: entry [i][j] receives the page id read for
+ * logical page j of the i-th classified sequence (entries it did not read are
+ * left untouched).  A call whose batch * max_pages_per_seq exceeds capacity
+ * returns SP_ERR_INVALID_ARG before any launch.  d_out = NULL stops the
+ * recording.  The ids let a test check the page-table walk bit-exactly (the
+ * pages of sequence b are page_table[b][0 .. ceil(L_b / page_size))). */
+SP_API sp_status sp_debug_gathered_pages(sp_handle *h, int *d_out, size_t capacity);
 
 /* ------------------------------------------------------------------------- */
 /* The attention step alone (Eq. 1-3), for step-level checks and for callers  */

@@ -18,18 +18,20 @@ SP_OK, SP_ERR_INVALID_ARG, SP_ERR_UNSUPPORTED, SP_ERR_CUDA, SP_ERR_OOM, SP_ERR_D
 SP_F32, SP_BF16 = 0, 1
 SP_POOL_MEAN, SP_POOL_LAST = 0, 1
 SP_KV_CONTIGUOUS, SP_KV_PAGED = 0, 1
-SP_DEV_BAD_SEQ_ID, SP_DEV_BAD_LENGTH, SP_DEV_BAD_PAGE = 1, 2, 4
+SP_DEV_BAD_SEQ_ID, SP_DEV_BAD_LENGTH, SP_DEV_BAD_PAGE, SP_DEV_TIMEOUT = 1, 2, 4, 8
 SP_OPT_SPLIT_TOKENS, SP_OPT_GEMM_PATH, SP_OPT_ATTN_PATH, SP_OPT_PROFILE = 1, 2, 3, 4
 SP_OPT_RECURSIVE = 5
 SP_OPT_ATTN_SEG_COST = 6
 SP_OPT_ACT_PRECISION = 7
+SP_OPT_DEBUG_STALL = 8
 STAGES = ["input_norm", "qkv", "rope", "attention", "merge", "o_proj", "post_norm", "gate_up",
           "swiglu", "down", "readout", "fusion"]
 
 EXPORTED = ["sp_create", "sp_destroy", "sp_classify", "sp_classify_host", "sp_check_status",
             "sp_last_error", "sp_set_option", "sp_last_launch_count", "sp_attend_workspace_bytes",
             "sp_attend", "sp_stage_times", "sp_project_workspace_bytes", "sp_project",
-            "sp_attend_static", "sp_classify_hidden", "sp_classify_hidden_host"]
+            "sp_attend_static", "sp_classify_hidden", "sp_classify_hidden_host",
+            "sp_debug_gathered_pages"]
 
 
 class sp_config(C.Structure):
@@ -101,6 +103,7 @@ def load_library(path: str | None = None):
                                      C.POINTER(sp_kv_cache), vp, vp, vp, vp, i, vp, vp]
     lib.sp_attend.argtypes = [vp, C.POINTER(sp_attn_dims), i, vp, vp, C.POINTER(sp_kv_cache), vp,
                               vp, vp, vp, i, vp, C.c_size_t, vp, vp]
+    lib.sp_debug_gathered_pages.argtypes = [vp, vp, C.c_size_t]
     for name in EXPORTED:
         if name not in ("sp_last_error", "sp_last_launch_count", "sp_attend_workspace_bytes",
                         "sp_project_workspace_bytes"):
@@ -187,6 +190,15 @@ def sp_set_option(handle, key, value):
 
 def sp_last_launch_count(handle) -> int:
     return load_library().sp_last_launch_count(handle)
+
+
+def sp_debug_gathered_pages(handle, out=None):
+    """Record the page ids the attention step of later classify calls reads
+    into the int32 device tensor `out` ([batch][max_pages_per_seq]); None stops."""
+    if out is None:
+        _check(load_library().sp_debug_gathered_pages(handle, None, 0))
+    else:
+        _check(load_library().sp_debug_gathered_pages(handle, _ptr(out), out.numel()))
 
 
 def sp_stage_times(handle) -> dict:

@@ -92,6 +92,9 @@ struct sp_handle {
     int opt_split = 0, opt_gemm = 0, opt_attn = 0, opt_profile = 0, opt_recursive = 0;
     int opt_seg_cost = -1;  // attention segment-boundary cost in tiles (-1 = default)
     int opt_prec = 0;       // activation precision of the MLP inputs (SP_OPT_ACT_PRECISION)
+    int opt_stall = 0;      // one-shot failure-path test (SP_OPT_DEBUG_STALL)
+    int *dbg_pages = nullptr;     // sp_debug_gathered_pages: recording buffer (device)
+    size_t dbg_pages_cap = 0;     // its capacity in ints
     int T = 1;        // tasks sharing the pass; cfg.k_rows holds T * k_task rows per sequence
     int k_task = 0;   // soft-prompt rows per task
     float *h2_all = nullptr;      // recursive probing: step outputs [k][max_batch][d] fp32
@@ -514,6 +517,10 @@ sp_status sp_set_option(sp_handle *h, int key, int value) {
         if (value != 0 && value != 1) return fail(SP_ERR_INVALID_ARG, "bad recursion flag");
         h->opt_recursive = value;
         return SP_OK;
+    case SP_OPT_DEBUG_STALL:
+        if (value != 0 && value != 1) return fail(SP_ERR_INVALID_ARG, "bad stall flag");
+        h->opt_stall = value;
+        return SP_OK;
     case SP_OPT_ACT_PRECISION:
         if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad activation precision");
         h->opt_prec = value;
@@ -536,6 +543,14 @@ sp_status sp_set_option(sp_handle *h, int key, int value) {
 }
 
 int sp_last_launch_count(const sp_handle *h) { return h ? h->last_launches : -1; }
+
+sp_status sp_debug_gathered_pages(sp_handle *h, int *d_out, size_t capacity) {
+    if (!h) return fail(SP_ERR_INVALID_ARG, "handle is NULL");
+    if (d_out && capacity == 0) return fail(SP_ERR_INVALID_ARG, "capacity must be > 0");
+    h->dbg_pages = d_out;
+    h->dbg_pages_cap = d_out ? capacity : 0;
+    return SP_OK;
+}
 
 sp_status sp_stage_times(sp_handle *h, float *ms, int n) {
     if (!h || !ms || n < 0) return fail(SP_ERR_INVALID_ARG, "bad arguments");
@@ -760,6 +775,12 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     a.q = h->q; a.k_new = h->k_new; a.v_new = h->v_new;
     a.status = h->status;
     a.gathered = nullptr;
+    if (h->dbg_pages && kv->layout == SP_KV_PAGED) {
+        if ((size_t)batch * kv->max_pages_per_seq > h->dbg_pages_cap)
+            return fail(SP_ERR_INVALID_ARG, "gathered-pages buffer holds %zu ids, the call needs %zu",
+                        h->dbg_pages_cap, (size_t)batch * kv->max_pages_per_seq);
+        a.gathered = h->dbg_pages;
+    }
     a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
     a.out = h->o.out(tc_o);
     s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, h->n_sm, h->opt_split,
@@ -773,8 +794,10 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     const void *x = d_hidden ? (const void *)h->xrows : d_rows ? d_rows : h->soft_prompt;
     const int row_mod = (d_rows || d_hidden) ? 0 : k;
     const int x_bf16 = d_hidden ? 0 : wb;
+    const int stall = h->opt_stall;  // one-shot: this call's output projection only
+    h->opt_stall = 0;
     mark(SP_STAGE_O_PROJ, 0);
-    s = h->gemm.run(wb, h->opt_gemm, h->o, h->w_o, h->y, M, h->status, st, &launches, &ns);
+    s = h->gemm.run(wb, h->opt_gemm, h->o, h->w_o, h->y, M, h->status, st, &launches, &ns, true, stall);
     mark(SP_STAGE_O_PROJ, 1);
     if (s != SP_OK) return fail(s, "output projection launch failed");
     mark(SP_STAGE_POST_NORM, 0);

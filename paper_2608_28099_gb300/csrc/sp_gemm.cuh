@@ -27,14 +27,16 @@ bool encode_kv_pages_bf16(CUtensorMap *map, const void *pool, long long n_page_h
 // TMA map of rotated queries [rows][Hq][128] fp32 by (k rows x G heads) boxes.
 bool encode_q_group_f32(CUtensorMap *map, const float *q, int rows, int Hq, int G, int k);
 bool tc_supported(int N, int K);
-int tc_bn_for(int M);
-TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes);
+// Rows per tile for M activation rows: 16..128, or 256 (plain bf16 only: the
+// MMA's N side is then 256) for M >= 256.
+int tc_bn_for(int M, bool lo = true);
+TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo = true);
 // w_blocked: the weights are stored blocked (block_weights_layout) and map_w
 // views them as [N K / 64][64] rows.
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
                            float *y, int *status, cudaStream_t st, bool w_blocked = false,
-                           bool lo = true);
+                           bool lo = true, int inject_stall = 0);
 
 // Weights [N][K] (es bytes per element) re-laid out as contiguous 16 KB blocks
 // [N / 128][K / 64][128][64]: one weight tile's k-block is one sequential read
@@ -50,8 +52,8 @@ inline void block_weights_layout(const char *src, char *dst, int N, int K, size_
         }
 }
 
-constexpr int kNumBn = 4;  // tile widths 16, 32, 64, 128
-inline int bn_index(int bn) { return bn == 16 ? 0 : bn == 32 ? 1 : bn == 64 ? 2 : 3; }
+constexpr int kNumBn = 5;  // tile widths 16, 32, 64, 128, 256
+inline int bn_index(int bn) { return bn == 16 ? 0 : bn == 32 ? 1 : bn == 64 ? 2 : bn == 128 ? 3 : 4; }
 inline int bn_value(int i) { return 16 << i; }
 
 // A frozen weight matrix on the device, with its TMA map when tensor cores apply.
@@ -107,6 +109,7 @@ inline void init_act(ActBuf &a, void *ptr, int rows_max, int K, bool want_maps) 
     bool ok = true;
     const bf16 *hi = (const bf16 *)ptr, *lo = hi + (size_t)rows_max * K;
     for (int i = 0; i < kNumBn; ++i) {
+        if (bn_value(i) > 128 && rows_max < bn_value(i)) break;  // never planned (M <= rows_max)
         ok = ok && encode_kmajor_bf16(&a.hi[i], hi, rows_max, K, bn_value(i));
         ok = ok && encode_kmajor_bf16(&a.lo[i], lo, rows_max, K, bn_value(i));
     }
@@ -127,12 +130,14 @@ struct GemmPlanner {
     }
     // Enqueue the projection; *nsplit receives the number of partials in y.
     sp_status run(int w_bf16, int path, const ActBuf &x, const WeightMat &w, float *y, int M,
-                  int *status, cudaStream_t st, int *launches, int *nsplit, bool lo = true) const {
+                  int *status, cudaStream_t st, int *launches, int *nsplit, bool lo = true,
+                  int inject_stall = 0) const {
         cudaError_t e;
         if (use_tc(w, x, path)) {
-            const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity);
+            const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo);
             const int bi = bn_index(p.bn);
-            e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked, lo);
+            e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked, lo,
+                               inject_stall);
             *nsplit = p.splits;
         } else {
             e = launch_gemm_simt(w_bf16, x.ptr, w.ptr, y, M, w.N, w.K, st, w.blocked);

@@ -64,6 +64,10 @@ struct TcArgs {
     float *y;         // [split][M][N]
     size_t split_stride;
     int *status;
+    // failure-path test: CTA (0, 0, 0) never loads its first k-block, so its
+    // MMA warp's wait runs out; every wait of the launch gives up after wait_ns
+    int inject_stall;
+    unsigned long long wait_ns;
 };
 
 template <int BN, bool LO>
@@ -115,7 +119,9 @@ __global__ void __launch_bounds__(128, 1)
         const uint64_t pol_w = policy_evict_first();
         const uint64_t pol_x = policy_evict_last();
         const int pre = nkb < Cfg::STAGES ? nkb : Cfg::STAGES;
+        const bool skip0 = g.inject_stall && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0;
         for (int i = 0; i < pre; ++i) {
+            if (skip0 && i == 0) continue;
             mbar_arrive_expect_tx(&full[i], Cfg::STAGE);
             tma_load_2d_hint(smem + i * Cfg::STAGE, &map_w, &full[i],
                              g.w_blocked ? 0 : (kb0 + i) * BK,
@@ -128,8 +134,9 @@ __global__ void __launch_bounds__(128, 1)
             const uint32_t ph = (i / Cfg::STAGES) & 1;
             uint8_t *st = smem + s * Cfg::STAGE;
             const int kc = (kb0 + i) * BK;
+            if (skip0 && i == 0) continue;
             if (i >= pre) {
-                if (!mbar_wait(&empty[s], ph ^ 1, abort)) break;
+                if (!mbar_wait(&empty[s], ph ^ 1, abort, g.wait_ns)) break;
                 mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
                 tma_load_2d_hint(st, &map_w, &full[s], g.w_blocked ? 0 : kc,
                                  g.w_blocked ? (blockIdx.y * g.n_kb + kb0 + i) * 128 : n0, pol_w);
@@ -144,7 +151,7 @@ __global__ void __launch_bounds__(128, 1)
         for (int i = 0; i < nkb; ++i) {
             const int s = i % Cfg::STAGES;
             const uint32_t ph = (i / Cfg::STAGES) & 1;
-            if (!mbar_wait(&full[s], ph, abort)) break;
+            if (!mbar_wait(&full[s], ph, abort, g.wait_ns)) break;
             tc_fence_after();
             uint8_t *st = smem + s * Cfg::STAGE;
             const uint64_t a = sw128_kmajor_desc(st);
@@ -194,7 +201,7 @@ __global__ void __launch_bounds__(128, 1)
     if (warp == 0 && lane == 0) {
         // no TMA write may still be in flight when the CTA's shared memory goes away
         for (int i = issued > Cfg::STAGES ? issued - Cfg::STAGES : 0; i < issued; ++i)
-            mbar_wait_drain(&full[i % Cfg::STAGES], (i / Cfg::STAGES) & 1);
+            mbar_wait_drain(&full[i % Cfg::STAGES], (i / Cfg::STAGES) & 1, g.wait_ns);
     }
     tc_fence_before();
     __syncthreads();
@@ -226,8 +233,8 @@ struct PkCfg {
     static constexpr int B_BYTES = BN * BK * 2;       // one activation plane of a k-block
     static constexpr int NB = (LO ? 2 : 1) * BN;      // MMA N
     static constexpr int X_STAGE = (LO ? 2 : 1) * B_BYTES;  // hi (+ lo)
-    static constexpr int W_STAGES = BN <= 32 ? 8 : (BN == 64 ? 6 : (LO ? 5 : 6));
-    static constexpr int X_STAGES = BN <= 32 ? 4 : (LO ? 3 : 4);
+    static constexpr int W_STAGES = BN <= 32 ? 8 : (BN == 64 ? 6 : (LO || BN == 256 ? 5 : 6));
+    static constexpr int X_STAGES = BN <= 32 ? 4 : (LO || BN == 256 ? 3 : 4);
     static constexpr int ACC_COLS = NB < 32 ? 32 : NB;     // hi and lo halves
     static constexpr int TMEM_COLS = 2 * ACC_COLS;              // double-buffered
     static constexpr int OFF_X = W_STAGES * A_BYTES;
@@ -541,11 +548,11 @@ bool encode_q_group_f32(CUtensorMap *map, const float *q, int rows, int Hq, int 
     return r == CUDA_SUCCESS;
 }
 
-int tc_bn_for(int M) {
+int tc_bn_for(int M, bool lo) {
     if (M <= 16) return 16;
     if (M <= 32) return 32;
     if (M <= 64) return 64;
-    return 128;
+    return (!lo && M >= 256) ? 256 : 128;
 }
 
 bool tc_supported(int N, int K) { return N % 128 == 0 && K % BK == 0 && K >= BK; }
@@ -560,9 +567,9 @@ static int planes_for(long long tiles, int n_kb, long long L) {
     return most;
 }
 
-TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes) {
+TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo) {
     TcPlan p;
-    p.bn = tc_bn_for(M);
+    p.bn = tc_bn_for(M, lo);
     p.m_tiles = ceil_div(M, p.bn);
     p.n_tiles = N / 128;
     p.n_kb = K / BK;
@@ -606,7 +613,8 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes) {
 
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
-                           float *y, int *status, cudaStream_t st, bool w_blocked, bool lo) {
+                           float *y, int *status, cudaStream_t st, bool w_blocked, bool lo,
+                           int inject_stall) {
     if (p.persistent) {
         PkArgs g;
         g.M = M;
@@ -629,6 +637,8 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                         : launch_pk<64, false>(map_w, map_xhi, map_xlo, g, p.grid, st);
         case 128: return lo ? launch_pk<128, true>(map_w, map_xhi, map_xlo, g, p.grid, st)
                         : launch_pk<128, false>(map_w, map_xhi, map_xlo, g, p.grid, st);
+        case 256: return lo ? cudaErrorInvalidValue  // N = 512: beyond one MMA
+                        : launch_pk<256, false>(map_w, map_xhi, map_xlo, g, p.grid, st);
         default: return cudaErrorInvalidValue;
         }
     }
@@ -642,6 +652,8 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
     g.y = y;
     g.split_stride = (size_t)M * N;
     g.status = status;
+    g.inject_stall = inject_stall;
+    g.wait_ns = inject_stall ? 1000000ull : sm100::kWaitLimitNs;
     dim3 grid(p.m_tiles, p.n_tiles, p.splits);
     switch (p.bn) {
     case 16: return lo ? launch_tile<16, true>(map_w, map_xhi, map_xlo, g, grid, st)
@@ -652,6 +664,8 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                     : launch_tile<64, false>(map_w, map_xhi, map_xlo, g, grid, st);
     case 128: return lo ? launch_tile<128, true>(map_w, map_xhi, map_xlo, g, grid, st)
                     : launch_tile<128, false>(map_w, map_xhi, map_xlo, g, grid, st);
+    case 256: return lo ? cudaErrorInvalidValue  // N = 512: beyond one MMA
+                    : launch_tile<256, false>(map_w, map_xhi, map_xlo, g, grid, st);
     default: return cudaErrorInvalidValue;
     }
 }

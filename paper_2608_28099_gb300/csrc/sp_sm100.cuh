@@ -51,14 +51,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
 }
 // Wait for the phase of `parity` to complete.  Returns false (and raises
 // *abort) after kWaitLimitNs, or early if another thread raised *abort.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort) {
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort,
+                                          uint64_t limit_ns = kWaitLimitNs) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_ns();
     for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((it & 63) == 0) {
             if (*abort) return false;
-            if (global_ns() - t0 > kWaitLimitNs) {
+            if (global_ns() - t0 > limit_ns) {
                 *abort = 1;
                 return false;
             }
@@ -68,12 +69,13 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
 
 // Time-limited wait that ignores *abort: used to drain in-flight copies and
 // MMAs before shared memory or TMEM is released.
-__device__ __forceinline__ bool mbar_wait_drain(uint64_t *bar, uint32_t parity) {
+__device__ __forceinline__ bool mbar_wait_drain(uint64_t *bar, uint32_t parity,
+                                                uint64_t limit_ns = kWaitLimitNs) {
     if (mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = global_ns();
     for (uint32_t it = 1;; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 63) == 0 && global_ns() - t0 > kWaitLimitNs) return false;
+        if ((it & 63) == 0 && global_ns() - t0 > limit_ns) return false;
     }
 }
 

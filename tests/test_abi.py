@@ -78,6 +78,7 @@ def test_null_handle_calls_fail_cleanly(lib):
     assert lib.sp_set_option(None, 1, 0) == sp.SP_ERR_INVALID_ARG
     assert lib.sp_destroy(None) == sp.SP_OK
     assert lib.sp_last_launch_count(None) == -1
+    assert lib.sp_debug_gathered_pages(None, None, 0) == sp.SP_ERR_INVALID_ARG
 
 
 def test_attend_rejects_bad_dims_on_host(lib):

@@ -307,3 +307,49 @@ def test_mlp_activation_precision_options(prec):
     run = GpuRun(w, options={sp.SP_OPT_ACT_PRECISION: prec})
     compare(run.logits(), oracle_logits(w), label=f"precision option {prec}")
     run.close()
+
+
+def test_tensor_core_wait_timeout_is_reported_and_the_handle_recovers():
+    # the failure path of the bounded waits: one CTA of the output projection
+    # never receives its first k-block, its MMA warp gives up after 1 ms, the
+    # kernel drains, frees TMEM and reports SP_DEV_TIMEOUT; nothing faults
+    torch = torch_dev()
+    w = wl.custom(SMALL_BF16, [20, 300, 64, 5], wl.LAYOUT_PAGED, 151, rows_per_seq=True)
+    run = GpuRun(w)
+    h = run.model.handle
+    out = torch.empty((4, SMALL_BF16.n_classes), dtype=torch.float32, device="cuda")
+    sp.sp_set_option(h, sp.SP_OPT_DEBUG_STALL, 1)
+    sp.sp_classify(h, torch.cuda.current_stream(), 4, run.ids, run.cache.seq_lens, run.cache.desc,
+                   run.rows, out)
+    assert sp.sp_check_status(h) & sp.SP_DEV_TIMEOUT
+    # the option was one-shot: the next call on the same handle is clean and exact
+    compare(run.logits(), oracle_logits(w), label="after timeout")
+    run.close()
+
+
+def test_classify_records_the_gathered_pages_bit_exact():
+    # the page-table walk of the full call on the 8b paged configuration
+    # (K/V values drawn on the device; lengths and page table as the host draw)
+    torch = torch_dev()
+    ensure_built()
+    spec = wl.named("8b_paged", rows_per_seq=True)
+    dw = wl.generate_on_device(spec)
+    cache = sp.DevicePagedCache(dw)
+    B = spec.batch
+    model = sp.Model(spec.shape, dw.weights, B, int(dw.seq_lens.max()))
+    h = model.handle
+    max_pages = dw.page_table.shape[1]
+    rec = torch.full((B, max_pages), -1, dtype=torch.int32, device="cuda")
+    sp.sp_debug_gathered_pages(h, rec)
+    rows = torch.from_numpy(np.ascontiguousarray(dw.rows).view(np.int16)).cuda()
+    ids = torch.arange(B, dtype=torch.int32, device="cuda")
+    out = torch.empty((B, spec.shape.n_classes), dtype=torch.float32, device="cuda")
+    sp.sp_classify(h, torch.cuda.current_stream(), B, ids, cache.seq_lens, cache.desc, rows, out)
+    assert sp.sp_check_status(h) == 0
+    got = rec.cpu().numpy()
+    for b in range(B):
+        npg = (int(dw.seq_lens[b]) + 15) // 16
+        assert np.array_equal(got[b, :npg], dw.page_table[b, :npg])
+        assert np.all(got[b, npg:] == -1)  # pages past the length are never read
+    sp.sp_debug_gathered_pages(h, None)
+    model.close()
