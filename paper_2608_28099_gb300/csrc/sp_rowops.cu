@@ -62,39 +62,55 @@ __global__ void __launch_bounds__(256) rmsnorm_rows_kernel(const T *__restrict__
     }
 }
 
-// One thread per rotated pair (query heads, then key heads) or value element
-// of one row: grid (ceil(per_row / 256), B * k).
-__global__ void qkv_rope_kernel(QkvRopeArgs a) {
+// One block per row m = b k + r: the row's position L_b + r0 + r is resolved
+// once (from the caller's ids and lengths, before the dependency wait), then
+// each thread rotates four pairs (i, i + dh/2) of a query or key head at a time
+// (16-byte loads of the partial sums and of the (cos, sin) table) or copies
+// four values.
+__global__ void __launch_bounds__(256) qkv_rope_kernel(QkvRopeArgs a) {
     pdl_trigger();
-    pdl_wait();
-    if (a.zero_ints && blockIdx.x == 0 && blockIdx.y == 0)
-        for (int t = threadIdx.x; t < a.n_zero; t += blockDim.x) a.zero_ints[t] = 0;
-    const int m = blockIdx.y;
+    __shared__ int s_pos;
+    const int m = blockIdx.x;
     const int b = m / a.k, r = m % a.k;
-    const int dh = a.dh, half = dh >> 1;
-    const int nrot = (a.Hq + a.Hkv) * half;
-    const int nval = a.Hkv * dh;
-    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= nrot + nval) return;
-    SeqRef s = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.n_seqs, a.max_seq_len,
-                           idx == 0 ? a.status : nullptr);
+    if (threadIdx.x == 0) {
+        const SeqRef s = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.n_seqs,
+                                     a.max_seq_len, a.status);
+        s_pos = s.len + a.r0 + (a.k_task ? r % a.k_task : r);
+    }
+    pdl_wait();
+    if (a.zero_ints && m == 0)
+        for (int t = threadIdx.x; t < a.n_zero; t += blockDim.x) a.zero_ints[t] = 0;
+    __syncthreads();
+    const int dh = a.dh, half = dh >> 1, q4 = half >> 2;
     const int nqkv = (a.Hq + 2 * a.Hkv) * dh;
     const size_t row = (size_t)(a.shared ? r : m) * nqkv;
     const int kns = a.kn_stride ? a.kn_stride : a.k;
     const size_t mn = (size_t)b * kns + a.r0 + r;  // row of k_new / v_new
-    if (idx < nrot) {
-        const int pos = s.len + a.r0 + (a.k_task ? r % a.k_task : r);
-        const int h = idx / half, i = idx - h * half;
-        const float x0 = part_get(a.y, row + h * dh + i);
-        const float x1 = part_get(a.y, row + h * dh + i + half);
-        const float2 c = a.rope_cs[(size_t)pos * half + i];
-        float *dst = h < a.Hq ? a.q + ((size_t)m * a.Hq + h) * dh
-                              : a.k_new + (mn * a.Hkv + (h - a.Hq)) * dh;
-        dst[i] = x0 * c.x - x1 * c.y;
-        dst[i + half] = x1 * c.x + x0 * c.y;
-    } else {
-        const int j = idx - nrot;
-        a.v_new[mn * nval + j] = part_get(a.y, row + (size_t)(a.Hq + a.Hkv) * dh + j);
+    const float2 *cs = a.rope_cs + (size_t)s_pos * half;
+    const int nrot = (a.Hq + a.Hkv) * q4, nval = a.Hkv * dh / 4;
+    for (int it = threadIdx.x; it < nrot + nval; it += blockDim.x) {
+        if (it < nrot) {
+            const int h = it / q4, i = (it - h * q4) * 4;
+            const float4 x0 = part_get4(a.y, row + (size_t)h * dh + i);
+            const float4 x1 = part_get4(a.y, row + (size_t)h * dh + i + half);
+            const float4 c01 = *(const float4 *)(cs + i), c23 = *(const float4 *)(cs + i + 2);
+            const float c[4] = {c01.x, c01.z, c23.x, c23.z}, sn[4] = {c01.y, c01.w, c23.y, c23.w};
+            const float a0[4] = {x0.x, x0.y, x0.z, x0.w}, a1[4] = {x1.x, x1.y, x1.z, x1.w};
+            float o0[4], o1[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                o0[e] = a0[e] * c[e] - a1[e] * sn[e];
+                o1[e] = a1[e] * c[e] + a0[e] * sn[e];
+            }
+            float *dst = h < a.Hq ? a.q + ((size_t)m * a.Hq + h) * dh
+                                  : a.k_new + (mn * a.Hkv + (h - a.Hq)) * dh;
+            *(float4 *)(dst + i) = make_float4(o0[0], o0[1], o0[2], o0[3]);
+            *(float4 *)(dst + i + half) = make_float4(o1[0], o1[1], o1[2], o1[3]);
+        } else {
+            const int j = (it - nrot) * 4;
+            *(float4 *)(a.v_new + mn * a.Hkv * dh + j) =
+                part_get4(a.y, row + (size_t)(a.Hq + a.Hkv) * dh + j);
+        }
     }
 }
 
@@ -363,9 +379,7 @@ cudaError_t launch_rmsnorm_rows(int x_bf16, const void *x, int row_mod, const fl
 }
 
 cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st) {
-    const int per_row = (a.Hq + a.Hkv) * (a.dh / 2) + a.Hkv * a.dh;
-    dim3 grid(ceil_div(per_row, 256), a.B * a.k);
-    return launch_k(qkv_rope_kernel, grid, dim3(256), 0, st, a);
+    return launch_k(qkv_rope_kernel, dim3(a.B * a.k), dim3(256), 0, st, a);
 }
 
 cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mod,
