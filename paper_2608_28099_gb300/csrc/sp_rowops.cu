@@ -172,98 +172,111 @@ __global__ void swiglu_kernel(PartIn y, int M, int f, int blk, ActOut a) {
     }
 }
 
-// Pooling and the linear head, column-parallel: block (chunk, b) pools 64
-// hidden columns of sequence b (h2 = h1 + y summed over the k rows by two
-// row groups, then mean or last) and writes its partial dot products with
-// every head row to part[b][chunk][C]; two classes are reduced at a time.
-constexpr int kReadoutCols = 64;
+// Pooling and the linear head, column-parallel: block (chunk, b) pools 256
+// hidden columns of sequence b (h2 = h1 + y summed over the k rows by two row
+// groups, four columns per thread with 16-byte loads, then mean or last) and
+// writes its partial dot products with every head row to part[b][chunk][C];
+// two classes are reduced at a time.
+constexpr int kReadoutCols = 256;
 constexpr int kReadoutGroups = 2;  // row groups of a block (threads = 64 x 2)
 
-// six blocks per SM: all blocks of a 4b-sized call in one wave
-__global__ void __launch_bounds__(kReadoutCols * kReadoutGroups, 6)
+__device__ __forceinline__ float4 f4_add(float4 a, float4 b) {
+    return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+
+__global__ void __launch_bounds__(64 * kReadoutGroups, 4)
 readout_partial_kernel(PartIn y, const float *__restrict__ h1, const float *__restrict__ head_w,
                        int pool, int k, int d, int C, float *__restrict__ part, size_t sb, size_t sr,
                        int n_tasks, const float *__restrict__ g_final, float *__restrict__ part_ss) {
     pdl_trigger();
-    __shared__ float acc_s[kReadoutGroups][kReadoutCols];
+    __shared__ float4 acc_s[kReadoutGroups][64];
     __shared__ float pooled[kReadoutCols];
     __shared__ float red[4][8];
     const int chunk = blockIdx.x, b = blockIdx.y;
-    const int c = threadIdx.x & (kReadoutCols - 1), rg = threadIdx.x / kReadoutCols;
-    const int col = chunk * kReadoutCols + c;
+    const int c = threadIdx.x & 63, rg = threadIdx.x >> 6;
+    const int col = chunk * kReadoutCols + 4 * c;  // d % 4 == 0: a group is all in or all out
+    const bool in_d = col < d;
     const size_t base = (size_t)b * sb;
     head_w += (size_t)(b % n_tasks) * C * d;  // this task's head
     // the head is a constant of the handle, not an output of the previous
     // kernel: the first classes' weights are fetched before the wait
-    const float hw0 = (rg < C && col < d) ? head_w[(size_t)rg * d + col] : 0.f;
+    const float4 hw0 = (rg < C && in_d) ? *(const float4 *)(head_w + (size_t)rg * d + col)
+                                        : make_float4(0.f, 0.f, 0.f, 0.f);
     pdl_wait();
-    float acc = 0.f;
-    if (col < d) {
-        if (pool == SP_POOL_LAST) {
-            if (rg == 0) {
-                const size_t o = base + (size_t)(k - 1) * sr + col;
-                acc = h1[o] + part_get(y, o);
-            }
-        } else {
-            // rows rg, rg + G, ... (G row groups), four at a time with the loads
-            // of all their partials issued together
-            for (int r0 = rg; r0 < k; r0 += 4 * kReadoutGroups) {
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (in_d) {
+        // rows rg, rg + G, ... (G row groups) four at a time (all rows when
+        // pooling the last one is a single row), the loads of their h1 values
+        // and of two partials each issued together
+        const int r_first = pool == SP_POOL_LAST ? k - 1 : rg;
+        const int r_step = pool == SP_POOL_LAST ? k : kReadoutGroups;
+        if (pool != SP_POOL_LAST || rg == 0) {
+            for (int r0 = r_first; r0 < k; r0 += 4 * r_step) {
                 size_t o[4];
                 bool in[4];
-                float v[4];
+                float4 v[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    const int r = r0 + u * kReadoutGroups;
+                    const int r = r0 + u * r_step;
                     in[u] = r < k;
                     o[u] = base + (size_t)(in[u] ? r : r0) * sr + col;
-                    v[u] = in[u] ? h1[o[u]] : 0.f;
+                    v[u] = in[u] ? *(const float4 *)(h1 + o[u]) : make_float4(0.f, 0.f, 0.f, 0.f);
                 }
-                for (int i0 = 0; i0 < y.n; i0 += 8) {
-                    float pv[4][8];
+                for (int i0 = 0; i0 < y.n; i0 += 2) {
+                    float4 pv[4][2];
 #pragma unroll
                     for (int u = 0; u < 4; ++u)
 #pragma unroll
-                        for (int jj = 0; jj < 8; ++jj)
-                            pv[u][jj] = (in[u] && i0 + jj < y.n) ? y.y[(size_t)(i0 + jj) * y.stride + o[u]] : 0.f;
+                        for (int jj = 0; jj < 2; ++jj)
+                            pv[u][jj] = (in[u] && i0 + jj < y.n)
+                                            ? *(const float4 *)(y.y + (size_t)(i0 + jj) * y.stride + o[u])
+                                            : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
                     for (int u = 0; u < 4; ++u)
 #pragma unroll
-                        for (int jj = 0; jj < 8; ++jj) v[u] += pv[u][jj];
+                        for (int jj = 0; jj < 2; ++jj) v[u] = f4_add(v[u], pv[u][jj]);
                 }
-                acc += (v[0] + v[1]) + (v[2] + v[3]);
+                acc = f4_add(acc, f4_add(f4_add(v[0], v[1]), f4_add(v[2], v[3])));
             }
         }
     }
     acc_s[rg][c] = acc;
     __syncthreads();
-    if (threadIdx.x < kReadoutCols) {
-        float sum = 0.f;
+    if (threadIdx.x < 64) {
+        float4 sum = acc_s[0][c];
 #pragma unroll
-        for (int q = 0; q < kReadoutGroups; ++q) sum += acc_s[q][c];
-        const float p = pool == SP_POOL_LAST ? sum : sum / (float)k;
+        for (int q = 1; q < kReadoutGroups; ++q) sum = f4_add(sum, acc_s[q][c]);
+        const float dv = pool == SP_POOL_LAST ? 1.f : (float)k;
+        const float p[4] = {sum.x / dv, sum.y / dv, sum.z / dv, sum.w / dv};
         if (g_final) {
             // LM-head readout: the chunk's share of the pooled row's square sum,
-            // and the pooled value times the final-norm gain (the 1/rms factor
+            // and the pooled values times the final-norm gain (the 1/rms factor
             // is applied to the finished dot products)
-            float sq = col < d ? p * p : 0.f;
+            float sq = in_d ? (p[0] * p[0] + p[1] * p[1]) + (p[2] * p[2] + p[3] * p[3]) : 0.f;
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
             if ((threadIdx.x & 31) == 0) red[3][4 + (threadIdx.x >> 5)] = sq;
-            pooled[c] = col < d ? p * g_final[col] : 0.f;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) pooled[4 * c + e] = in_d ? p[e] * g_final[col + e] : 0.f;
         } else {
-            pooled[c] = p;
+#pragma unroll
+            for (int e = 0; e < 4; ++e) pooled[4 * c + e] = p[e];
         }
     }
     __syncthreads();
     if (g_final && threadIdx.x == 0)
         part_ss[(size_t)b * gridDim.x + chunk] = red[3][4] + red[3][5];
-    // row group rg takes class c0 + rg; its two warps hold the chunk's 64 columns
+    // row group rg takes class c0 + rg; its two warps hold the chunk's 256 columns
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
     for (int c0 = 0; c0 < C; c0 += kReadoutGroups) {
         const int cls = c0 + rg;
-        const bool use = cls < C && col < d;
-        const float hw = c0 == 0 ? hw0 : (use ? head_w[(size_t)cls * d + col] : 0.f);
-        float v = use ? hw * pooled[c] : 0.f;
+        const bool use = cls < C && in_d;
+        const float4 hw = c0 == 0 ? hw0
+                                  : (use ? *(const float4 *)(head_w + (size_t)cls * d + col)
+                                         : make_float4(0.f, 0.f, 0.f, 0.f));
+        float v = use ? (hw.x * pooled[4 * c] + hw.y * pooled[4 * c + 1]) +
+                            (hw.z * pooled[4 * c + 2] + hw.w * pooled[4 * c + 3])
+                      : 0.f;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
         if (lane == 0) red[w >> 1][w & 1] = v;
@@ -414,7 +427,7 @@ cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const
     if (!sr) sr = d;
     if (n_tasks < 1) n_tasks = 1;
     float *ss = g_final ? scratch + (size_t)B * chunks * C : nullptr;
-    cudaError_t e = launch_k(readout_partial_kernel, dim3(chunks, B), dim3(kReadoutCols * kReadoutGroups), 0, st, y, h1,
+    cudaError_t e = launch_k(readout_partial_kernel, dim3(chunks, B), dim3(64 * kReadoutGroups), 0, st, y, h1,
                              head_w, pool, k, d, C, scratch, sb, sr, n_tasks, g_final, ss);
     if (e != cudaSuccess) return e;
     return launch_k(readout_finish_kernel, dim3(B), dim3(64), 0, st, (const float *)scratch, chunks,
