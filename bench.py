@@ -52,7 +52,7 @@ FLUSH_BYTES = 256 << 20
 # DRAM read + write per launch of the dominant kernel, from one ncu capture of
 # the current kernel on the same workload; a workload or kernel without such a
 # capture reports null.
-TRAFFIC_BYTES = {}
+TRAFFIC_BYTES = {("27b_long", "attention"): 1080543104}
 
 
 def parse_args():
