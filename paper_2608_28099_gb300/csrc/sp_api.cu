@@ -783,6 +783,10 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     }
     a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
     a.out = h->o.out(tc_o);
+    if (tc_o) {  // the output projection's weights, prefetched by the attention's early finishers
+        a.l2_next = h->w_o.ptr;
+        a.l2_next_bytes = (size_t)d * hq * dh * h->es;
+    }
     s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, h->n_sm, h->opt_split,
                           &launches, st, true,
                           h->opt_profile ? h->ev[SP_STAGE_ATTN] : nullptr,

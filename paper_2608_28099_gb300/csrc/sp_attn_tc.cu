@@ -257,7 +257,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int T = prefix[B];
     const int n_grp = min((int)gridDim.x / Hkv, ceil_div(T, max(1, a.tc_min_tiles)));
     const int grp = blockIdx.x / Hkv, g = blockIdx.x - grp * Hkv;
-    if (grp >= n_grp) return;  // uniform over the CTA: no tile for this one
+    if (grp >= n_grp) {  // uniform over the CTA: no tile for this one
+        if (threadIdx.x == 0 && a.l2_next)
+            prefetch_l2_share(a.l2_next, a.l2_next_bytes, blockIdx.x, gridDim.x);
+        return;
+    }
     int *cuts = (int *)(smem + OFF_CUTS);
     for (int j = threadIdx.x; j <= n_grp; j += THREADS) cuts[j] = share_start(prefix, B, T, n_grp, j, a.tc_seg_cost);
     __syncthreads();
@@ -834,6 +838,11 @@ __global__ void __launch_bounds__(THREADS, 1)
     tc_fence_before();
     __syncthreads();
     if (threadIdx.x == 0 && *abort && a.status) atomicOr(a.status, SP_DEV_TIMEOUT);
+    // the cache stream of the slower CTAs leaves DRAM time for the next
+    // projection's weights: this CTA's share goes to L2 (the K/V tiles were
+    // loaded evict-first, so the weights stay)
+    if (threadIdx.x == 0 && a.l2_next)
+        prefetch_l2_share(a.l2_next, a.l2_next_bytes, blockIdx.x, gridDim.x);
     if (warp == MMA_WARP) tmem_dealloc(tmem, TMEM_COLS);
 }
 

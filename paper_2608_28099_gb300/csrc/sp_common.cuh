@@ -223,6 +223,8 @@ struct AttnArgs {
     int *gathered;                // [B][max_pages] or NULL
     float scale_log2;             // log2(e) / sqrt(dh)
     ActOut out;                   // merge output [B][k][Hq][dh]
+    const void *l2_next;          // tensor-core kernel: prefetched into L2 by the CTAs as
+    size_t l2_next_bytes;         // they finish (the next projection's weights), or NULL
 };
 
 // Plan: tokens per split-KV work unit and number of units per sequence.

@@ -121,6 +121,22 @@ __device__ __forceinline__ void tma_load_4d_hint(void *smem_dst, const CUtensorM
         "l"((uint64_t)map), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "l"(policy)
         : "memory");
 }
+// Bulk prefetch of `bytes` (a multiple of 16) of global memory into L2.
+__device__ __forceinline__ void prefetch_l2_bulk(const void *src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"((uint64_t)src), "r"(bytes)
+                 : "memory");
+}
+// This CTA's share (1 / parts, part = its index) of [base, base + bytes),
+// prefetched into L2 in 64 KB requests by the calling thread.
+__device__ __forceinline__ void prefetch_l2_share(const void *base, size_t bytes, int part,
+                                                  int parts) {
+    const size_t per = ((bytes + parts - 1) / parts + 15) & ~(size_t)15;
+    const size_t lo = per * (size_t)part, hi = lo + per < bytes ? lo + per : bytes;
+    for (size_t o = lo; o + 16 <= hi; o += 65536) {
+        const size_t n = hi - o < 65536 ? hi - o : 65536;
+        prefetch_l2_bulk((const char *)base + o, (uint32_t)(n & ~(size_t)15));
+    }
+}
 __device__ __forceinline__ uint64_t policy_evict_first() {
     uint64_t p;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
