@@ -645,7 +645,12 @@ def run_sweep(args):
             p_us = sum(stage_us.get(n, 0.0) for n in proj)
             M = B * k
             hbm_floor = p_bytes / (hbm * 1e9) * 1e6
-            tensor_floor = 2 * p_flops / (tfl_sus * 1e12) * 1e6  # bf16 hi + lo operand passes
+            # MMA work issued: Q/K/V and O always take hi + lo activations (two
+            # passes); gate/up and down take plain bf16 when the mean pools >= 8 rows
+            mlp_passes = 1 if k >= 8 else 2
+            issued = sum(st_work[n]["flops"] * (mlp_passes if n in ("gate_up", "down") else 2)
+                         for n in proj)
+            tensor_floor = issued / (tfl_sus * 1e12) * 1e6
             line = {"sweep_point": s.name, "B": B, "L": f"U[{lo},{hi}]", "k": k, "C": C,
                     "rows": M, "us_per_call": ms * 1e3, "seq_per_s": B / (ms / 1e3),
                     "hbm_gbs": totals["total_bytes"] / (ms / 1e3) / 1e9,
@@ -668,8 +673,10 @@ def run_sweep(args):
     summary = {"sweep": args.sweep, "points": len(results),
                "projection_crossover": {"largest_hbm_bound_rows": max(hbm_rows) if hbm_rows else None,
                                         "smallest_tensor_bound_rows": min(tensor_rows) if tensor_rows else None,
-                                        "note": "tensor floor counts the hi and lo bf16 passes; "
-                                                "the same tcgen05 kernel serves both sides"},
+                                        "note": "tensor floor counts two MMA passes for hi + lo "
+                                                "activations (Q/K/V, O; the MLP when k < 8) and one "
+                                                "for plain bf16; the same tcgen05 kernels serve both "
+                                                "sides"},
                "peaks": {"hbm_gbs": hbm, "bf16_tflops_sustained": tfl_sus, "source": peak_src},
                "clocks": clk, "steps": args.steps, "warmup": args.warmup,
                "l2": "flushed between steps (256 MiB write)"}
