@@ -79,6 +79,7 @@ struct sp_handle {
     void *stage_rows = nullptr;
     float *stage_logits = nullptr;
     float *readout_part = nullptr;  // [B][chunks][C] partial head dot products
+    int *readout_cnt = nullptr;     // [max_batch T] finished chunks per sequence (zero between calls)
     // input fusion (optional): x_{b,r} = W_fc_h RMSNorm(h_b; g_h) + fc_prompt[r]
     bool fused = false;
     WeightMat w_fc_h;             // [d][d]: the columns of W_fc acting on the hidden state
@@ -406,7 +407,8 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
                             h->fused ? M * d * 4 : 0,                    // xrows
                             h->fused ? (size_t)k * d * 4 : 0,            // fc_prompt
                             h->fused ? (size_t)c.max_batch * d * es : 0,  // stage hidden
-                            h->fused ? M * d * 4 : 0};                   // h2_all
+                            h->fused ? M * d * 4 : 0,                    // h2_all
+                            (size_t)c.max_batch * h->T * 4};             // readout counters
     for (size_t sz : sizes) total += align256(sz);
     void *arena = nullptr;
     if ((st = dev_alloc(h, &arena, total)) != SP_OK) return cleanup(st);
@@ -434,12 +436,15 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     h->fc_prompt = (float *)h->arena.take(sizes[19]);
     h->stage_hidden = h->arena.take(sizes[20]);
     h->h2_all = (float *)h->arena.take(sizes[21]);
+    h->readout_cnt = (int *)h->arena.take(sizes[22]);
     if (h->fused) init_act(h->xh, p_xh, c.max_batch, d, h->w_fc_h.tc);
     init_act(h->xn, p_xn, (int)M, d, h->w_qkv.tc);
     init_act(h->o, p_o_act, (int)M, hq * dh, h->w_o.tc);
     init_act(h->n, p_n, (int)M, d, h->w_gu.tc);
     init_act(h->a, p_a, (int)M, f, h->w_down.tc);
-    if (cudaMemset(h->status, 0, 256) != cudaSuccess) return cleanup(fail(SP_ERR_CUDA, "memset failed"));
+    if (cudaMemset(h->status, 0, 256) != cudaSuccess ||
+        cudaMemset(h->readout_cnt, 0, sizes[22]) != cudaSuccess)
+        return cleanup(fail(SP_ERR_CUDA, "memset failed"));
 
     // projections of the shared soft prompt rows (they do not depend on the
     // sequence), on CUDA cores with fp32 activations
@@ -653,8 +658,8 @@ static sp_status recursive_impl(sp_handle *h, cudaStream_t st, int batch, const 
         ++launches;
     }
     SP_CUDA(launch_readout(PartIn{nullptr, 0, 0}, h->h2_all, h->head_w, h->head_b, c.pool, B, k, d, C,
-                           h->readout_part, d_logits, st, (size_t)d, Bd, 1, h->g_final, c.rms_eps));
-    launches += 2;
+                           h->readout_part, d_logits, h->readout_cnt, st, (size_t)d, Bd, 1, h->g_final, c.rms_eps));
+    ++launches;
     h->last_launches = launches;
     return SP_OK;
 }
@@ -826,10 +831,10 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     mark(SP_STAGE_READOUT, 0);
     // one pooled readout per (sequence, task): rows [B][T][k_task][d]
     SP_CUDA(launch_readout(PartIn{h->y, ns, (size_t)M * d}, h->h1, h->head_w, h->head_b, c.pool,
-                           batch * h->T, h->k_task, d, C, h->readout_part, d_logits, st,
+                           batch * h->T, h->k_task, d, C, h->readout_part, d_logits, h->readout_cnt, st,
                            (size_t)h->k_task * d, (size_t)d, h->T, h->g_final, c.rms_eps));
     mark(SP_STAGE_READOUT, 1);
-    launches += 2;
+    ++launches;
     h->last_launches = launches;
     return SP_OK;
 }

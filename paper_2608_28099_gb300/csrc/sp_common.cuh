@@ -289,14 +289,16 @@ cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mo
 cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_t st);
 
 // logits[b] = W_head pool_r(h1 + y) + bias, via per-chunk partial dot
-// products in `scratch` (readout_scratch_bytes); two launches.
+// products in `scratch` (readout_scratch_bytes); one launch: the block that
+// finishes a sequence's last chunk (counters[b], zero before the launch and
+// cleared again by that block) adds the chunks up.
 size_t readout_scratch_bytes(int B, int d, int C);
 // Row r of sequence b of (h1 + y) sits at b sb + r sr (0 = the dense [B][k][d]
 // strides k d and d).  With n_tasks > 1, "sequence" b is (sequence b / n_tasks,
 // task b % n_tasks) and reads head [b % n_tasks] of head_w [n_tasks][C][d].
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
                            int pool, int B, int k, int d, int C, float *scratch, float *logits,
-                           cudaStream_t st, size_t sb = 0, size_t sr = 0, int n_tasks = 1,
+                           int *counters, cudaStream_t st, size_t sb = 0, size_t sr = 0, int n_tasks = 1,
                            const float *g_final = nullptr, float eps = 0.f);
 
 // ---------------------------------------------------------------------------

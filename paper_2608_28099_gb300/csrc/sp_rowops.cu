@@ -187,9 +187,12 @@ __device__ __forceinline__ float4 f4_add(float4 a, float4 b) {
 __global__ void __launch_bounds__(64 * kReadoutGroups, 4)
 readout_partial_kernel(PartIn y, const float *__restrict__ h1, const float *__restrict__ head_w,
                        int pool, int k, int d, int C, float *__restrict__ part, size_t sb, size_t sr,
-                       int n_tasks, const float *__restrict__ g_final, float *__restrict__ part_ss) {
+                       int n_tasks, const float *__restrict__ g_final, float *__restrict__ part_ss,
+                       int *__restrict__ counters, const float *__restrict__ head_b,
+                       float *__restrict__ logits, float eps) {
     pdl_trigger();
     __shared__ float4 acc_s[kReadoutGroups][64];
+    __shared__ int is_last;
     __shared__ float pooled[kReadoutCols];
     __shared__ float red[4][8];
     const int chunk = blockIdx.x, b = blockIdx.y;
@@ -286,26 +289,31 @@ readout_partial_kernel(PartIn y, const float *__restrict__ h1, const float *__re
                 red[threadIdx.x][0] + red[threadIdx.x][1];
         __syncthreads();
     }
-}
-
-__global__ void readout_finish_kernel(const float *__restrict__ part, int n_chunks, int C,
-                                      const float *__restrict__ head_b, float *__restrict__ logits,
-                                      int n_tasks, const float *__restrict__ part_ss, int d,
-                                      float eps) {
-    pdl_trigger();
-    pdl_wait();
-    const int b = blockIdx.x;
-    if (head_b) head_b += (size_t)(b % n_tasks) * C;
+    // the block that finishes sequence b's last chunk adds the chunks' dot
+    // products in chunk order (the bits do not depend on which block is last),
+    // applies the LM-head 1/rms and the bias, and clears the counter
+    __threadfence();  // this block's partials are visible before it is counted
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const int before = atomicAdd(counters + b, 1);
+        is_last = before == (int)gridDim.x - 1;
+        if (is_last) counters[b] = 0;
+    }
+    __syncthreads();
+    if (!is_last) return;
+    __threadfence();  // the other blocks' partials are read after their count
+    const int n_chunks = gridDim.x;
     float inv = 1.f;  // 1 / rms of the pooled row (LM-head readout)
-    if (part_ss) {
+    if (g_final) {
         float ss = 0.f;
-        for (int j = 0; j < n_chunks; ++j) ss += part_ss[(size_t)b * n_chunks + j];
+        for (int j = 0; j < n_chunks; ++j) ss += __ldcg(part_ss + (size_t)b * n_chunks + j);
         inv = rsqrtf(ss / (float)d + eps);
     }
-    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+    const float *hb = head_b ? head_b + (size_t)(b % n_tasks) * C : nullptr;
+    for (int cl = threadIdx.x; cl < C; cl += blockDim.x) {
         float acc = 0.f;
-        for (int j = 0; j < n_chunks; ++j) acc += part[((size_t)b * n_chunks + j) * C + c];
-        logits[(size_t)b * C + c] = acc * inv + (head_b ? head_b[c] : 0.f);
+        for (int j = 0; j < n_chunks; ++j) acc += __ldcg(part + ((size_t)b * n_chunks + j) * C + cl);
+        logits[(size_t)b * C + cl] = acc * inv + (hb ? hb[cl] : 0.f);
     }
 }
 
@@ -420,18 +428,16 @@ size_t readout_scratch_bytes(int B, int d, int C) {
 
 cudaError_t launch_readout(PartIn y, const float *h1, const float *head_w, const float *head_b,
                            int pool, int B, int k, int d, int C, float *scratch, float *logits,
-                           cudaStream_t st, size_t sb, size_t sr, int n_tasks,
+                           int *counters, cudaStream_t st, size_t sb, size_t sr, int n_tasks,
                            const float *g_final, float eps) {
     const int chunks = ceil_div(d, kReadoutCols);
     if (!sb) sb = (size_t)k * d;
     if (!sr) sr = d;
     if (n_tasks < 1) n_tasks = 1;
     float *ss = g_final ? scratch + (size_t)B * chunks * C : nullptr;
-    cudaError_t e = launch_k(readout_partial_kernel, dim3(chunks, B), dim3(64 * kReadoutGroups), 0, st, y, h1,
-                             head_w, pool, k, d, C, scratch, sb, sr, n_tasks, g_final, ss);
-    if (e != cudaSuccess) return e;
-    return launch_k(readout_finish_kernel, dim3(B), dim3(64), 0, st, (const float *)scratch, chunks,
-                    C, head_b, logits, n_tasks, (const float *)ss, d, eps);
+    return launch_k(readout_partial_kernel, dim3(chunks, B), dim3(64 * kReadoutGroups), 0, st, y, h1,
+                    head_w, pool, k, d, C, scratch, sb, sr, n_tasks, g_final, ss, counters, head_b,
+                    logits, eps);
 }
 
 cudaError_t launch_to_act(const float *x, size_t n, ActOut out, cudaStream_t st) {
