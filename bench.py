@@ -52,7 +52,10 @@ FLUSH_BYTES = 256 << 20
 # DRAM read + write per launch of the dominant kernel, from one ncu capture of
 # the current kernel on the same workload; a workload or kernel without such a
 # capture reports null.
-TRAFFIC_BYTES = {("27b_long", "attention"): 1080543104}
+# The attention kernel's figure includes the output projection's weights that its
+# CTAs prefetch into L2 as they finish (52.4 MB on 27b_long): the next kernel's
+# bytes, issued early.
+TRAFFIC_BYTES = {("27b_long", "attention"): 1132938112}
 
 
 def parse_args():
