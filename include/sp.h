@@ -262,7 +262,7 @@ enum {
                                  hi + lo planes, ~16 mantissa bits), 1 = hi + lo
                                  always, 2 = plain bf16 always.  The Q/K/V and
                                  output projections always take hi + lo        */
-    SP_OPT_DEBUG_STALL = 8    /* test of the failure path: 1 = in the next
+    SP_OPT_DEBUG_STALL = 8,   /* test of the failure path: 1 = in the next
                                  sp_classify only, the first CTA of the output
                                  projection (when it runs on the one-CTA-per-tile
                                  schedule) never loads its first k-block, so its
@@ -272,6 +272,19 @@ enum {
                                  reports SP_DEV_TIMEOUT (that call's logits are
                                  invalid, the handle stays usable).  Resets
                                  itself after that call                          */
+    SP_OPT_GEMM_SCHEDULE = 9, /* tensor-core projections: 0 = automatic, 1 = one
+                                 CTA per (weight tile, K split), 2 = persistent
+                                 stream-K (one CTA per SM, an even share of the
+                                 (tile, k-block) units each) wherever its partial
+                                 planes fit the handle's scratch.  Changes the
+                                 work split only, never the result beyond the
+                                 order of the fp32 partial sums                 */
+    SP_OPT_ATTN_MERGE = 10    /* tensor-core attention: where the partials of a
+                                 (sequence, kv head) split over several CTAs are
+                                 merged: 0 = automatic, 1 = inside the attention
+                                 kernel (by the CTA that completes the pair),
+                                 2 = in a second kernel over (head, sequence,
+                                 query row).  Both merge in segment order        */
 };
 
 /* Stages of sp_classify, in launch order. */

@@ -94,6 +94,7 @@ struct sp_handle {
     int opt_seg_cost = -1;  // attention segment-boundary cost in tiles (-1 = default)
     int opt_prec = 0;       // activation precision of the MLP inputs (SP_OPT_ACT_PRECISION)
     int opt_stall = 0;      // one-shot failure-path test (SP_OPT_DEBUG_STALL)
+    int opt_merge = 0;      // where the attention partials are merged (SP_OPT_ATTN_MERGE)
     int *dbg_pages = nullptr;     // sp_debug_gathered_pages: recording buffer (device)
     size_t dbg_pages_cap = 0;     // its capacity in ints
     int T = 1;        // tasks sharing the pass; cfg.k_rows holds T * k_task rows per sequence
@@ -216,13 +217,13 @@ int *attention_counters(void *ws) { return (int *)ws; }
 sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_path, int n_sm,
                             int forced_split, int *launches, cudaStream_t st, bool counters_zeroed,
                             cudaEvent_t *ev_attn = nullptr, cudaEvent_t *ev_merge = nullptr,
-                            int seg_cost = -1) {
+                            int seg_cost = -1, int merge_mode = 0) {
     a.tc_ctas = attn_tc_ctas(n_sm, a.Hkv);
     a.tc_min_tiles = forced_split > 0 ? forced_split / 64 : kAttnMinTiles;
     a.tc_seg_cost = seg_cost >= 0 ? seg_cost : kAttnSegCost;
     // few sequences over many groups: each pair has many partials, merged by a
     // kernel spread over (head, sequence, row) instead of one CTA per pair
-    a.tc_merge_kernel = 4 * a.B < a.tc_ctas / a.Hkv;
+    a.tc_merge_kernel = merge_mode == 2 || (merge_mode == 0 && 4 * a.B < a.tc_ctas / a.Hkv);
     const size_t need = attention_workspace_bytes(a.B, a.Hkv, a.R, a.dh, a.n_splits, n_sm);
     if (ws_bytes < need) return fail(SP_ERR_INVALID_ARG, "attention workspace too small (%zu < %zu)", ws_bytes, need);
     const size_t pairs = (size_t)a.B * a.Hkv;
@@ -530,6 +531,14 @@ sp_status sp_set_option(sp_handle *h, int key, int value) {
         if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad activation precision");
         h->opt_prec = value;
         return SP_OK;
+    case SP_OPT_ATTN_MERGE:
+        if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad attention merge mode");
+        h->opt_merge = value;
+        return SP_OK;
+    case SP_OPT_GEMM_SCHEDULE:
+        if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad gemm schedule");
+        h->gemm.sched = value;
+        return SP_OK;
     case SP_OPT_ATTN_SEG_COST:
         if (value < -1 || value > 1024) return fail(SP_ERR_INVALID_ARG, "bad segment cost");
         h->opt_seg_cost = value;
@@ -795,7 +804,8 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     s = enqueue_attention(a, h->attn_ws, h->attn_ws_bytes, h->opt_attn, h->n_sm, h->opt_split,
                           &launches, st, true,
                           h->opt_profile ? h->ev[SP_STAGE_ATTN] : nullptr,
-                          h->opt_profile ? h->ev[SP_STAGE_MERGE] : nullptr, h->opt_seg_cost);
+                          h->opt_profile ? h->ev[SP_STAGE_MERGE] : nullptr, h->opt_seg_cost,
+                          h->opt_merge);
     if (s != SP_OK) return s;
     if (h->opt_profile) h->ev_used[SP_STAGE_ATTN] = h->ev_used[SP_STAGE_MERGE] = true;
 

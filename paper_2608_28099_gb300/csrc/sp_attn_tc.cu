@@ -15,10 +15,13 @@
 // each of its segments leaves an unnormalised partial (max, sum, O) in slot
 // (j + b) Hkv + g (unique: segments are ordered by both j and b), and the CTA
 // that completes the pair's last segment (a counter per pair, zero before the
-// launch) combines the partials in the exp2 domain, in segment order, in that
-// segment's epilogue.  The cuts between shares weigh every sequence start as
-// a number of tiles (the cost of a segment boundary), so shares with more
-// boundaries hold fewer tiles.
+// launch) combines the partials in the exp2 domain, in segment order: in that
+// segment's epilogue, or, when it is the last segment of the CTA's share (the
+// usual case: such segments end with the kernel), after every role has
+// finished, by all 384 threads, with the partials staged through the idle K/V
+// ring in one round of copies.  The cuts between shares weigh every sequence
+// start as a number of tiles (the cost of a segment boundary), so shares with
+// more boundaries hold fewer tiles.
 //
 // All R = G * k query rows of the KV head's group share every K/V tile: the
 // GQA group and the k soft-prompt rows together form the M side of the MMA.
@@ -91,6 +94,7 @@ constexpr int SMEM_BYTES = OFF_SEQ + MAX_B * 8 + 1024;
 constexpr int THREADS = 384;                   // 2 softmax warpgroups, 2 producers, 2 MMA
 constexpr int PRODUCER_WARP = 8, MMA_WARP = 9, MMA_WARP1 = 10, PRODUCER_WARP1 = 11;
 constexpr float RESCALE_LOG2 = 8.f;            // tolerate p <= 2^8 before rescaling O
+constexpr int kStagedSegs = 4;                 // most partials merged through the idle ring
 // TMEM columns: S0 [0,64) S1 [64,128) O0 [128,256) O1 [256,384) Qhi [384,448) Qlo [448,512);
 // P_w (64 bf16 per row) overwrites the first 32 columns of S_w once S_w is read.
 constexpr uint32_t TMEM_COLS = 512;
@@ -122,6 +126,8 @@ struct Bars {
     uint32_t tmem;
     int abort;
     int merge_now;             // this segment completed its pair: merge it in the epilogue
+    int fm_merge, fm_b, fm_nseg;  // the share's last segment completed its pair: merged at the end
+    long long fm_slot0;           // partial slot of the pair's first segment
     int wsum[THREADS / 32];    // tile-prefix scan
 };
 static_assert(sizeof(Bars) <= 512, "barrier block");
@@ -291,6 +297,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         mbar_init(&bars->q_full, 1);
         bars->abort = 0;
         bars->merge_now = 0;
+        bars->fm_merge = 0;
         fence_mbar_init();
         if (paged) {
             prefetch_tmap(&map_k);
@@ -773,6 +780,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 // partials here, in segment order (the result does not depend on
                 // which CTA finishes last), while its own are still in L2
                 const int n_seg = j_last - j_first + 1;
+                const int staged_max = min(kStagedSegs, (STG * KV_STAGE) / (R * (DH * 4 + 8)));
                 __threadfence();  // this segment's partial is visible before it is counted
                 named_sync(BAR_EPI, n_cons);
                 if (ct == 0) {
@@ -782,9 +790,18 @@ __global__ void __launch_bounds__(THREADS, 1)
                     bars->merge_now = last;
                 }
                 named_sync(BAR_EPI, n_cons);
-                if (bars->merge_now && have && active) {
+                const size_t slot0 = ((size_t)j_first + b) * Hkv + g;  // segment e: + e Hkv
+                if (bars->merge_now && x >= x1 && n_seg <= staged_max) {
+                    // the share's last segment: merged by the whole CTA once every
+                    // role is done (below), through the idle K/V ring
+                    if (ct == 0) {
+                        bars->fm_b = b;
+                        bars->fm_nseg = n_seg;
+                        bars->fm_slot0 = (long long)slot0;
+                        bars->fm_merge = 1;
+                    }
+                } else if (bars->merge_now && have && active) {
                     __threadfence();  // the other segments' partials are read after their count
-                    const size_t slot0 = ((size_t)j_first + b) * Hkv + g;  // segment e: + e Hkv
 #pragma unroll 1
                     for (int c0 = wg * (DH / 2); c0 < (wg + 1) * (DH / 2); c0 += 32) {
                         float acc[32], mm = -INFINITY, ll = 0.f;
@@ -838,6 +855,78 @@ __global__ void __launch_bounds__(THREADS, 1)
     tc_fence_before();
     __syncthreads();
     if (threadIdx.x == 0 && *abort && a.status) atomicOr(a.status, SP_DEV_TIMEOUT);
+    if (bars->fm_merge) {
+        // Merge of the pair completed by this share's last segment, by all 384
+        // threads: every partial of the pair lands in the idle K/V ring in one
+        // round of cp.async copies (O of segment e as [e][row][dh], then (max,
+        // sum) as [e][row]), then thread (row, c) combines 16-byte units c, c + 8,
+        // c + 16, c + 24 of its row in segment order, in the arithmetic of the
+        // register merge above, so the bits do not depend on which path ran.
+        // Shared-memory reads are conflict-free and eight lanes store 64
+        // contiguous bytes per plane.  Loads through registers would need a
+        // dependent round trip per two segments, each waiting behind the other
+        // SMs' cache streams.
+        const int b = bars->fm_b, n_seg = bars->fm_nseg;
+        const size_t slot0 = (size_t)bars->fm_slot0;
+        const bool good = !*abort;  // every wait is over: uniform
+        __threadfence();            // the other segments' partials are read after their count
+        uint8_t *stage = smem + OFF_KV;
+        float2 *st_ml = (float2 *)(stage + (size_t)n_seg * R * DH * 4);
+        const int units = R * (DH / 4);  // 16-byte units of one segment's O
+        for (int idx = threadIdx.x; idx < n_seg * units; idx += THREADS) {
+            const int e = idx / units, rem = idx - e * units;
+            cp_async16(stage + (size_t)idx * 16, a.part_o + (slot0 + (size_t)e * Hkv) * R * DH + (size_t)rem * 4);
+        }
+        for (int idx = threadIdx.x; idx < n_seg * R; idx += THREADS) {
+            const int e = idx / R, rr = idx - e * R;
+            st_ml[idx] = __ldcg((const float2 *)(a.part_ml + ((slot0 + (size_t)e * Hkv) * R + rr) * 2));
+        }
+        asm volatile("cp.async.wait_all;" ::: "memory");
+        __syncthreads();
+        if (good) {
+            for (int item = threadIdx.x; item < R * 8; item += THREADS) {
+                const int rr = item >> 3, c = item & 7;
+                float2 ml[kStagedSegs];
+                float4 ov[kStagedSegs][4];
+#pragma unroll
+                for (int e = 0; e < kStagedSegs; ++e) {
+                    const int ee = min(e, n_seg - 1);
+                    ml[e] = st_ml[ee * R + rr];
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        ov[e][q] = ld_shared_v4f(stage + (((size_t)ee * R + rr) * (DH / 4) + c + 8 * q) * 16);
+                }
+                float acc[16], mm = -INFINITY, ll = 0.f;
+#pragma unroll
+                for (int j = 0; j < 16; ++j) acc[j] = 0.f;
+#pragma unroll
+                for (int e = 0; e < kStagedSegs; ++e) {
+                    if (e >= n_seg) break;
+                    const float mn = fmaxf(mm, ml[e].x);
+                    if (mn == -INFINITY) continue;
+                    const float al = mm == -INFINITY ? 0.f : exp2f(mm - mn);
+                    const float wt = ml[e].x == -INFINITY ? 0.f : exp2f(ml[e].x - mn);
+                    ll = ll * al + wt * ml[e].y;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        acc[4 * q] = acc[4 * q] * al + wt * ov[e][q].x;
+                        acc[4 * q + 1] = acc[4 * q + 1] * al + wt * ov[e][q].y;
+                        acc[4 * q + 2] = acc[4 * q + 2] * al + wt * ov[e][q].z;
+                        acc[4 * q + 3] = acc[4 * q + 3] * al + wt * ov[e][q].w;
+                    }
+                    mm = mn;
+                }
+                const float il = ll > 0.f ? 1.f / ll : 0.f;
+                const int hl = rr / k, r = rr - hl * k;
+                const size_t o0 = (((size_t)b * k + r) * a.Hq + g * a.G + hl) * DH;
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    act_store4(a.out, o0 + (size_t)(c + 8 * q) * 4,
+                               make_float4(acc[4 * q] * il, acc[4 * q + 1] * il, acc[4 * q + 2] * il,
+                                           acc[4 * q + 3] * il));
+            }
+        }
+    }
     // the cache stream of the slower CTAs leaves DRAM time for the next
     // projection's weights: this CTA's share goes to L2 (the K/V tiles were
     // loaded evict-first, so the weights stay)

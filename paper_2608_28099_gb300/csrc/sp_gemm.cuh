@@ -30,7 +30,10 @@ bool tc_supported(int N, int K);
 // Rows per tile for M activation rows: 16..128, or 256 (plain bf16 only: the
 // MMA's N side is then 256) for M >= 256.
 int tc_bn_for(int M, bool lo = true);
-TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo = true);
+// sched: 0 = automatic, 1 = tile kernel, 2 = persistent stream-K (when its
+// partial planes fit).
+TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo = true,
+               int sched = 0);
 // w_blocked: the weights are stored blocked (block_weights_layout) and map_w
 // views them as [N K / 64][64] rows.
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
@@ -119,6 +122,7 @@ inline void init_act(ActBuf &a, void *ptr, int rows_max, int K, bool want_maps) 
 struct GemmPlanner {
     int n_sm = 148;
     size_t y_capacity = 0;  // bytes available for [splits][M][N] partials
+    int sched = 0;          // SP_OPT_GEMM_SCHEDULE
     void init(int sms, size_t cap) {
         n_sm = sms;
         y_capacity = cap;
@@ -134,7 +138,7 @@ struct GemmPlanner {
                   int inject_stall = 0) const {
         cudaError_t e;
         if (use_tc(w, x, path)) {
-            const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo);
+            const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched);
             const int bi = bn_index(p.bn);
             e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked, lo,
                                inject_stall);

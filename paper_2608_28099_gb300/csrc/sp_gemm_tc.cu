@@ -567,7 +567,7 @@ static int planes_for(long long tiles, int n_kb, long long L) {
     return most;
 }
 
-TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo) {
+TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo, int sched) {
     TcPlan p;
     p.bn = tc_bn_for(M, lo);
     p.m_tiles = ceil_div(M, p.bn);
@@ -593,7 +593,8 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo) 
     // (estimates in units of one CTA's k-block time, 16 KB of weights).
     const int waves = ceil_div(tiles * p.splits, n_sm);
     const double fill = (double)tiles * p.splits / ((double)waves * n_sm);
-    if (waves > 1 && fill < 0.8) {
+    if (sched == 1) return p;
+    if (sched == 2 || (waves > 1 && fill < 0.8)) {
         const long long U = (long long)tiles * p.n_kb;
         long long L = (U + n_sm - 1) / n_sm;
         if (L < 2) L = 2;
@@ -601,7 +602,7 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo) 
         const double plane_units = 2.0 * (double)M * N * 4.0 / ((double)n_sm * 16384.0);
         const double cost_tile = (double)waves * (p.kb_per_split + 4);
         const double cost_pk = (double)L + 4.0 + planes * plane_units;
-        if (cost_pk < cost_tile && (size_t)planes * M * N * sizeof(float) <= y_capacity_bytes) {
+        if ((sched == 2 || cost_pk < cost_tile) && (size_t)planes * M * N * sizeof(float) <= y_capacity_bytes) {
             p.persistent = true;
             p.units_per_cta = (int)L;
             p.splits = planes;

@@ -191,6 +191,14 @@ __device__ __forceinline__ void st_shared_v4(void *p, uint32_t a, uint32_t b, ui
                  : "memory");
 }
 
+__device__ __forceinline__ float4 ld_shared_v4f(const void *p) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(smem_u32(p)));
+    return v;
+}
+
 // ---- tcgen05 ---------------------------------------------------------------
 // Allocate `ncols` TMEM columns (power of two >= 32); warp-wide.
 __device__ __forceinline__ void tmem_alloc(uint32_t *slot, uint32_t ncols) {
