@@ -289,7 +289,12 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     const int d = c.d_model, hq = c.n_q_heads, hkv = c.n_kv_heads, dh = c.head_dim, f = c.d_ff;
     const int k = c.k_rows, C = c.n_classes;
     h->nqkv = (hq + 2 * hkv) * dh;
-    h->gu_blk = f;  // gate block then up block (no interleave)
+    // [W_gate; W_up] for the tensor cores: 64-row blocks interleaved (gate rows
+    // 64i.., then the matching up rows), so that one 128-row weight tile holds
+    // both halves of 64 SwiGLU features and the gate/up projection can apply
+    // SwiGLU in its epilogue; otherwise the gate block then the up block
+    const bool gu_tc = c.w_dtype == SP_BF16 && tc_supported(2 * f, d) && f % 64 == 0;
+    h->gu_blk = gu_tc ? 64 : f;
     const size_t es = h->es;
     auto cleanup = [&](sp_status s) {
         sp_destroy(h);
@@ -324,8 +329,14 @@ sp_status sp_create(const sp_config *cfg, const sp_weights *w, sp_handle **out) 
     }
     {
         std::vector<char> buf((size_t)2 * f * d * es);
-        memcpy(buf.data(), w->w_gate, (size_t)f * d * es);
-        memcpy(buf.data() + (size_t)f * d * es, w->w_up, (size_t)f * d * es);
+        const int blk = h->gu_blk;
+        const size_t rowb = (size_t)d * es;
+        for (int i = 0; i < f / blk; ++i) {
+            memcpy(buf.data() + (size_t)2 * i * blk * rowb, (const char *)w->w_gate + (size_t)i * blk * rowb,
+                   (size_t)blk * rowb);
+            memcpy(buf.data() + (size_t)(2 * i + 1) * blk * rowb, (const char *)w->w_up + (size_t)i * blk * rowb,
+                   (size_t)blk * rowb);
+        }
         if ((st = upload_weight(h->w_gu, buf.data(), 2 * f, d)) != SP_OK) return cleanup(st);
     }
     if ((st = upload_weight(h->w_o, (const char *)w->w_o, d, hq * dh)) != SP_OK) return cleanup(st);
@@ -824,15 +835,21 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
                                  c.rms_eps, M, d, h->h1, h->n.out(tc_gu, mlp_lo), st));
     mark(SP_STAGE_POST_NORM, 1);
     ++launches;
-    // a5: gate/up + SwiGLU
+    // a5: gate/up + SwiGLU: in the projection's epilogue when it runs one CTA
+    // per weight tile (no K split), else a separate kernel over the partials
+    const ActOut a_out = h->a.out(tc_down, mlp_lo);
+    const bool glu = h->gu_blk == 64 && h->gemm.glu_fusable(h->w_gu, h->n, h->opt_gemm, M, mlp_lo);
     mark(SP_STAGE_GATE_UP, 0);
-    s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, M, h->status, st, &launches, &ns, mlp_lo);
+    s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, M, h->status, st, &launches, &ns, mlp_lo, 0,
+                    glu ? &a_out : nullptr);
     mark(SP_STAGE_GATE_UP, 1);
     if (s != SP_OK) return fail(s, "gate/up projection launch failed");
-    mark(SP_STAGE_SWIGLU, 0);
-    SP_CUDA(launch_swiglu(PartIn{h->y, ns, (size_t)M * 2 * f}, M, f, h->gu_blk, h->a.out(tc_down, mlp_lo), st));
-    mark(SP_STAGE_SWIGLU, 1);
-    ++launches;
+    if (!glu) {
+        mark(SP_STAGE_SWIGLU, 0);
+        SP_CUDA(launch_swiglu(PartIn{h->y, ns, (size_t)M * 2 * f}, M, f, h->gu_blk, a_out, st));
+        mark(SP_STAGE_SWIGLU, 1);
+        ++launches;
+    }
     // a6-a7: down projection + residual, pooling, linear head
     mark(SP_STAGE_DOWN, 0);
     s = h->gemm.run(wb, h->opt_gemm, h->a, h->w_down, h->y, M, h->status, st, &launches, &ns, mlp_lo);

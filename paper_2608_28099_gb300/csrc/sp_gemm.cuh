@@ -39,7 +39,7 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo =
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
                            float *y, int *status, cudaStream_t st, bool w_blocked = false,
-                           bool lo = true, int inject_stall = 0);
+                           bool lo = true, int inject_stall = 0, const ActOut *glu = nullptr);
 
 // Weights [N][K] (es bytes per element) re-laid out as contiguous 16 KB blocks
 // [N / 128][K / 64][128][64]: one weight tile's k-block is one sequential read
@@ -132,16 +132,24 @@ struct GemmPlanner {
     bool use_tc(const WeightMat &w, const ActBuf &x, int path) const {
         return path != 1 && w.tc && x.maps;
     }
+    // Would the gate/up projection ([gate block; up block] per 128-row tile)
+    // run with the SwiGLU epilogue (one CTA per tile, no K split)?
+    bool glu_fusable(const WeightMat &w, const ActBuf &x, int path, int M, bool lo) const {
+        if (!use_tc(w, x, path)) return false;
+        const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched);
+        return !p.persistent && p.splits == 1 && p.bn >= 32;
+    }
     // Enqueue the projection; *nsplit receives the number of partials in y.
+    // glu: write silu(gate) * up there instead of partials (glu_fusable).
     sp_status run(int w_bf16, int path, const ActBuf &x, const WeightMat &w, float *y, int M,
                   int *status, cudaStream_t st, int *launches, int *nsplit, bool lo = true,
-                  int inject_stall = 0) const {
+                  int inject_stall = 0, const ActOut *glu = nullptr) const {
         cudaError_t e;
         if (use_tc(w, x, path)) {
             const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched);
             const int bi = bn_index(p.bn);
             e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked, lo,
-                               inject_stall);
+                               inject_stall, glu);
             *nsplit = p.splits;
         } else {
             e = launch_gemm_simt(w_bf16, x.ptr, w.ptr, y, M, w.N, w.K, st, w.blocked);

@@ -18,7 +18,9 @@
 // Two schedules, fp32 partials in planes of Y that the consumers add:
 //  * tile kernel: one CTA per (tile, K split); split-K when the tiles alone
 //    leave SMs idle.  Roles: warp 0 lane 0 TMA, warp 1 lane 0 MMA, warp 2
-//    TMEM, all four warps the epilogue (warp w: TMEM lanes 32w..32w+31).
+//    TMEM, all eight warps the epilogue (warp w: TMEM lanes 32 (w & 3).., the
+//    column chunks of half w >> 2).  A gate/up projection with one K split can
+//    apply SwiGLU in the epilogue instead of writing partials.
 //  * persistent stream-K kernel, for tile counts that fill the SMs badly:
 //    one CTA per SM owns the contiguous (tile, k-block) units [c L, (c+1) L)
 //    in tile-major order.  Its weight and activation rings run across tile
@@ -68,10 +70,17 @@ struct TcArgs {
     // MMA warp's wait runs out; every wait of the launch gives up after wait_ns
     int inject_stall;
     unsigned long long wait_ns;
+    // SwiGLU epilogue (glu_f > 0, one K split): weight tile t holds gate rows
+    // 64t..64t+63 then the matching up rows, and the CTA writes
+    // glu[m][64t + j] = silu(gate) * up instead of a partial plane
+    int glu_f;
+    ActOut glu;
 };
 
+constexpr int TILE_THREADS = 256;  // warps 0-2 also TMA, MMA and TMEM owner
+
 template <int BN, bool LO>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(TILE_THREADS, 1)
     gemm_tile_kernel(const __grid_constant__ CUtensorMap map_w,
                    const __grid_constant__ CUtensorMap map_xhi,
                    const __grid_constant__ CUtensorMap map_xlo, TcArgs g) {
@@ -171,22 +180,64 @@ __global__ void __launch_bounds__(128, 1)
     // epilogue: TMEM -> registers -> fp32 partial tile
     const bool have = mbar_wait_drain(done, 0) && !*abort;
     tc_fence_after();
-    if (have) {
-        const int n = n0 + warp * 32 + lane;
-        float *y = g.y + (size_t)blockIdx.z * g.split_stride;
-        const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
-        if constexpr (BN == 16) {
-            float v[16], u[16] = {};
-            tmem_ld16(trow, v);
-            if (LO) tmem_ld16(trow + 16, u);
+    // epilogue over all eight warps: warp w reads TMEM lanes 32 (w & 3).. and
+    // the column chunks of half w >> 2
+    const int quad = warp & 3, half = warp >> 2;
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+    if (g.glu_f) {
+        if constexpr (BN >= 32) {
+            // SwiGLU epilogue, per 64-column chunk: every warp puts 32 columns of
+            // its 32 rows (TMEM lanes) into the idle ring as [column][132] fp32
+            // (two buffers), then thread (fq, cg) forms features 4 fq..4 fq + 3
+            // of columns 4 cg..4 cg + 3 from gate rows 4 fq.. and up rows
+            // 64 + 4 fq..: 16-byte shared loads, four features per store
+            float *xb = (float *)smem;
+            const int row = quad * 32 + lane, fq = threadIdx.x & 15, cg = threadIdx.x >> 4;
+            const size_t feat = (size_t)blockIdx.y * 64 + 4 * fq;
+#pragma unroll 1
+            for (int c0 = 0; c0 < BN; c0 += 64) {
+                float *buf = xb + ((c0 >> 6) & 1) * (64 * 132);
+                if (have && c0 + half * 32 < BN) {
+                    float v[32], u[32] = {};
+                    tmem_ld32(trow + c0 + half * 32, v);
+                    if (LO) tmem_ld32(trow + BN + c0 + half * 32, u);
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                const int m = m0 + j;
-                if (m < g.M) y[(size_t)m * g.N + n] = v[j] + u[j];
+                    for (int j = 0; j < 32; ++j) buf[(half * 32 + j) * 132 + row] = v[j] + u[j];
+                }
+                __syncthreads();
+                if (have) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int cc = 4 * cg + e, m = m0 + c0 + cc;
+                        if (c0 + cc >= BN || m >= g.M) break;
+                        const float4 gt = ld_shared_v4f(buf + cc * 132 + 4 * fq);
+                        const float4 up = ld_shared_v4f(buf + cc * 132 + 64 + 4 * fq);
+                        act_store4(g.glu, (size_t)m * g.glu_f + feat,
+                                   make_float4(__fdividef(gt.x, 1.f + __expf(-gt.x)) * up.x,
+                                               __fdividef(gt.y, 1.f + __expf(-gt.y)) * up.y,
+                                               __fdividef(gt.z, 1.f + __expf(-gt.z)) * up.z,
+                                               __fdividef(gt.w, 1.f + __expf(-gt.w)) * up.w));
+                    }
+                }
+            }
+        }
+    } else if (have) {
+        const int n = n0 + quad * 32 + lane;
+        float *y = g.y + (size_t)blockIdx.z * g.split_stride;
+        if constexpr (BN == 16) {
+            if (half == 0) {
+                float v[16], u[16] = {};
+                tmem_ld16(trow, v);
+                if (LO) tmem_ld16(trow + 16, u);
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const int m = m0 + j;
+                    if (m < g.M) y[(size_t)m * g.N + n] = v[j] + u[j];
+                }
             }
         } else {
 #pragma unroll 1
-            for (int c0 = 0; c0 < BN; c0 += 32) {
+            for (int c0 = half * 32; c0 < BN; c0 += 64) {
                 float v[32], u[32] = {};
                 tmem_ld32(trow + c0, v);
                 if (LO) tmem_ld32(trow + BN + c0, u);
@@ -220,7 +271,7 @@ cudaError_t launch_tile(const CUtensorMap &mw, const CUtensorMap &mh, const CUte
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    return launch_k(gemm_tile_kernel<BN, LO>, grid, dim3(128), (size_t)smem, st, mw, mh, ml, g);
+    return launch_k(gemm_tile_kernel<BN, LO>, grid, dim3(TILE_THREADS), (size_t)smem, st, mw, mh, ml, g);
 }
 
 
@@ -615,7 +666,7 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo, 
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
                            float *y, int *status, cudaStream_t st, bool w_blocked, bool lo,
-                           int inject_stall) {
+                           int inject_stall, const ActOut *glu) {
     if (p.persistent) {
         PkArgs g;
         g.M = M;
@@ -655,6 +706,13 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
     g.status = status;
     g.inject_stall = inject_stall;
     g.wait_ns = inject_stall ? 1000000ull : sm100::kWaitLimitNs;
+    g.glu_f = 0;
+    memset(&g.glu, 0, sizeof g.glu);
+    if (glu) {
+        if (p.persistent || p.splits != 1 || p.bn < 32 || N % 128) return cudaErrorInvalidValue;
+        g.glu_f = N / 2;
+        g.glu = *glu;
+    }
     dim3 grid(p.m_tiles, p.n_tiles, p.splits);
     switch (p.bn) {
     case 16: return lo ? launch_tile<16, true>(map_w, map_xhi, map_xlo, g, grid, st)

@@ -167,7 +167,7 @@ __global__ void swiglu_kernel(PartIn y, int M, int f, int blk, ActOut a) {
         const float gx[4] = {g.x, g.y, g.z, g.w}, ux[4] = {u.x, u.y, u.z, u.w};
         float r[4];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) r[e] = gx[e] / (1.f + __expf(-gx[e])) * ux[e];
+        for (int e = 0; e < 4; ++e) r[e] = __fdividef(gx[e], 1.f + __expf(-gx[e])) * ux[e];
         act_store4(a, (size_t)idx, make_float4(r[0], r[1], r[2], r[3]));
     }
 }
