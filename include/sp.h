@@ -255,13 +255,14 @@ enum {
                                  between CTA shares balance (-1..1024); -1 = the
                                  built-in default.  Changes the work split only,
                                  never the result beyond rounding order          */
-    SP_OPT_ACT_PRECISION = 7, /* activations fed to the tensor-core MLP
-                                 projections (gate/up and down): 0 = automatic
-                                 (plain bf16 when pool is SP_POOL_MEAN and at
-                                 least 8 rows per task are pooled, else bf16
-                                 hi + lo planes, ~16 mantissa bits), 1 = hi + lo
-                                 always, 2 = plain bf16 always.  The Q/K/V and
-                                 output projections always take hi + lo        */
+    SP_OPT_ACT_PRECISION = 7, /* activations fed to the tensor-core
+                                 projections: 0 = automatic (with pool
+                                 SP_POOL_MEAN, plain bf16 for gate/up and down
+                                 from 8 rows per task pooled, and for Q/K/V and
+                                 output too from 16; bf16 hi + lo planes, ~16
+                                 mantissa bits, otherwise), 1 = hi + lo always,
+                                 2 = plain bf16 for gate/up and down, hi + lo
+                                 for Q/K/V and output, 3 = plain bf16 always    */
     SP_OPT_DEBUG_STALL = 8,   /* test of the failure path: 1 = in the next
                                  sp_classify only, the first CTA of the output
                                  projection (when it runs on the one-CTA-per-tile
