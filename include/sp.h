@@ -256,13 +256,13 @@ enum {
                                  built-in default.  Changes the work split only,
                                  never the result beyond rounding order          */
     SP_OPT_ACT_PRECISION = 7, /* activations fed to the tensor-core
-                                 projections: 0 = automatic (with pool
-                                 SP_POOL_MEAN, plain bf16 for gate/up and down
-                                 from 8 rows per task pooled, and for Q/K/V and
-                                 output too from 16; bf16 hi + lo planes, ~16
-                                 mantissa bits, otherwise), 1 = hi + lo always,
-                                 2 = plain bf16 for gate/up and down, hi + lo
-                                 for Q/K/V and output, 3 = plain bf16 always    */
+                                 projections: 0 = automatic (gate/up and down
+                                 take plain bf16 when pool is SP_POOL_MEAN and
+                                 at least 8 rows per task are pooled, else bf16
+                                 hi + lo planes, ~16 mantissa bits; Q/K/V and
+                                 output take hi + lo), 1 = hi + lo always, 2 =
+                                 plain bf16 for gate/up and down, 3 = plain bf16
+                                 always, 4 = plain bf16 except Q/K/V            */
     SP_OPT_DEBUG_STALL = 8,   /* test of the failure path: 1 = in the next
                                  sp_classify only, the first CTA of the output
                                  projection (when it runs on the one-CTA-per-tile
@@ -280,12 +280,17 @@ enum {
                                  planes fit the handle's scratch.  Changes the
                                  work split only, never the result beyond the
                                  order of the fp32 partial sums                 */
-    SP_OPT_ATTN_MERGE = 10    /* tensor-core attention: where the partials of a
+    SP_OPT_ATTN_MERGE = 10,   /* tensor-core attention: where the partials of a
                                  (sequence, kv head) split over several CTAs are
                                  merged: 0 = automatic, 1 = inside the attention
                                  kernel (by the CTA that completes the pair),
                                  2 = in a second kernel over (head, sequence,
                                  query row).  Both merge in segment order        */
+    SP_OPT_QUERY_PRECISION = 11 /* tensor-core attention: queries as 0 =
+                                 automatic (plain bf16 when pool is
+                                 SP_POOL_MEAN and at least 16 rows per task are
+                                 pooled, else hi + lo), 1 = bf16 hi + lo (two
+                                 score MMAs per step), 2 = plain bf16 (one)     */
 };
 
 /* Stages of sp_classify, in launch order. */

@@ -26,6 +26,7 @@ SP_OPT_ACT_PRECISION = 7
 SP_OPT_DEBUG_STALL = 8
 SP_OPT_GEMM_SCHEDULE = 9
 SP_OPT_ATTN_MERGE = 10
+SP_OPT_QUERY_PRECISION = 11
 STAGES = ["input_norm", "qkv", "rope", "attention", "merge", "o_proj", "post_norm", "gate_up",
           "swiglu", "down", "readout", "fusion"]
 

@@ -95,6 +95,7 @@ struct sp_handle {
     int opt_prec = 0;       // activation precision of the MLP inputs (SP_OPT_ACT_PRECISION)
     int opt_stall = 0;      // one-shot failure-path test (SP_OPT_DEBUG_STALL)
     int opt_merge = 0;      // where the attention partials are merged (SP_OPT_ATTN_MERGE)
+    int opt_qprec = 0;      // attention query precision (SP_OPT_QUERY_PRECISION)
     int *dbg_pages = nullptr;     // sp_debug_gathered_pages: recording buffer (device)
     size_t dbg_pages_cap = 0;     // its capacity in ints
     int T = 1;        // tasks sharing the pass; cfg.k_rows holds T * k_task rows per sequence
@@ -539,8 +540,12 @@ sp_status sp_set_option(sp_handle *h, int key, int value) {
         h->opt_stall = value;
         return SP_OK;
     case SP_OPT_ACT_PRECISION:
-        if (value < 0 || value > 3) return fail(SP_ERR_INVALID_ARG, "bad activation precision");
+        if (value < 0 || value > 4) return fail(SP_ERR_INVALID_ARG, "bad activation precision");
         h->opt_prec = value;
+        return SP_OK;
+    case SP_OPT_QUERY_PRECISION:
+        if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad query precision");
+        h->opt_qprec = value;
         return SP_OK;
     case SP_OPT_ATTN_MERGE:
         if (value < 0 || value > 2) return fail(SP_ERR_INVALID_ARG, "bad attention merge mode");
@@ -726,12 +731,16 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     int ns = 1;
     // The MLP inputs (the post-norm n and the SwiGLU output a) go to the tensor
     // cores as plain bf16 when the head averages at least 8 rows per pooled
-    // state, and the Q/K/V and output projection inputs (x_hat, o) too from 16
-    // rows on (the rows' independent rounding errors average out in the mean;
-    // the measured budget is in the design notes); else as hi + lo planes.
+    // state (the rows' independent rounding errors average out in the mean;
+    // the measured budget is in the design notes), else as hi + lo planes; the
+    // Q/K/V and output projection inputs (x_hat, o) as hi + lo unless an option
+    // asks otherwise, and the attention's queries as plain bf16 from 16 pooled
+    // rows on.
     const bool mean = c.pool == SP_POOL_MEAN;
     const bool mlp_lo = h->opt_prec == 1 || (h->opt_prec == 0 && !(mean && h->k_task >= 8));
-    const bool proj_lo = h->opt_prec == 1 || h->opt_prec == 2 || (h->opt_prec == 0 && !(mean && h->k_task >= 16));
+    const bool proj_lo = h->opt_prec != 3 && h->opt_prec != 4;
+    const bool qkv_lo = h->opt_prec != 3;
+    const bool q_plain = h->opt_qprec == 2 || (h->opt_qprec == 0 && mean && h->k_task >= 16);
 
     // a1-a2: pre-norm, Q/K/V projection, rotation at positions L_b + r
     PartIn yqkv = {h->qkv_shared, 1, 0};
@@ -748,21 +757,21 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         if (s != SP_OK) return fail(s, "fusion projection launch failed");
         mark(SP_STAGE_INPUT_NORM, 0);
         SP_CUDA(launch_residual_norm(0, PartIn{h->y, ns_fc, (size_t)batch * d}, h->fc_prompt, k,
-                                     h->g_in, c.rms_eps, M, d, h->xrows, h->xn.out(tc_qkv, proj_lo), st, k));
+                                     h->g_in, c.rms_eps, M, d, h->xrows, h->xn.out(tc_qkv, qkv_lo), st, k));
         mark(SP_STAGE_INPUT_NORM, 1);
         ++launches;
         mark(SP_STAGE_QKV, 0);
-        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, proj_lo);
+        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, qkv_lo);
         mark(SP_STAGE_QKV, 1);
         if (s != SP_OK) return fail(s, "Q/K/V projection launch failed");
         yqkv = PartIn{h->y, ns, stride_qkv};
     } else if (d_rows) {
         mark(SP_STAGE_INPUT_NORM, 0);
-        SP_CUDA(launch_rmsnorm_rows(wb, d_rows, 0, h->g_in, c.rms_eps, M, d, h->xn.out(tc_qkv, proj_lo), st));
+        SP_CUDA(launch_rmsnorm_rows(wb, d_rows, 0, h->g_in, c.rms_eps, M, d, h->xn.out(tc_qkv, qkv_lo), st));
         mark(SP_STAGE_INPUT_NORM, 1);
         ++launches;
         mark(SP_STAGE_QKV, 0);
-        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, proj_lo);
+        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, qkv_lo);
         mark(SP_STAGE_QKV, 1);
         if (s != SP_OK) return fail(s, "Q/K/V projection launch failed");
         yqkv = PartIn{h->y, ns, stride_qkv};
@@ -809,6 +818,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         a.gathered = h->dbg_pages;
     }
     a.scale_log2 = (float)(1.4426950408889634 / sqrt((double)dh));
+    a.tc_q_plain = q_plain;
     a.out = h->o.out(tc_o, proj_lo);
     if (tc_o) {  // the output projection's weights, prefetched by the attention's early finishers
         a.l2_next = h->w_o.ptr;

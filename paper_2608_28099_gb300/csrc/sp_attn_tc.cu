@@ -511,7 +511,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                     // 16 dims of Q = 8 TMEM columns
                     mma_bf16_ts(s_tmem, tmem + QHI_COL + (uint32_t)(kk * 8), bk, idesc_s,
                                 kk > 0 ? 1u : 0u);
-                    mma_bf16_ts(s_tmem, tmem + QLO_COL + (uint32_t)(kk * 8), bk, idesc_s, 1u);
+                    if (!a.tc_q_plain)
+                        mma_bf16_ts(s_tmem, tmem + QLO_COL + (uint32_t)(kk * 8), bk, idesc_s, 1u);
                 }
                 mma_commit(&bars->s_full[w]);
             };
@@ -606,7 +607,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 lo[2 * c4 + 1] = pack_bf16(l4[2], l4[3]);
             }
             tmem_st32u(lane_base + QHI_COL + wg * 32, hi);
-            tmem_st32u(lane_base + QLO_COL + wg * 32, lo);
+            if (!a.tc_q_plain) tmem_st32u(lane_base + QLO_COL + wg * 32, lo);
             tc_fence_before();
         };
         pdl_wait();  // the rotated queries come from the previous kernel

@@ -212,6 +212,8 @@ struct AttnArgs {
     int tc_min_tiles;             // tensor-core kernel: fewest 64-token tiles per CTA
     int tc_seg_cost;              // tensor-core kernel: cost of a segment boundary, in tiles,
                                   // that the cuts between shares balance
+    int tc_q_plain;               // tensor-core kernel: 1 = queries as plain bf16 (one score
+                                  // MMA per step), 0 = bf16 hi + lo (two)
     int tc_merge_kernel;          // tensor-core kernel: 1 = merge in a second kernel (small
                                   // batches), 0 = inside the attention kernel
     float *part_o;                // CUDA cores: [B][Hkv][n_splits][subs][R][dh]; tensor

@@ -297,11 +297,11 @@ def test_device_status_reports_bad_inputs():
     run.close()
 
 
-@pytest.mark.parametrize("prec", [0, 1, 2, 3])
+@pytest.mark.parametrize("prec", [0, 1, 2, 3, 4])
 def test_mlp_activation_precision_options(prec):
     # automatic (bf16 MLP inputs here: mean over 8 rows), hi + lo, plain bf16
-    # for the MLP, plain bf16 for every projection: all inside the tolerance on
-    # a multi-tile shape
+    # for the MLP, plain bf16 for every projection, for all but Q/K/V: all
+    # inside the tolerance on a multi-tile shape
     shape = wl.Shape(512, 8, 2, 128, 1024, 8, 4)
     w = wl.custom(shape, [5, 40, 129, 257, 700, 1024, 64, 3], wl.LAYOUT_PAGED, 81,
                   rows_per_seq=True)
