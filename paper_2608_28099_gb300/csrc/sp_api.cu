@@ -853,7 +853,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     const bool glu = h->gu_blk == 64 && h->gemm.glu_fusable(h->w_gu, h->n, h->opt_gemm, M, mlp_lo);
     mark(SP_STAGE_GATE_UP, 0);
     s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, M, h->status, st, &launches, &ns, mlp_lo, 0,
-                    glu ? &a_out : nullptr);
+                    glu ? &a_out : nullptr, true);
     mark(SP_STAGE_GATE_UP, 1);
     if (s != SP_OK) return fail(s, "gate/up projection launch failed");
     if (!glu) {

@@ -18,6 +18,7 @@ struct TcPlan {
     int units_per_cta;  // persistent: (tile, k-block) units per CTA
     int grid;           // CTAs
     int splits;         // partial planes of Y
+    int nt;             // tile kernel: weight tiles per CTA (1, or 2 sharing each activation block)
 };
 
 bool encode_kmajor_bf16(CUtensorMap *map, const void *base, int rows, int K, int box_rows);
@@ -31,9 +32,10 @@ bool tc_supported(int N, int K);
 // MMA's N side is then 256) for M >= 256.
 int tc_bn_for(int M, bool lo = true);
 // sched: 0 = automatic, 1 = tile kernel, 2 = persistent stream-K (when its
-// partial planes fit).
+// partial planes fit).  keep_unsplit: a projection that fits one wave unsplit
+// stays unsplit (the gate/up projection's SwiGLU epilogue needs that).
 TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo = true,
-               int sched = 0);
+               int sched = 0, bool keep_unsplit = false);
 // w_blocked: the weights are stored blocked (block_weights_layout) and map_w
 // views them as [N K / 64][64] rows.
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
@@ -136,17 +138,18 @@ struct GemmPlanner {
     // run with the SwiGLU epilogue (one CTA per tile, no K split)?
     bool glu_fusable(const WeightMat &w, const ActBuf &x, int path, int M, bool lo) const {
         if (!use_tc(w, x, path)) return false;
-        const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched);
+        const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched, true);
         return !p.persistent && p.splits == 1 && p.bn >= 32;
     }
     // Enqueue the projection; *nsplit receives the number of partials in y.
-    // glu: write silu(gate) * up there instead of partials (glu_fusable).
+    // glu: write silu(gate) * up there instead of partials (glu_fusable);
+    // gate_up: plan as glu_fusable does (whether or not glu is given).
     sp_status run(int w_bf16, int path, const ActBuf &x, const WeightMat &w, float *y, int M,
                   int *status, cudaStream_t st, int *launches, int *nsplit, bool lo = true,
-                  int inject_stall = 0, const ActOut *glu = nullptr) const {
+                  int inject_stall = 0, const ActOut *glu = nullptr, bool gate_up = false) const {
         cudaError_t e;
         if (use_tc(w, x, path)) {
-            const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched);
+            const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched, gate_up || glu);
             const int bi = bn_index(p.bn);
             e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked, lo,
                                inject_stall, glu);

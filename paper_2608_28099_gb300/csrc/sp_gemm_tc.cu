@@ -48,15 +48,18 @@ constexpr int A_BYTES = 128 * BK * 2;
 
 // ---------------------------------------------------------------- tile kernel
 // LO: the activations come as hi and lo planes (the MMA's N side is [hi; lo],
-// 2 BN rows), else as plain bf16 (N = BN).
-template <int BN, bool LO>
+// 2 BN rows), else as plain bf16 (N = BN).  NT: weight tiles per CTA sharing
+// each activation k-block (2: twice the weight bytes in flight per stage for
+// the same activation bytes; plain bf16 only), each with its own accumulator.
+template <int BN, bool LO, int NT = 1>
 struct TileCfg {
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int NB = (LO ? 2 : 1) * BN;                 // MMA N
-    static constexpr int STAGE = A_BYTES + (LO ? 2 : 1) * B_BYTES;
+    static constexpr int STAGE = NT * A_BYTES + (LO ? 2 : 1) * B_BYTES;
     static constexpr int STAGES = 196608 / STAGE < 10 ? 196608 / STAGE : 10;  // 192 KB ring
-    static constexpr int TMEM_COLS = NB < 32 ? 32 : NB;          // hi and lo halves
+    static constexpr int TMEM_COLS = NT * NB < 32 ? 32 : NT * NB;  // hi and lo halves per tile
     static constexpr int SMEM = STAGES * STAGE + 1024 /*align*/ + 256 /*barriers*/;
+    static_assert(TMEM_COLS <= 512, "TMEM");
 };
 
 struct TcArgs {
@@ -79,12 +82,12 @@ struct TcArgs {
 
 constexpr int TILE_THREADS = 256;  // warps 0-2 also TMA, MMA and TMEM owner
 
-template <int BN, bool LO>
+template <int BN, bool LO, int NT>
 __global__ void __launch_bounds__(TILE_THREADS, 1)
     gemm_tile_kernel(const __grid_constant__ CUtensorMap map_w,
                    const __grid_constant__ CUtensorMap map_xhi,
                    const __grid_constant__ CUtensorMap map_xlo, TcArgs g) {
-    using Cfg = TileCfg<BN, LO>;
+    using Cfg = TileCfg<BN, LO, NT>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = (uint8_t *)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t *full = (uint64_t *)(smem + Cfg::STAGES * Cfg::STAGE);
@@ -94,7 +97,7 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
     volatile int *abort = (volatile int *)(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * BN, n0 = blockIdx.y * 128;
+    const int m0 = blockIdx.x * BN, t0 = blockIdx.y * NT, n0 = t0 * 128;  // first weight tile
     const int kb0 = blockIdx.z * g.kb_per_split;
     const int nkb = min(g.kb_per_split, g.n_kb - kb0);
     pdl_trigger();
@@ -129,12 +132,16 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
         const uint64_t pol_x = policy_evict_last();
         const int pre = nkb < Cfg::STAGES ? nkb : Cfg::STAGES;
         const bool skip0 = g.inject_stall && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0;
+        auto load_w = [&](int i, uint8_t *st, uint64_t *bar) {
+#pragma unroll
+            for (int j = 0; j < NT; ++j)
+                tma_load_2d_hint(st + j * A_BYTES, &map_w, bar, g.w_blocked ? 0 : (kb0 + i) * BK,
+                                 g.w_blocked ? ((t0 + j) * g.n_kb + kb0 + i) * 128 : n0 + j * 128, pol_w);
+        };
         for (int i = 0; i < pre; ++i) {
             if (skip0 && i == 0) continue;
             mbar_arrive_expect_tx(&full[i], Cfg::STAGE);
-            tma_load_2d_hint(smem + i * Cfg::STAGE, &map_w, &full[i],
-                             g.w_blocked ? 0 : (kb0 + i) * BK,
-                             g.w_blocked ? (blockIdx.y * g.n_kb + kb0 + i) * 128 : n0, pol_w);
+            load_w(i, smem + i * Cfg::STAGE, &full[i]);
         }
         issued = pre;
         pdl_wait();
@@ -147,12 +154,11 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
             if (i >= pre) {
                 if (!mbar_wait(&empty[s], ph ^ 1, abort, g.wait_ns)) break;
                 mbar_arrive_expect_tx(&full[s], Cfg::STAGE);
-                tma_load_2d_hint(st, &map_w, &full[s], g.w_blocked ? 0 : kc,
-                                 g.w_blocked ? (blockIdx.y * g.n_kb + kb0 + i) * 128 : n0, pol_w);
+                load_w(i, st, &full[s]);
                 issued = i + 1;
             }
-            tma_load_2d_hint(st + A_BYTES, &map_xhi, &full[s], kc, m0, pol_x);
-            if (LO) tma_load_2d_hint(st + A_BYTES + Cfg::B_BYTES, &map_xlo, &full[s], kc, m0, pol_x);
+            tma_load_2d_hint(st + NT * A_BYTES, &map_xhi, &full[s], kc, m0, pol_x);
+            if (LO) tma_load_2d_hint(st + NT * A_BYTES + Cfg::B_BYTES, &map_xlo, &full[s], kc, m0, pol_x);
         }
     } else if (warp == 1 && lane == 0) {
         // MMA issuer
@@ -163,12 +169,16 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
             if (!mbar_wait(&full[s], ph, abort, g.wait_ns)) break;
             tc_fence_after();
             uint8_t *st = smem + s * Cfg::STAGE;
-            const uint64_t a = sw128_kmajor_desc(st);
-            const uint64_t bh = sw128_kmajor_desc(st + A_BYTES);  // [hi; lo], 2 BN rows
+            const uint64_t bh = sw128_kmajor_desc(st + NT * A_BYTES);  // [hi; lo], 2 BN rows
 #pragma unroll
             for (int kk = 0; kk < BK / 16; ++kk) {
-                // +32 bytes along K per 16-element MMA step (encoded >> 4)
-                mma_bf16(tmem, a + 2 * kk, bh + 2 * kk, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+#pragma unroll
+                for (int j = 0; j < NT; ++j) {
+                    // +32 bytes along K per 16-element MMA step (encoded >> 4)
+                    const uint64_t a = sw128_kmajor_desc(st + j * A_BYTES);
+                    mma_bf16(tmem + (uint32_t)(j * Cfg::NB), a + 2 * kk, bh + 2 * kk, idesc,
+                             (i > 0 || kk > 0) ? 1u : 0u);
+                }
             }
             mma_commit(&empty[s]);
         }
@@ -183,7 +193,9 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
     // epilogue over all eight warps: warp w reads TMEM lanes 32 (w & 3).. and
     // the column chunks of half w >> 2
     const int quad = warp & 3, half = warp >> 2;
-    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16);
+#pragma unroll 1
+    for (int tj = 0; tj < NT; ++tj) {
+    const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(tj * Cfg::NB);
     if (g.glu_f) {
         if constexpr (BN >= 32) {
             // SwiGLU epilogue, per 64-column chunk: every warp puts 32 columns of
@@ -193,10 +205,10 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
             // 64 + 4 fq..: 16-byte shared loads, four features per store
             float *xb = (float *)smem;
             const int row = quad * 32 + lane, fq = threadIdx.x & 15, cg = threadIdx.x >> 4;
-            const size_t feat = (size_t)blockIdx.y * 64 + 4 * fq;
+            const size_t feat = (size_t)(t0 + tj) * 64 + 4 * fq;
 #pragma unroll 1
             for (int c0 = 0; c0 < BN; c0 += 64) {
-                float *buf = xb + ((c0 >> 6) & 1) * (64 * 132);
+                float *buf = xb + ((tj * ((BN + 63) / 64) + (c0 >> 6)) & 1) * (64 * 132);  // chunks alternate
                 if (have && c0 + half * 32 < BN) {
                     float v[32], u[32] = {};
                     tmem_ld32(trow + c0 + half * 32, v);
@@ -222,7 +234,7 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
             }
         }
     } else if (have) {
-        const int n = n0 + quad * 32 + lane;
+        const int n = n0 + tj * 128 + quad * 32 + lane;
         float *y = g.y + (size_t)blockIdx.z * g.split_stride;
         if constexpr (BN == 16) {
             if (half == 0) {
@@ -249,6 +261,7 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
             }
         }
     }
+    }  // weight tiles of the CTA
     if (warp == 0 && lane == 0) {
         // no TMA write may still be in flight when the CTA's shared memory goes away
         for (int i = issued > Cfg::STAGES ? issued - Cfg::STAGES : 0; i < issued; ++i)
@@ -260,18 +273,19 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
     if (warp == 2) tmem_dealloc(tmem, Cfg::TMEM_COLS);
 }
 
-template <int BN, bool LO>
+template <int BN, bool LO, int NT = 1>
 cudaError_t launch_tile(const CUtensorMap &mw, const CUtensorMap &mh, const CUtensorMap &ml,
                       const TcArgs &g, dim3 grid, cudaStream_t st) {
-    const int smem = TileCfg<BN, LO>::SMEM;
+    const int smem = TileCfg<BN, LO, NT>::SMEM;
     static bool attr_set = false;  // per device process-wide (one device per process here)
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_tile_kernel<BN, LO>,
+        cudaError_t e = cudaFuncSetAttribute(gemm_tile_kernel<BN, LO, NT>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    return launch_k(gemm_tile_kernel<BN, LO>, grid, dim3(TILE_THREADS), (size_t)smem, st, mw, mh, ml, g);
+    return launch_k(gemm_tile_kernel<BN, LO, NT>, grid, dim3(TILE_THREADS), (size_t)smem, st, mw, mh, ml,
+                    g);
 }
 
 
@@ -618,8 +632,10 @@ static int planes_for(long long tiles, int n_kb, long long L) {
     return most;
 }
 
-TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo, int sched) {
+TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo, int sched,
+               bool keep_unsplit) {
     TcPlan p;
+    p.nt = 1;
     p.bn = tc_bn_for(M, lo);
     p.m_tiles = ceil_div(M, p.bn);
     p.n_tiles = N / 128;
@@ -644,6 +660,33 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo, 
     // (estimates in units of one CTA's k-block time, 16 KB of weights).
     const int waves = ceil_div(tiles * p.splits, n_sm);
     const double fill = (double)tiles * p.splits / ((double)waves * n_sm);
+    // Two weight tiles per CTA (plain bf16, up to 128 rows: HBM-bound): each stage
+    // carries twice the weight bytes for the same activation bytes.  Taken when
+    // the paired grid still fills ~all SMs in one wave with no more K splits
+    // (extra splits cost the consumer more partial planes than the pairing saves:
+    // 27b_long gate/up 65.5 -> 63.4 us, its down projection unchanged at 7
+    // splits instead of 3 while the readout slowed by 2 us).
+    if (sched == 0 && !lo && p.bn <= 128 && p.n_tiles % 2 == 0) {
+        const int pairs = p.m_tiles * (p.n_tiles / 2);
+        int S2 = 1;
+        if (pairs < n_sm) {
+            S2 = n_sm / pairs;
+            const int max_s = p.n_kb / 2 > 0 ? p.n_kb / 2 : 1;
+            if (S2 > max_s) S2 = max_s;
+        }
+        while (S2 > 1 && (size_t)S2 * M * N * sizeof(float) > y_capacity_bytes) --S2;
+        const int kbs2 = ceil_div(p.n_kb, S2);
+        S2 = ceil_div(p.n_kb, kbs2);
+        (void)keep_unsplit;  // S2 <= splits keeps an unsplit projection unsplit
+        if (S2 <= p.splits && pairs * S2 <= n_sm && pairs * S2 * 100 >= n_sm * 85) {
+            p.nt = 2;
+            p.kb_per_split = kbs2;
+            p.splits = S2;
+            p.grid = pairs * S2;
+            p.units_per_cta = kbs2;
+            return p;
+        }
+    }
     if (sched == 1) return p;
     if (sched == 2 || (waves > 1 && fill < 0.8)) {
         const long long U = (long long)tiles * p.n_kb;
@@ -713,7 +756,17 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
         g.glu_f = N / 2;
         g.glu = *glu;
     }
-    dim3 grid(p.m_tiles, p.n_tiles, p.splits);
+    dim3 grid(p.m_tiles, p.n_tiles / p.nt, p.splits);
+    if (p.nt == 2) {
+        if (lo || p.n_tiles % 2) return cudaErrorInvalidValue;
+        switch (p.bn) {
+        case 16: return launch_tile<16, false, 2>(map_w, map_xhi, map_xlo, g, grid, st);
+        case 32: return launch_tile<32, false, 2>(map_w, map_xhi, map_xlo, g, grid, st);
+        case 64: return launch_tile<64, false, 2>(map_w, map_xhi, map_xlo, g, grid, st);
+        case 128: return launch_tile<128, false, 2>(map_w, map_xhi, map_xlo, g, grid, st);
+        default: return cudaErrorInvalidValue;
+        }
+    }
     switch (p.bn) {
     case 16: return lo ? launch_tile<16, true>(map_w, map_xhi, map_xlo, g, grid, st)
                     : launch_tile<16, false>(map_w, map_xhi, map_xlo, g, grid, st);
