@@ -30,7 +30,7 @@ __device__ __forceinline__ float block_sum(float v, float *red) {
 // One block per row, d % 8 == 0: 8-element vector loads, four chunks in
 // flight per thread.
 template <typename T>
-__global__ void __launch_bounds__(256) rmsnorm_rows_kernel(const T *__restrict__ x, int row_mod,
+__global__ void __launch_bounds__(256) rmsnorm_rows_loop_kernel(const T *__restrict__ x, int row_mod,
                                                            const float *__restrict__ gain, float eps,
                                                            int d, ActOut out) {
     pdl_trigger();
@@ -117,7 +117,7 @@ __global__ void __launch_bounds__(256) qkv_rope_kernel(QkvRopeArgs a) {
 // h1 = x + y, n = RMSNorm(h1): one block per row, 4-element vectors.  Row m
 // reads x row (row_mod ? m % row_mod : m) and y row m / y_div.
 template <typename TX>
-__global__ void __launch_bounds__(1024) residual_norm_kernel(PartIn y, int y_div,
+__global__ void __launch_bounds__(1024) residual_norm_loop_kernel(PartIn y, int y_div,
                                                              const TX *__restrict__ x,
                                                              int row_mod,
                                                              const float *__restrict__ gain,
@@ -148,6 +148,127 @@ __global__ void __launch_bounds__(1024) residual_norm_kernel(PartIn y, int y_div
         const float4 gv = *(const float4 *)(gain + c * 4);
         act_store4(n, (size_t)m * d + c * 4,
                    make_float4(v.x * inv * gv.x, v.y * inv * gv.y, v.z * inv * gv.z, v.w * inv * gv.w));
+    }
+}
+
+// Register-resident norms for d <= 8192: one block of kNormThreads per row; each
+// thread keeps its chunks in registers between the sum of squares and the
+// output (no second pass over the row), with every load of the row issued
+// before the first add.
+constexpr int kNormThreads = 256;
+constexpr int kNormMaxD = 8192;
+
+int sm_count_cached() {
+    static int n = 0;
+    if (!n) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    }
+    return n;
+}
+
+__device__ __forceinline__ float4 load4(const float *p) { return *(const float4 *)p; }
+__device__ __forceinline__ float4 load4(const bf16 *p) {
+    const uint2 u = *(const uint2 *)p;
+    return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xffff0000u),
+                       __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xffff0000u));
+}
+
+template <int TPB>
+__device__ __forceinline__ float norm_block_sum(float v, float *red) {
+    v = warp_sum(v);
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    if (l == 0) red[w] = v;
+    __syncthreads();
+    float t = l < TPB / 32 ? red[l] : 0.f;
+    return warp_sum(t);
+}
+
+template <typename T, int V, int TPB>  // V: 4-element chunks per thread, d <= 4 V TPB
+__global__ void __launch_bounds__(TPB) rmsnorm_rows_kernel(const T *__restrict__ x, int row_mod,
+                                                                    const float *__restrict__ gain,
+                                                                    float eps, int d, ActOut out) {
+    pdl_trigger();
+    __shared__ float red[TPB / 32];
+    const int m = blockIdx.x, nch = d >> 2;
+    float4 gv[V];
+#pragma unroll
+    for (int i = 0; i < V; ++i) {  // constant: before the dependency wait
+        const int c = threadIdx.x + i * TPB;
+        gv[i] = c < nch ? *(const float4 *)(gain + c * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    pdl_wait();
+    const T *xr = x + (size_t)(row_mod ? m % row_mod : m) * d;
+    float4 v[V];
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+        const int c = threadIdx.x + i * TPB;
+        v[i] = c < nch ? load4(xr + c * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int i = 0; i < V; ++i) ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+    ss = norm_block_sum<TPB>(ss, red);
+    const float inv = rsqrtf(ss / (float)d + eps);
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+        const int c = threadIdx.x + i * TPB;
+        if (c < nch)
+            act_store4(out, (size_t)m * d + c * 4,
+                       make_float4(v[i].x * inv * gv[i].x, v[i].y * inv * gv[i].y, v[i].z * inv * gv[i].z,
+                                   v[i].w * inv * gv[i].w));
+    }
+}
+
+// h1 = x + y, n = RMSNorm(h1): as above, h1 kept in registers.
+template <typename TX, int V, int TPB>
+__global__ void __launch_bounds__(TPB) residual_norm_kernel(PartIn y, int y_div,
+                                                                     const TX *__restrict__ x, int row_mod,
+                                                                     const float *__restrict__ gain,
+                                                                     float eps, int d,
+                                                                     float *__restrict__ h1, ActOut n) {
+    pdl_trigger();
+    __shared__ float red[TPB / 32];
+    const int m = blockIdx.x, nch = d >> 2;
+    float4 gv[V];
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+        const int c = threadIdx.x + i * TPB;
+        gv[i] = c < nch ? *(const float4 *)(gain + c * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    pdl_wait();
+    const TX *xr = x + (size_t)(row_mod ? m % row_mod : m) * d;
+    const size_t yrow = (size_t)(m / y_div) * d;
+    float4 v[V];
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+        const int c = threadIdx.x + i * TPB;
+        if (c < nch) {
+            const float4 yv = part_get4(y, yrow + c * 4);
+            const float4 xv = load4(xr + c * 4);
+            v[i] = make_float4(xv.x + yv.x, xv.y + yv.y, xv.z + yv.z, xv.w + yv.w);
+        } else {
+            v[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+    }
+    float ss = 0.f;
+    float *hr = h1 + (size_t)m * d;
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+        const int c = threadIdx.x + i * TPB;
+        if (c < nch) *(float4 *)(hr + c * 4) = v[i];
+        ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+    }
+    ss = norm_block_sum<TPB>(ss, red);
+    const float inv = rsqrtf(ss / (float)d + eps);
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+        const int c = threadIdx.x + i * TPB;
+        if (c < nch)
+            act_store4(n, (size_t)m * d + c * 4,
+                       make_float4(v[i].x * inv * gv[i].x, v[i].y * inv * gv[i].y, v[i].z * inv * gv[i].z,
+                                   v[i].w * inv * gv[i].w));
     }
 }
 
@@ -391,12 +512,32 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const float *__restrict_
 
 cudaError_t launch_rmsnorm_rows(int x_bf16, const void *x, int row_mod, const float *gain,
                                 float eps, int M, int d, ActOut out, cudaStream_t st) {
-    if (x_bf16)
-        return launch_k(rmsnorm_rows_kernel<bf16>, dim3(M), dim3(kRowThreads), 0, st, (const bf16 *)x,
-                        row_mod, gain, eps, d, out);
-    else
-        return launch_k(rmsnorm_rows_kernel<float>, dim3(M), dim3(kRowThreads), 0, st, (const float *)x,
-                        row_mod, gain, eps, d, out);
+    if (d > kNormMaxD) {
+        if (x_bf16)
+            return launch_k(rmsnorm_rows_loop_kernel<bf16>, dim3(M), dim3(kRowThreads), 0, st,
+                            (const bf16 *)x, row_mod, gain, eps, d, out);
+        return launch_k(rmsnorm_rows_loop_kernel<float>, dim3(M), dim3(kRowThreads), 0, st,
+                        (const float *)x, row_mod, gain, eps, d, out);
+    }
+    // few rows: 1024 threads per row, else 256 (more rows in flight per SM)
+    const bool wide = M < 2 * sm_count_cached();
+    const int V = ceil_div(d / 4, wide ? 1024 : kNormThreads);
+#define SP_NORM_CASE(VV, TT)                                                                   \
+    case VV:                                                                                   \
+        return x_bf16 ? launch_k(rmsnorm_rows_kernel<bf16, VV, TT>, dim3(M), dim3(TT), 0, st,  \
+                                 (const bf16 *)x, row_mod, gain, eps, d, out)                  \
+                      : launch_k(rmsnorm_rows_kernel<float, VV, TT>, dim3(M), dim3(TT), 0, st, \
+                                 (const float *)x, row_mod, gain, eps, d, out);
+    if (wide) {
+        switch (V) { SP_NORM_CASE(1, 1024) SP_NORM_CASE(2, 1024) }
+    } else {
+        switch (V) {
+            SP_NORM_CASE(1, 256) SP_NORM_CASE(2, 256) SP_NORM_CASE(3, 256) SP_NORM_CASE(4, 256)
+            SP_NORM_CASE(5, 256) SP_NORM_CASE(6, 256) SP_NORM_CASE(7, 256) SP_NORM_CASE(8, 256)
+        }
+    }
+#undef SP_NORM_CASE
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st) {
@@ -406,12 +547,31 @@ cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st) {
 cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mod,
                                  const float *gain, float eps, int M, int d, float *h1, ActOut n,
                                  cudaStream_t st, int y_div) {
-    if (x_bf16)
-        return launch_k(residual_norm_kernel<bf16>, dim3(M), dim3(kWideThreads), 0, st, y, y_div,
-                        (const bf16 *)x, row_mod, gain, eps, d, h1, n);
-    else
-        return launch_k(residual_norm_kernel<float>, dim3(M), dim3(kWideThreads), 0, st, y, y_div,
+    if (d > kNormMaxD) {
+        if (x_bf16)
+            return launch_k(residual_norm_loop_kernel<bf16>, dim3(M), dim3(kWideThreads), 0, st, y, y_div,
+                            (const bf16 *)x, row_mod, gain, eps, d, h1, n);
+        return launch_k(residual_norm_loop_kernel<float>, dim3(M), dim3(kWideThreads), 0, st, y, y_div,
                         (const float *)x, row_mod, gain, eps, d, h1, n);
+    }
+    const bool wide = M < 2 * sm_count_cached();
+    const int V = ceil_div(d / 4, wide ? 1024 : kNormThreads);
+#define SP_NORM_CASE(VV, TT)                                                                     \
+    case VV:                                                                                     \
+        return x_bf16 ? launch_k(residual_norm_kernel<bf16, VV, TT>, dim3(M), dim3(TT), 0, st, y,  \
+                                 y_div, (const bf16 *)x, row_mod, gain, eps, d, h1, n)           \
+                      : launch_k(residual_norm_kernel<float, VV, TT>, dim3(M), dim3(TT), 0, st, y, \
+                                 y_div, (const float *)x, row_mod, gain, eps, d, h1, n);
+    if (wide) {
+        switch (V) { SP_NORM_CASE(1, 1024) SP_NORM_CASE(2, 1024) }
+    } else {
+        switch (V) {
+            SP_NORM_CASE(1, 256) SP_NORM_CASE(2, 256) SP_NORM_CASE(3, 256) SP_NORM_CASE(4, 256)
+            SP_NORM_CASE(5, 256) SP_NORM_CASE(6, 256) SP_NORM_CASE(7, 256) SP_NORM_CASE(8, 256)
+        }
+    }
+#undef SP_NORM_CASE
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_swiglu(PartIn y, int M, int f, int blk, ActOut a, cudaStream_t st) {
