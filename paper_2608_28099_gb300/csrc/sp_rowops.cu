@@ -66,8 +66,74 @@ __global__ void __launch_bounds__(256) rmsnorm_rows_loop_kernel(const T *__restr
 // once (from the caller's ids and lengths, before the dependency wait), then
 // each thread rotates four pairs (i, i + dh/2) of a query or key head at a time
 // (16-byte loads of the partial sums and of the (cos, sin) table) or copies
-// four values.
-__global__ void __launch_bounds__(256) qkv_rope_kernel(QkvRopeArgs a) {
+// four values.  With few rows the block has 1024 threads, so that a row's items
+// take one pass.
+template <int TPB>
+__global__ void __launch_bounds__(TPB) qkv_rope_kernel(QkvRopeArgs a) {
+    pdl_trigger();
+    __shared__ int s_pos;
+    const int m = blockIdx.x;
+    const int b = m / a.k, r = m % a.k;
+    if (threadIdx.x == 0) {
+        const SeqRef s = resolve_seq(a.seq_ids, a.seq_lens, a.lens_by_batch, b, a.n_seqs,
+                                     a.max_seq_len, a.status);
+        s_pos = s.len + a.r0 + (a.k_task ? r % a.k_task : r);
+    }
+    pdl_wait();
+    if (a.zero_ints && m == 0)
+        for (int t = threadIdx.x; t < a.n_zero; t += blockDim.x) a.zero_ints[t] = 0;
+    __syncthreads();
+    const int dh = a.dh, half = dh >> 1, q4 = half >> 2;
+    const int nqkv = (a.Hq + 2 * a.Hkv) * dh;
+    const size_t row = (size_t)(a.shared ? r : m) * nqkv;
+    const int kns = a.kn_stride ? a.kn_stride : a.k;
+    const size_t mn = (size_t)b * kns + a.r0 + r;  // row of k_new / v_new
+    const float2 *cs = a.rope_cs + (size_t)s_pos * half;
+    const int nrot = (a.Hq + a.Hkv) * q4, nval = a.Hkv * dh / 4, total = nrot + nval;
+    constexpr int U = 1;  // items per pass (two per pass measured slower with many rows)
+    for (int base = threadIdx.x; base < total; base += U * TPB) {
+        float4 x0[U], x1[U], c01[U], c23[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int it = base + u * TPB;
+            if (it < nrot) {
+                const int h = it / q4, i = (it - h * q4) * 4;
+                x0[u] = part_get4(a.y, row + (size_t)h * dh + i);
+                x1[u] = part_get4(a.y, row + (size_t)h * dh + i + half);
+                c01[u] = *(const float4 *)(cs + i);
+                c23[u] = *(const float4 *)(cs + i + 2);
+            } else if (it < total) {
+                x0[u] = part_get4(a.y, row + (size_t)(a.Hq + a.Hkv) * dh + (it - nrot) * 4);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int it = base + u * TPB;
+            if (it < nrot) {
+                const int h = it / q4, i = (it - h * q4) * 4;
+                const float c[4] = {c01[u].x, c01[u].z, c23[u].x, c23[u].z};
+                const float sn[4] = {c01[u].y, c01[u].w, c23[u].y, c23[u].w};
+                const float a0[4] = {x0[u].x, x0[u].y, x0[u].z, x0[u].w};
+                const float a1[4] = {x1[u].x, x1[u].y, x1[u].z, x1[u].w};
+                float o0[4], o1[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    o0[e] = a0[e] * c[e] - a1[e] * sn[e];
+                    o1[e] = a1[e] * c[e] + a0[e] * sn[e];
+                }
+                float *dst = h < a.Hq ? a.q + ((size_t)m * a.Hq + h) * dh
+                                      : a.k_new + (mn * a.Hkv + (h - a.Hq)) * dh;
+                *(float4 *)(dst + i) = make_float4(o0[0], o0[1], o0[2], o0[3]);
+                *(float4 *)(dst + i + half) = make_float4(o1[0], o1[1], o1[2], o1[3]);
+            } else if (it < total) {
+                *(float4 *)(a.v_new + mn * a.Hkv * dh + (it - nrot) * 4) = x0[u];
+            }
+        }
+    }
+}
+
+// The same with 256 threads and one item per loop step (many rows).
+__global__ void __launch_bounds__(256) qkv_rope_rows_kernel(QkvRopeArgs a) {
     pdl_trigger();
     __shared__ int s_pos;
     const int m = blockIdx.x;
@@ -541,7 +607,10 @@ cudaError_t launch_rmsnorm_rows(int x_bf16, const void *x, int row_mod, const fl
 }
 
 cudaError_t launch_qkv_rope(const QkvRopeArgs &a, cudaStream_t st) {
-    return launch_k(qkv_rope_kernel, dim3(a.B * a.k), dim3(256), 0, st, a);
+    // few rows: 1024 threads per row (one pass of items), else 256
+    if (a.B * a.k < 2 * sm_count_cached())
+        return launch_k(qkv_rope_kernel<1024>, dim3(a.B * a.k), dim3(1024), 0, st, a);
+    return launch_k(qkv_rope_rows_kernel, dim3(a.B * a.k), dim3(256), 0, st, a);
 }
 
 cudaError_t launch_residual_norm(int x_bf16, PartIn y, const void *x, int row_mod,
