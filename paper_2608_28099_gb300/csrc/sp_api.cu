@@ -742,8 +742,22 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     const bool qkv_lo = h->opt_prec != 3;
     const bool q_plain = h->opt_qprec == 2 || (h->opt_qprec == 0 && mean && h->k_task >= 16);
 
-    // a1-a2: pre-norm, Q/K/V projection, rotation at positions L_b + r
+    // a1-a2: pre-norm, Q/K/V projection, rotation at positions L_b + r (in the
+    // projection's epilogue when it runs one CTA per head, else a kernel of its own)
     PartIn yqkv = {h->qkv_shared, 1, 0};
+    const bool rope_fused = (d_rows || d_hidden) && dh == 128 &&
+                            h->gemm.rope_fusable(h->w_qkv, h->xn, h->opt_gemm, M, qkv_lo);
+    RopeEpi re;
+    memset(&re, 0, sizeof re);
+    re.rope_cs = h->rope_cs;
+    re.Hq = hq; re.Hkv = hkv; re.k = k; re.kn_stride = 0; re.r0 = 0; re.k_task = h->k_task;
+    re.seq_ids = d_seq_ids; re.seq_lens = d_seq_lens; re.lens_by_batch = lens_by_batch;
+    re.n_seqs = kv->n_seqs; re.max_seq_len = c.max_seq_len;
+    re.q = h->q; re.k_new = h->k_new; re.v_new = h->v_new;
+    re.status = h->status;
+    re.zero_ints = attention_counters(h->attn_ws);
+    re.n_zero = batch * hkv;
+    const RopeEpi *rp = rope_fused ? &re : nullptr;
     if (d_hidden) {
         // input fusion: u_b = W_fc_h RMSNorm(h_b; g_h); x_{b,r} = u_b + fc_prompt[r],
         // stored for the residual, and x_hat = RMSNorm(x; g_in) for Q/K/V
@@ -761,7 +775,8 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         mark(SP_STAGE_INPUT_NORM, 1);
         ++launches;
         mark(SP_STAGE_QKV, 0);
-        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, qkv_lo);
+        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, qkv_lo, 0,
+                        nullptr, false, rp);
         mark(SP_STAGE_QKV, 1);
         if (s != SP_OK) return fail(s, "Q/K/V projection launch failed");
         yqkv = PartIn{h->y, ns, stride_qkv};
@@ -771,7 +786,8 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         mark(SP_STAGE_INPUT_NORM, 1);
         ++launches;
         mark(SP_STAGE_QKV, 0);
-        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, qkv_lo);
+        s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, qkv_lo, 0,
+                        nullptr, false, rp);
         mark(SP_STAGE_QKV, 1);
         if (s != SP_OK) return fail(s, "Q/K/V projection launch failed");
         yqkv = PartIn{h->y, ns, stride_qkv};
@@ -792,10 +808,12 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     plan_attention(batch, hkv, k, c.max_seq_len, h->opt_split, h->n_sm, &split_tokens, &n_splits);
     r.zero_ints = attention_counters(h->attn_ws);
     r.n_zero = batch * hkv;
-    mark(SP_STAGE_ROPE, 0);
-    SP_CUDA(launch_qkv_rope(r, st));
-    mark(SP_STAGE_ROPE, 1);
-    ++launches;
+    if (!rope_fused) {
+        mark(SP_STAGE_ROPE, 0);
+        SP_CUDA(launch_qkv_rope(r, st));
+        mark(SP_STAGE_ROPE, 1);
+        ++launches;
+    }
 
     // a3: attention over [cache ; new keys]
     AttnArgs a;

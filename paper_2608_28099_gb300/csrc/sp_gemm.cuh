@@ -11,6 +11,22 @@
 
 namespace sp {
 
+// Rotation epilogue of the Q/K/V projection (rows [(Hq + 2 Hkv) 128][K], one
+// 128-row weight tile per head): the CTA of tile t writes head t of its rows
+// rotated at L_b + r0 + (k_task ? r % k_task : r) into q (query heads) or k_new,
+// or copied into v_new, instead of a partial plane (Sec. 3.3; the same
+// arithmetic as the separate rotation kernel).
+struct RopeEpi {
+    const float2 *rope_cs;   // [max_seq_len + k][64] (cos, sin)
+    int Hq, Hkv, k, kn_stride, r0, k_task;
+    const int *seq_ids, *seq_lens;
+    int lens_by_batch, n_seqs, max_seq_len;
+    float *q, *k_new, *v_new;
+    int *status;
+    int *zero_ints;          // cleared for the next kernel (the attention's merge counters)
+    int n_zero;
+};
+
 struct TcPlan {
     int bn, m_tiles, n_tiles, n_kb;
     bool persistent;    // persistent stream-K kernel, else one CTA per (tile, K split)
@@ -41,7 +57,8 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo =
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
                            float *y, int *status, cudaStream_t st, bool w_blocked = false,
-                           bool lo = true, int inject_stall = 0, const ActOut *glu = nullptr);
+                           bool lo = true, int inject_stall = 0, const ActOut *glu = nullptr,
+                           const RopeEpi *rope = nullptr);
 
 // Weights [N][K] (es bytes per element) re-laid out as contiguous 16 KB blocks
 // [N / 128][K / 64][128][64]: one weight tile's k-block is one sequential read
@@ -141,18 +158,26 @@ struct GemmPlanner {
         const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched, true);
         return !p.persistent && p.splits == 1 && p.bn >= 32;
     }
+    // Would the Q/K/V projection run with the rotation epilogue (one CTA per
+    // weight tile = head, no K split)?
+    bool rope_fusable(const WeightMat &w, const ActBuf &x, int path, int M, bool lo) const {
+        if (!use_tc(w, x, path)) return false;
+        const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched);
+        return !p.persistent && p.splits == 1 && p.nt == 1 && p.bn >= 32;
+    }
     // Enqueue the projection; *nsplit receives the number of partials in y.
     // glu: write silu(gate) * up there instead of partials (glu_fusable);
     // gate_up: plan as glu_fusable does (whether or not glu is given).
     sp_status run(int w_bf16, int path, const ActBuf &x, const WeightMat &w, float *y, int M,
                   int *status, cudaStream_t st, int *launches, int *nsplit, bool lo = true,
-                  int inject_stall = 0, const ActOut *glu = nullptr, bool gate_up = false) const {
+                  int inject_stall = 0, const ActOut *glu = nullptr, bool gate_up = false,
+                  const RopeEpi *rope = nullptr) const {
         cudaError_t e;
         if (use_tc(w, x, path)) {
             const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched, gate_up || glu);
             const int bi = bn_index(p.bn);
             e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked, lo,
-                               inject_stall, glu);
+                               inject_stall, glu, rope);
             *nsplit = p.splits;
         } else {
             e = launch_gemm_simt(w_bf16, x.ptr, w.ptr, y, M, w.N, w.K, st, w.blocked);

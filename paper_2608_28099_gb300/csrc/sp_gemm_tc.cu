@@ -58,7 +58,8 @@ struct TileCfg {
     static constexpr int STAGE = NT * A_BYTES + (LO ? 2 : 1) * B_BYTES;
     static constexpr int STAGES = 196608 / STAGE < 10 ? 196608 / STAGE : 10;  // 192 KB ring
     static constexpr int TMEM_COLS = NT * NB < 32 ? 32 : NT * NB;  // hi and lo halves per tile
-    static constexpr int SMEM = STAGES * STAGE + 1024 /*align*/ + 256 /*barriers*/;
+    static constexpr int OFF_POS = STAGES * STAGE + 256;  // rotation epilogue: [BN] (pos, k_new row)
+    static constexpr int SMEM = STAGES * STAGE + 1024 /*align*/ + 256 /*barriers*/ + BN * 8;
     static_assert(TMEM_COLS <= 512, "TMEM");
 };
 
@@ -78,6 +79,8 @@ struct TcArgs {
     // glu[m][64t + j] = silu(gate) * up instead of a partial plane
     int glu_f;
     ActOut glu;
+    // rotation epilogue (rope.rope_cs != NULL; RopeEpi)
+    RopeEpi rope;
 };
 
 constexpr int TILE_THREADS = 256;  // warps 0-2 also TMA, MMA and TMEM owner
@@ -117,6 +120,25 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
     if (warp == 2) {
         tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
         tmem_relinquish();
+    }
+    // rotation epilogue: the rows' positions and k_new rows, resolved from the
+    // caller's ids and lengths while the main loop runs (they need no wait)
+    int2 *pos_s = (int2 *)(smem + Cfg::OFF_POS);
+    const bool rope_on = g.rope.rope_cs != nullptr;
+    if (rope_on && threadIdx.x >= 64) {
+        for (int j = threadIdx.x - 64; j < BN; j += TILE_THREADS - 64) {
+            const int m = m0 + j;
+            int2 pm = make_int2(0, 0);
+            if (m < g.M) {
+                const int b = m / g.rope.k, r = m - b * g.rope.k;
+                const SeqRef sq = resolve_seq(g.rope.seq_ids, g.rope.seq_lens, g.rope.lens_by_batch, b,
+                                              g.rope.n_seqs, g.rope.max_seq_len,
+                                              blockIdx.y == 0 ? g.rope.status : nullptr);
+                pm.x = sq.len + g.rope.r0 + (g.rope.k_task ? r % g.rope.k_task : r);
+                pm.y = b * (g.rope.kn_stride ? g.rope.kn_stride : g.rope.k) + g.rope.r0 + r;
+            }
+            pos_s[j] = pm;
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -193,10 +215,66 @@ __global__ void __launch_bounds__(TILE_THREADS, 1)
     // epilogue over all eight warps: warp w reads TMEM lanes 32 (w & 3).. and
     // the column chunks of half w >> 2
     const int quad = warp & 3, half = warp >> 2;
+    if (rope_on && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0)
+        for (int t = threadIdx.x; t < g.rope.n_zero; t += TILE_THREADS) g.rope.zero_ints[t] = 0;
 #pragma unroll 1
     for (int tj = 0; tj < NT; ++tj) {
     const uint32_t trow = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)(tj * Cfg::NB);
-    if (g.glu_f) {
+    if (rope_on) {
+        if constexpr (BN >= 32) {
+            // rotation epilogue, per 64-column chunk: the rows go through the idle
+            // ring as in the SwiGLU epilogue, then thread (fq, cg) rotates pairs
+            // (i, i + 64), i = 4 fq..4 fq + 3, of columns 4 cg..4 cg + 3 (TMEM
+            // lanes i and 64 + i), or copies them for a value head
+            float *xb = (float *)smem;
+            const int row = quad * 32 + lane, fq = threadIdx.x & 15, cg = threadIdx.x >> 4;
+            const int h = blockIdx.y, i = 4 * fq;  // head = weight tile
+            const int Hq = g.rope.Hq, Hkv = g.rope.Hkv;
+#pragma unroll 1
+            for (int c0 = 0; c0 < BN; c0 += 64) {
+                float *buf = xb + ((c0 >> 6) & 1) * (64 * 132);
+                if (have && c0 + half * 32 < BN) {
+                    float v[32], u[32] = {};
+                    tmem_ld32(trow + c0 + half * 32, v);
+                    if (LO) tmem_ld32(trow + BN + c0 + half * 32, u);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) buf[(half * 32 + j) * 132 + row] = v[j] + u[j];
+                }
+                __syncthreads();
+                if (have) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int cc = 4 * cg + e, m = m0 + c0 + cc;
+                        if (c0 + cc >= BN || m >= g.M) break;
+                        const float4 x0 = ld_shared_v4f(buf + cc * 132 + i);
+                        const float4 x1 = ld_shared_v4f(buf + cc * 132 + 64 + i);
+                        const int2 pm = pos_s[c0 + cc];
+                        float *dst;
+                        if (h < Hq + Hkv) {
+                            const float2 *cs = g.rope.rope_cs + (size_t)pm.x * 64;
+                            const float4 c01 = *(const float4 *)(cs + i), c23 = *(const float4 *)(cs + i + 2);
+                            const float c[4] = {c01.x, c01.z, c23.x, c23.z}, sn[4] = {c01.y, c01.w, c23.y, c23.w};
+                            const float a0[4] = {x0.x, x0.y, x0.z, x0.w}, a1[4] = {x1.x, x1.y, x1.z, x1.w};
+                            float o0[4], o1[4];
+#pragma unroll
+                            for (int q4 = 0; q4 < 4; ++q4) {
+                                o0[q4] = a0[q4] * c[q4] - a1[q4] * sn[q4];
+                                o1[q4] = a1[q4] * c[q4] + a0[q4] * sn[q4];
+                            }
+                            dst = h < Hq ? g.rope.q + ((size_t)m * Hq + h) * 128
+                                         : g.rope.k_new + ((size_t)pm.y * Hkv + (h - Hq)) * 128;
+                            *(float4 *)(dst + i) = make_float4(o0[0], o0[1], o0[2], o0[3]);
+                            *(float4 *)(dst + i + 64) = make_float4(o1[0], o1[1], o1[2], o1[3]);
+                        } else {
+                            dst = g.rope.v_new + ((size_t)pm.y * Hkv + (h - Hq - Hkv)) * 128;
+                            *(float4 *)(dst + i) = x0;
+                            *(float4 *)(dst + i + 64) = x1;
+                        }
+                    }
+                }
+            }
+        }
+    } else if (g.glu_f) {
         if constexpr (BN >= 32) {
             // SwiGLU epilogue, per 64-column chunk: every warp puts 32 columns of
             // its 32 rows (TMEM lanes) into the idle ring as [column][132] fp32
@@ -709,7 +787,7 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo, 
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
                            const CUtensorMap &map_xlo, const TcPlan &p, int M, int N, int K,
                            float *y, int *status, cudaStream_t st, bool w_blocked, bool lo,
-                           int inject_stall, const ActOut *glu) {
+                           int inject_stall, const ActOut *glu, const RopeEpi *rope) {
     if (p.persistent) {
         PkArgs g;
         g.M = M;
@@ -751,6 +829,11 @@ cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
     g.wait_ns = inject_stall ? 1000000ull : sm100::kWaitLimitNs;
     g.glu_f = 0;
     memset(&g.glu, 0, sizeof g.glu);
+    memset(&g.rope, 0, sizeof g.rope);
+    if (rope) {
+        if (p.persistent || p.splits != 1 || p.nt != 1 || p.bn < 32 || glu) return cudaErrorInvalidValue;
+        g.rope = *rope;
+    }
     if (glu) {
         if (p.persistent || p.splits != 1 || p.bn < 32 || N % 128) return cudaErrorInvalidValue;
         g.glu_f = N / 2;
