@@ -27,9 +27,10 @@
 // GQA group and the k soft-prompt rows together form the M side of the MMA.
 // Per 64-token tile i of a segment (w = i & 1):
 //   S_i   = Q K_i^T           M = 128 query rows, N = 64 tokens, K = 128 dims,
-//                             Q split into bf16 hi + lo held in TMEM (the
-//                             MMA's A operand, two MMAs per step), into TMEM
-//                             buffer S_w
+//                             Q held in TMEM (the MMA's A operand) as bf16 hi +
+//                             lo (two MMAs per step) or, when the head pools at
+//                             least 16 rows, plain bf16 (one), into TMEM buffer
+//                             S_w
 //   softmax                   warpgroup w (tiles alternate between two
 //                             warpgroups), one query row per thread; a row's
 //                             running max only moves when its max grows by
@@ -95,7 +96,8 @@ constexpr int THREADS = 384;                   // 2 softmax warpgroups, 2 produc
 constexpr int PRODUCER_WARP = 8, MMA_WARP = 9, MMA_WARP1 = 10, PRODUCER_WARP1 = 11;
 constexpr float RESCALE_LOG2 = 8.f;            // tolerate p <= 2^8 before rescaling O
 constexpr int kStagedSegs = 4;                 // most partials merged through the idle ring
-// TMEM columns: S0 [0,64) S1 [64,128) O0 [128,256) O1 [256,384) Qhi [384,448) Qlo [448,512);
+// TMEM columns: S0 [0,64) S1 [64,128) O0 [128,256) O1 [256,384) Qhi [384,448) Qlo [448,512)
+// (Qlo unused with plain queries);
 // P_w (64 bf16 per row) overwrites the first 32 columns of S_w once S_w is read.
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t O_COL = 128, QHI_COL = 384, QLO_COL = 448;

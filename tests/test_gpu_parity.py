@@ -310,6 +310,24 @@ def test_mlp_activation_precision_options(prec):
     run.close()
 
 
+@pytest.mark.parametrize("opts", [
+    {sp.SP_OPT_GEMM_SCHEDULE: 1}, {sp.SP_OPT_GEMM_SCHEDULE: 2},
+    {sp.SP_OPT_ATTN_MERGE: 1}, {sp.SP_OPT_ATTN_MERGE: 2},
+    {sp.SP_OPT_QUERY_PRECISION: 1}, {sp.SP_OPT_QUERY_PRECISION: 2},
+], ids=["gemm-tile", "gemm-persistent", "merge-in-kernel", "merge-kernel", "query-hi-lo",
+        "query-plain"])
+def test_work_split_and_query_precision_options(opts):
+    # every projection schedule, both places of the attention merge and both
+    # query precisions stay inside the tolerance: 16 pooled rows (plain bf16
+    # queries by default here), 8 ragged sequences over many tiles
+    shape = wl.Shape(512, 8, 2, 128, 1024, 16, 4)
+    w = wl.custom(shape, [5, 40, 129, 257, 700, 1024, 64, 3], wl.LAYOUT_PAGED, 83,
+                  rows_per_seq=True)
+    run = GpuRun(w, options=opts)
+    compare(run.logits(), oracle_logits(w), label=str(opts))
+    run.close()
+
+
 def test_tensor_core_wait_timeout_is_reported_and_the_handle_recovers():
     # the failure path of the bounded waits: one CTA of the output projection
     # never receives its first k-block, its MMA warp gives up after 1 ms, the
