@@ -27,8 +27,9 @@ __device__ __forceinline__ float block_sum(float v, float *red) {
     return warp_sum(t);
 }
 
-// One block per row, d % 8 == 0: 8-element vector loads, four chunks in
-// flight per thread.
+// RMSNorm for rows wider than the register-resident kernel below takes (d >
+// 8192): one block per row, d % 8 == 0, 8-element vector loads, four chunks in
+// flight per thread, two passes over the row.
 template <typename T>
 __global__ void __launch_bounds__(256) rmsnorm_rows_loop_kernel(const T *__restrict__ x, int row_mod,
                                                            const float *__restrict__ gain, float eps,
@@ -180,8 +181,9 @@ __global__ void __launch_bounds__(256) qkv_rope_rows_kernel(QkvRopeArgs a) {
     }
 }
 
-// h1 = x + y, n = RMSNorm(h1): one block per row, 4-element vectors.  Row m
-// reads x row (row_mod ? m % row_mod : m) and y row m / y_div.
+// h1 = x + y, n = RMSNorm(h1) for d > 8192: one block per row, 4-element
+// vectors, h1 re-read for the second pass.  Row m reads x row (row_mod ? m %
+// row_mod : m) and y row m / y_div (as the register-resident kernel below).
 template <typename TX>
 __global__ void __launch_bounds__(1024) residual_norm_loop_kernel(PartIn y, int y_div,
                                                              const TX *__restrict__ x,
