@@ -328,6 +328,16 @@ def test_work_split_and_query_precision_options(opts):
     run.close()
 
 
+def test_wide_model_takes_the_two_pass_norms():
+    # d > 8192 rows do not fit the register-resident norm kernels; the two-pass
+    # kernels serve them (input norm, residual + post-norm)
+    shape = wl.Shape(8448, 8, 2, 128, 1024, 8, 2)
+    w = wl.custom(shape, [64, 300, 1000], wl.LAYOUT_PAGED, 91, rows_per_seq=True)
+    run = GpuRun(w)
+    compare(run.logits(), oracle_logits(w), label="d = 8448")
+    run.close()
+
+
 def test_tensor_core_wait_timeout_is_reported_and_the_handle_recovers():
     # the failure path of the bounded waits: one CTA of the output projection
     # never receives its first k-block, its MMA warp gives up after 1 ms, the
