@@ -42,6 +42,10 @@ CASES = [
     ("contiguous", SMALL_BF16, [5, 129, 700], wl.LAYOUT_CONTIGUOUS),
     ("k1", wl.Shape(256, 8, 2, 128, 512, 1, 2), [40, 2000], wl.LAYOUT_PAGED),
     ("head_dim_64", wl.Shape(256, 8, 4, 64, 512, 3, 2), [90, 33], wl.LAYOUT_PAGED),
+    # 64 sequences x 8 rows and 48 heads: the Q/K/V projection runs one CTA per
+    # head with no K split, so the rotation happens in its epilogue
+    ("rotation_in_projection", wl.Shape(256, 32, 8, 128, 512, 8, 2),
+     [int(v) for v in np.random.default_rng(5).integers(0, 100, size=64)], wl.LAYOUT_PAGED),
 ]
 
 
