@@ -253,7 +253,8 @@ enum {
     SP_OPT_ATTN_SEG_COST = 6, /* tensor-core attention: the cost of a segment
                                  boundary, in 64-token tiles, that the cuts
                                  between CTA shares balance (-1..1024); -1 = the
-                                 built-in default.  Changes the work split only,
+                                 built-in default (12 for paged caches, 28 for
+                                 contiguous ones).  Changes the work split only,
                                  never the result beyond rounding order          */
     SP_OPT_ACT_PRECISION = 7, /* activations fed to the tensor-core
                                  projections: 0 = automatic (gate/up and down

@@ -221,7 +221,8 @@ sp_status enqueue_attention(AttnArgs &a, void *ws, size_t ws_bytes, int attn_pat
                             int seg_cost = -1, int merge_mode = 0) {
     a.tc_ctas = attn_tc_ctas(n_sm, a.Hkv);
     a.tc_min_tiles = forced_split > 0 ? forced_split / 64 : kAttnMinTiles;
-    a.tc_seg_cost = seg_cost >= 0 ? seg_cost : kAttnSegCost;
+    a.tc_seg_cost = seg_cost >= 0 ? seg_cost
+                                  : (a.kv.layout == SP_KV_CONTIGUOUS ? kAttnSegCostContiguous : kAttnSegCost);
     // few sequences over many groups: each pair has many partials, merged by a
     // kernel spread over (head, sequence, row) instead of one CTA per pair
     a.tc_merge_kernel = merge_mode == 2 || (merge_mode == 0 && 4 * a.B < a.tc_ctas / a.Hkv);

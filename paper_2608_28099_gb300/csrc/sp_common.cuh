@@ -241,6 +241,10 @@ constexpr int kAttnMinTiles = 8;
 // Default cost of a segment boundary in the tensor-core kernel, in 64-token
 // tiles (a pipeline drain, the epilogue and the next queries' load).
 constexpr int kAttnSegCost = 12;
+// The same for contiguous caches (cp.async tiles), measured on the 4B shape
+// (B = 16, ~16 tiles per share): 28 gave the attention 40.5 us against 42.6 us
+// at 12; on paged caches 20 was slower than 12 (27B long +1.3 us, 8B paged +6 us).
+constexpr int kAttnSegCostContiguous = 28;
 // Persistent CTAs of the tensor-core kernel: whole groups of Hkv (one CTA per
 // kv head), as many groups as the SMs hold, at least one.
 inline int attn_tc_ctas(int n_sm, int Hkv) { return (n_sm / Hkv > 1 ? n_sm / Hkv : 1) * Hkv; }
