@@ -777,7 +777,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         ++launches;
         mark(SP_STAGE_QKV, 0);
         s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, qkv_lo, 0,
-                        nullptr, false, rp);
+                        nullptr, rp);
         mark(SP_STAGE_QKV, 1);
         if (s != SP_OK) return fail(s, "Q/K/V projection launch failed");
         yqkv = PartIn{h->y, ns, stride_qkv};
@@ -788,7 +788,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
         ++launches;
         mark(SP_STAGE_QKV, 0);
         s = h->gemm.run(wb, h->opt_gemm, h->xn, h->w_qkv, h->y, M, h->status, st, &launches, &ns, qkv_lo, 0,
-                        nullptr, false, rp);
+                        nullptr, rp);
         mark(SP_STAGE_QKV, 1);
         if (s != SP_OK) return fail(s, "Q/K/V projection launch failed");
         yqkv = PartIn{h->y, ns, stride_qkv};
@@ -872,7 +872,7 @@ static sp_status classify_impl(sp_handle *h, cudaStream_t st, int batch, const i
     const bool glu = h->gu_blk == 64 && h->gemm.glu_fusable(h->w_gu, h->n, h->opt_gemm, M, mlp_lo);
     mark(SP_STAGE_GATE_UP, 0);
     s = h->gemm.run(wb, h->opt_gemm, h->n, h->w_gu, h->y, M, h->status, st, &launches, &ns, mlp_lo, 0,
-                    glu ? &a_out : nullptr, true);
+                    glu ? &a_out : nullptr);
     mark(SP_STAGE_GATE_UP, 1);
     if (s != SP_OK) return fail(s, "gate/up projection launch failed");
     if (!glu) {

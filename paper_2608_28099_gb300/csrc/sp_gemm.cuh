@@ -48,10 +48,9 @@ bool tc_supported(int N, int K);
 // MMA's N side is then 256) for M >= 256.
 int tc_bn_for(int M, bool lo = true);
 // sched: 0 = automatic, 1 = tile kernel, 2 = persistent stream-K (when its
-// partial planes fit).  keep_unsplit: a projection that fits one wave unsplit
-// stays unsplit (the gate/up projection's SwiGLU epilogue needs that).
+// partial planes fit).
 TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo = true,
-               int sched = 0, bool keep_unsplit = false);
+               int sched = 0);
 // w_blocked: the weights are stored blocked (block_weights_layout) and map_w
 // views them as [N K / 64][64] rows.
 cudaError_t launch_gemm_tc(const CUtensorMap &map_w, const CUtensorMap &map_xhi,
@@ -155,7 +154,7 @@ struct GemmPlanner {
     // run with the SwiGLU epilogue (one CTA per tile, no K split)?
     bool glu_fusable(const WeightMat &w, const ActBuf &x, int path, int M, bool lo) const {
         if (!use_tc(w, x, path)) return false;
-        const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched, true);
+        const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched);
         return !p.persistent && p.splits == 1 && p.bn >= 32;
     }
     // Would the Q/K/V projection run with the rotation epilogue (one CTA per
@@ -167,14 +166,14 @@ struct GemmPlanner {
     }
     // Enqueue the projection; *nsplit receives the number of partials in y.
     // glu: write silu(gate) * up there instead of partials (glu_fusable);
-    // gate_up: plan as glu_fusable does (whether or not glu is given).
+    // rope: the rotation epilogue (rope_fusable).
     sp_status run(int w_bf16, int path, const ActBuf &x, const WeightMat &w, float *y, int M,
                   int *status, cudaStream_t st, int *launches, int *nsplit, bool lo = true,
-                  int inject_stall = 0, const ActOut *glu = nullptr, bool gate_up = false,
+                  int inject_stall = 0, const ActOut *glu = nullptr,
                   const RopeEpi *rope = nullptr) const {
         cudaError_t e;
         if (use_tc(w, x, path)) {
-            const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched, gate_up || glu);
+            const TcPlan p = tc_plan(M, w.N, w.K, n_sm, y_capacity, lo, sched);
             const int bi = bn_index(p.bn);
             e = launch_gemm_tc(w.map, x.hi[bi], x.lo[bi], p, M, w.N, w.K, y, status, st, w.blocked, lo,
                                inject_stall, glu, rope);

@@ -710,8 +710,7 @@ static int planes_for(long long tiles, int n_kb, long long L) {
     return most;
 }
 
-TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo, int sched,
-               bool keep_unsplit) {
+TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo, int sched) {
     TcPlan p;
     p.nt = 1;
     p.bn = tc_bn_for(M, lo);
@@ -755,7 +754,7 @@ TcPlan tc_plan(int M, int N, int K, int n_sm, size_t y_capacity_bytes, bool lo, 
         while (S2 > 1 && (size_t)S2 * M * N * sizeof(float) > y_capacity_bytes) --S2;
         const int kbs2 = ceil_div(p.n_kb, S2);
         S2 = ceil_div(p.n_kb, kbs2);
-        (void)keep_unsplit;  // S2 <= splits keeps an unsplit projection unsplit
+        // (S2 <= splits also keeps an unsplit gate/up unsplit for its SwiGLU epilogue)
         if (S2 <= p.splits && pairs * S2 <= n_sm && pairs * S2 * 100 >= n_sm * 85) {
             p.nt = 2;
             p.kb_per_split = kbs2;
