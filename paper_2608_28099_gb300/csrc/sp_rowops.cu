@@ -362,18 +362,18 @@ __global__ void swiglu_kernel(PartIn y, int M, int f, int blk, ActOut a) {
 }
 
 // Pooling and the linear head, column-parallel: block (chunk, b) pools 256
-// hidden columns of sequence b (h2 = h1 + y summed over the k rows by two row
+// hidden columns of sequence b (h2 = h1 + y summed over the k rows by four row
 // groups, four columns per thread with 16-byte loads, then mean or last) and
 // writes its partial dot products with every head row to part[b][chunk][C];
-// two classes are reduced at a time.
+// four classes are reduced at a time (one per row group).
 constexpr int kReadoutCols = 256;
-constexpr int kReadoutGroups = 2;  // row groups of a block (threads = 64 x 2)
+constexpr int kReadoutGroups = 4;  // row groups of a block (threads = 64 x 4)
 
 __device__ __forceinline__ float4 f4_add(float4 a, float4 b) {
     return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
 }
 
-__global__ void __launch_bounds__(64 * kReadoutGroups, 4)
+__global__ void __launch_bounds__(64 * kReadoutGroups, 2)
 readout_partial_kernel(PartIn y, const float *__restrict__ h1, const float *__restrict__ head_w,
                        int pool, int k, int d, int C, float *__restrict__ part, size_t sb, size_t sr,
                        int n_tasks, const float *__restrict__ g_final, float *__restrict__ part_ss,
@@ -399,7 +399,7 @@ readout_partial_kernel(PartIn y, const float *__restrict__ h1, const float *__re
     if (in_d) {
         // rows rg, rg + G, ... (G row groups) four at a time (all rows when
         // pooling the last one is a single row), the loads of their h1 values
-        // and of two partials each issued together
+        // and of up to four partials each issued together
         const int r_first = pool == SP_POOL_LAST ? k - 1 : rg;
         const int r_step = pool == SP_POOL_LAST ? k : kReadoutGroups;
         if (pool != SP_POOL_LAST || rg == 0) {
@@ -414,19 +414,19 @@ readout_partial_kernel(PartIn y, const float *__restrict__ h1, const float *__re
                     o[u] = base + (size_t)(in[u] ? r : r0) * sr + col;
                     v[u] = in[u] ? *(const float4 *)(h1 + o[u]) : make_float4(0.f, 0.f, 0.f, 0.f);
                 }
-                for (int i0 = 0; i0 < y.n; i0 += 2) {
-                    float4 pv[4][2];
+                for (int i0 = 0; i0 < y.n; i0 += 4) {  // up to four planes per round
+                    float4 pv[4][4];
 #pragma unroll
                     for (int u = 0; u < 4; ++u)
 #pragma unroll
-                        for (int jj = 0; jj < 2; ++jj)
+                        for (int jj = 0; jj < 4; ++jj)
                             pv[u][jj] = (in[u] && i0 + jj < y.n)
                                             ? *(const float4 *)(y.y + (size_t)(i0 + jj) * y.stride + o[u])
                                             : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
                     for (int u = 0; u < 4; ++u)
 #pragma unroll
-                        for (int jj = 0; jj < 2; ++jj) v[u] = f4_add(v[u], pv[u][jj]);
+                        for (int jj = 0; jj < 4; ++jj) v[u] = f4_add(v[u], pv[u][jj]);
                 }
                 acc = f4_add(acc, f4_add(f4_add(v[0], v[1]), f4_add(v[2], v[3])));
             }
