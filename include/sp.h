@@ -298,13 +298,16 @@ enum {
 enum {
     SP_STAGE_INPUT_NORM = 0,  /* a1: RMSNorm of per-sequence rows                    */
     SP_STAGE_QKV = 1,         /* a2: Q/K/V projection (skipped for the shared prompt) */
-    SP_STAGE_ROPE = 2,        /* a2: rotation at L_b + r, new keys to scratch        */
+    SP_STAGE_ROPE = 2,        /* a2: rotation at L_b + r, new keys to scratch (not
+                                 a stage of its own when the Q/K/V projection's
+                                 epilogue rotates: reported as -1 then)           */
     SP_STAGE_ATTN = 3,        /* a3: split-KV attention over [cache ; new keys]      */
     SP_STAGE_MERGE = 4,       /* a3: log-sum-exp merge of the splits                 */
     SP_STAGE_O_PROJ = 5,      /* a4: output projection                               */
     SP_STAGE_POST_NORM = 6,   /* a4: residual + post-norm                            */
     SP_STAGE_GATE_UP = 7,     /* a5: gate/up projection                              */
-    SP_STAGE_SWIGLU = 8,      /* a5: SwiGLU                                          */
+    SP_STAGE_SWIGLU = 8,      /* a5: SwiGLU (-1 when the gate/up projection's
+                                 epilogue applies it)                             */
     SP_STAGE_DOWN = 9,        /* a6: down projection                                 */
     SP_STAGE_READOUT = 10,    /* a6-a7: residual, pooling, linear head               */
     SP_STAGE_FUSION = 11,     /* input fusion: hidden-state norm and its W_fc

@@ -30,6 +30,28 @@ def lib():
     return sp.load_library()
 
 
+def header_constants():
+    """Every `SP_NAME = value` of the enums in include/sp.h."""
+    text = open(os.path.join(ROOT, "include", "sp.h")).read()
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    return {m.group(1): int(m.group(2)) for m in re.finditer(r"\b(SP_[A-Z0-9_]+)\s*=\s*(-?\d+)", text)}
+
+
+def test_binding_constants_match_the_header():
+    consts = header_constants()
+    assert len(consts) > 30
+    for name, value in consts.items():
+        if name.startswith(("SP_OPT_", "SP_STAGE_", "SP_DEV_", "SP_ERR_", "SP_OK", "SP_POOL_",
+                            "SP_KV_", "SP_F32", "SP_BF16")) and name != "SP_N_STAGES":
+            assert hasattr(sp, name) or name.startswith("SP_STAGE_"), name
+            if hasattr(sp, name):
+                assert getattr(sp, name) == value, name
+    stages = sorted((v, n) for n, v in consts.items() if n.startswith("SP_STAGE_"))
+    header_names = [n[len("SP_STAGE_"):].lower() for _, n in stages]
+    assert [{"attn": "attention"}.get(x, x) for x in header_names] == sp.STAGES
+    assert consts["SP_N_STAGES"] == len(sp.STAGES)
+
+
 def test_every_declared_symbol_is_exported(lib):
     names = declared_symbols()
     assert len(names) >= 10
