@@ -297,6 +297,26 @@ def test_device_status_reports_bad_inputs():
     run.close()
 
 
+def test_empty_and_oversized_batches_are_refused_before_any_launch():
+    # batch must lie in 1..max_batch: an empty batch and one beyond the handle's
+    # max_batch are refused on the host (nothing is enqueued), and the handle
+    # stays usable
+    torch = torch_dev()
+    w = wl.custom(SMALL_BF16, [20, 40], wl.LAYOUT_PAGED, 141)
+    run = GpuRun(w, max_batch=2, max_seq_len=64)
+    h = run.model.handle
+    out = torch.full((3, SMALL_BF16.n_classes), 7.0, dtype=torch.float32, device="cuda")
+    st = torch.cuda.current_stream()
+    for batch in (0, 3):
+        with pytest.raises(sp.SpError) as e:
+            sp.sp_classify(h, st, batch, None, run.cache.seq_lens, run.cache.desc, None, out)
+        assert e.value.status == sp.SP_ERR_INVALID_ARG
+    torch.cuda.synchronize()
+    assert bool((out == 7.0).all())
+    compare(run.logits(use_rows=False), oracle_logits(w, use_rows=False))
+    run.close()
+
+
 @pytest.mark.parametrize("prec", [0, 1, 2, 3, 4])
 def test_mlp_activation_precision_options(prec):
     # automatic (bf16 MLP inputs here: mean over 8 rows), hi + lo, plain bf16
