@@ -398,6 +398,45 @@ def check_tasks_are_isolated_and_permutable():
     np.testing.assert_array_equal(c, a[:, perm])
 
 
+def check_task_rows_belong_to_their_task():
+    """Per-sequence rows [B, T, k, d]: task t reads its own rows rows[:, t] and
+    nothing else (task 0 is the single-task path on rows[:, 0]; changing task
+    1's rows changes task 1 only)."""
+    sh, w = random_layer(56)
+    layer = so.Layer(sh, w)
+    cw = wl.custom(sh, [3, 10], wl.LAYOUT_PAGED, 57)
+    prompts, heads, biases = _tasks(58, 2, sh)
+    rng = np.random.default_rng(59)
+    rows = f32(rng.standard_normal((2, 2, sh.k_rows, sh.d_model)) * 0.4)
+    a = so.classify_tasks(layer, cw.cache, cw.seq_ids, prompts, heads, biases, rows=rows)
+    t0 = so.Layer(sh, dataclasses.replace(w, head_w=heads[0], head_b=biases[0]))
+    np.testing.assert_array_equal(a[:, 0], so.classify(t0, cw.cache, cw.seq_ids, rows=rows[:, 0]))
+    rows2 = rows.copy()
+    rows2[:, 1] = rows2[:, 1, ::-1] * 2
+    b = so.classify_tasks(layer, cw.cache, cw.seq_ids, prompts, heads, biases, rows=rows2)
+    np.testing.assert_array_equal(a[:, 0], b[:, 0])
+    assert np.max(np.abs(a[:, 1] - b[:, 1])) > 1e-6
+
+
+def check_norm_gains_fold_into_the_next_projection():
+    """An RMSNorm gain scales channels of the normalised rows that feed only the
+    next projection: g_in * s with the columns of W_q, W_k, W_v divided by s,
+    or g_post * s with the columns of W_gate, W_up divided by s, leaves every
+    logit unchanged for any positive s; either gain scaled alone changes them."""
+    sh, w = random_layer(60)
+    cw = wl.custom(sh, [6, 17], wl.LAYOUT_CONTIGUOUS, 61)
+    s = f32(np.random.default_rng(62).uniform(0.5, 2.0, sh.d_model))
+    run = lambda ww: so.classify(so.Layer(sh, ww), cw.cache, cw.seq_ids)
+    base = run(w)
+    folded_in = dataclasses.replace(w, g_in=w.g_in * s, w_q=w.w_q / s, w_k=w.w_k / s, w_v=w.w_v / s)
+    folded_post = dataclasses.replace(w, g_post=w.g_post * s, w_gate=w.w_gate / s, w_up=w.w_up / s)
+    # the folded weights are rounded to fp32 like the originals: compare loosely
+    np.testing.assert_allclose(run(folded_in), base, rtol=1e-5, atol=1e-6)
+    np.testing.assert_allclose(run(folded_post), base, rtol=1e-5, atol=1e-6)
+    for alone in (dataclasses.replace(w, g_in=w.g_in * s), dataclasses.replace(w, g_post=w.g_post * s)):
+        assert np.max(np.abs(run(alone) - base)) > 1e-3
+
+
 def check_lm_head_readout_hand_example():
     g = read_golden("lm_head_readout_d2.txt")
     sh = wl.Shape(2, 1, 1, 2, 1, 2, 2, rms_eps=0.0, w_dtype=wl.F32, kv_dtype=wl.F32)
@@ -483,6 +522,7 @@ ALL_CHECKS = [check_bf16_decode_fixed_patterns, check_attention_step_matches_the
               check_attention_step_uniform_keys_closed_form,
               check_lm_head_readout_hand_example, check_lm_head_readout_is_scale_invariant,
               check_one_task_is_the_single_task_path, check_tasks_are_isolated_and_permutable,
+              check_task_rows_belong_to_their_task, check_norm_gains_fold_into_the_next_projection,
               check_recursive_k1_equals_parallel_fused,
               check_recursive_equals_stepwise_reconstruction,
               check_recursive_embedding_only_is_the_row_path,
@@ -668,6 +708,33 @@ def _bf16_low_half(orig):
     return f
 
 
+def _post_norm_takes_input_gain(orig):
+    def f(self, x, o):
+        saved, self.g_post = self.g_post, self.g_in
+        try:
+            return orig(self, x, o)
+        finally:
+            self.g_post = saved
+    return f
+
+
+def _input_norm_takes_post_gain(orig):
+    def f(self, x, positions):
+        saved, self.g_in = self.g_in, self.g_post
+        try:
+            return orig(self, x, positions)
+        finally:
+            self.g_in = saved
+    return f
+
+
+def _task_rows_of_first_task(orig):
+    def f(layer, cache, seq_ids, prompts, heads, biases=None, rows=None, hidden=None):
+        r = None if rows is None else np.repeat(rows[:, :1], rows.shape[1], axis=1)
+        return orig(layer, cache, seq_ids, prompts, heads, biases, r, hidden)
+    return f
+
+
 def _attention_step_mask_off_by_one(orig):
     def f(shape, cache, seq_ids, q, k_new, v_new):
         kr = q.shape[1]
@@ -713,6 +780,9 @@ MUTANTS = {
     "gate_up_swapped": (so.Layer, "finish", _gate_up_swapped),
     "readout_first_row": (so.Layer, "readout", _readout_first_row),
     "paged_gather_reversed": (so, "sequence_kv", _gather_reversed),
+    "post_norm_takes_input_gain": (so.Layer, "finish", _post_norm_takes_input_gain),
+    "input_norm_takes_post_gain": (so.Layer, "project_qkv", _input_norm_takes_post_gain),
+    "task_rows_of_first_task": (so, "classify_tasks", _task_rows_of_first_task),
 }
 
 
