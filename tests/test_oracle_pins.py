@@ -8,6 +8,7 @@ case that reduces to something simpler, or an independent library routine.
 """
 import dataclasses
 import hashlib
+import math
 
 import numpy as np
 import pytest
@@ -103,6 +104,21 @@ def check_rope_relative_and_norm():
     np.testing.assert_allclose(s1, s2, rtol=1e-10)
 
 
+def check_rope_frequencies_follow_theta():
+    """Pair i turns by p * theta^(-2i/dh): at theta = 100, p = 3, dh = 4 pair 0
+    turns 3 rad and pair 1 turns 3 / 10 = 0.3 rad; at dh = 8 pair 3 turns
+    3 * 100^(-3/4) rad (closed forms from the definition of the frequencies)."""
+    e0, e1 = np.eye(4)[0].reshape(1, 1, 4), np.eye(4)[1].reshape(1, 1, 4)
+    np.testing.assert_allclose(so.rope(e0, np.array([3]), 100.0).ravel(),
+                               [math.cos(3.0), 0.0, math.sin(3.0), 0.0], atol=1e-12)
+    np.testing.assert_allclose(so.rope(e1, np.array([3]), 100.0).ravel(),
+                               [0.0, math.cos(0.3), 0.0, math.sin(0.3)], atol=1e-12)
+    e3 = np.eye(8)[3].reshape(1, 1, 8)
+    a = 3.0 * 100.0 ** -0.75
+    np.testing.assert_allclose(so.rope(e3, np.array([3]), 100.0).ravel(),
+                               [0, 0, 0, math.cos(a), 0, 0, 0, math.sin(a)], atol=1e-12)
+
+
 def check_softmax_rows_sum_to_one():
     sh, w = random_layer(1)
     layer = so.Layer(sh, w)
@@ -113,6 +129,10 @@ def check_softmax_rows_sum_to_one():
     layer.rows_with_cache(layer.soft_prompt, kc, kc * 0.5, trace=tr)
     sums = tr["p"].sum(axis=-1)
     np.testing.assert_allclose(sums, 1.0, atol=1e-12)
+    # scores far beyond exp's range: [1000, 999] -> [1, e^-1] / (1 + e^-1)
+    e = math.exp(-1.0)
+    np.testing.assert_allclose(so.softmax_rows(np.array([[1000.0, 999.0]])), [[1 / (1 + e), e / (1 + e)]],
+                               rtol=1e-12)
     # row r sees exactly L + r + 1 keys
     for r in range(sh.k_rows):
         nz = np.count_nonzero(tr["p"][r], axis=-1)
@@ -437,6 +457,29 @@ def check_norm_gains_fold_into_the_next_projection():
         assert np.max(np.abs(run(alone) - base)) > 1e-3
 
 
+def check_classify_follows_the_sequence_ids():
+    """Logits of a batch of ids are the per-sequence logits in the ids' order
+    (sequences of different lengths, so any mix-up shows)."""
+    sh, w = random_layer(64)
+    layer = so.Layer(sh, w)
+    cw = wl.custom(sh, [2, 9, 14], wl.LAYOUT_PAGED, 65)
+    ref = so.classify(layer, cw.cache, np.arange(3))
+    for ids in ([2, 0, 1], [1, 1]):
+        ids = np.array(ids, dtype=np.int32)
+        np.testing.assert_array_equal(so.classify(layer, cw.cache, ids), ref[ids])
+    assert np.max(np.abs(ref[0] - ref[2])) > 1e-6
+
+
+def check_lm_head_readout_eps_inside_the_root():
+    # a constant pooled vector c with gain 1 and head I normalises to
+    # c / sqrt(c^2 + eps): 0.5 / sqrt(0.25 + 0.75) = 0.5
+    sh = wl.Shape(2, 1, 1, 2, 1, 2, 2, rms_eps=0.75, w_dtype=wl.F32, kv_dtype=wl.F32)
+    _, w = random_layer(66, d=2, hq=1, hkv=1, dh=2, f=1, k=2, C=2)
+    w = dataclasses.replace(w, head_w=np.eye(2), head_b=None, g_final=f32([1.0, 1.0]))
+    z = so.Layer(sh, w).readout(np.full((2, 2), 0.5))
+    np.testing.assert_allclose(z, [0.5, 0.5], rtol=1e-12)
+
+
 def check_lm_head_readout_hand_example():
     g = read_golden("lm_head_readout_d2.txt")
     sh = wl.Shape(2, 1, 1, 2, 1, 2, 2, rms_eps=0.0, w_dtype=wl.F32, kv_dtype=wl.F32)
@@ -523,6 +566,8 @@ ALL_CHECKS = [check_bf16_decode_fixed_patterns, check_attention_step_matches_the
               check_lm_head_readout_hand_example, check_lm_head_readout_is_scale_invariant,
               check_one_task_is_the_single_task_path, check_tasks_are_isolated_and_permutable,
               check_task_rows_belong_to_their_task, check_norm_gains_fold_into_the_next_projection,
+              check_rope_frequencies_follow_theta, check_classify_follows_the_sequence_ids,
+              check_lm_head_readout_eps_inside_the_root,
               check_recursive_k1_equals_parallel_fused,
               check_recursive_equals_stepwise_reconstruction,
               check_recursive_embedding_only_is_the_row_path,
@@ -735,6 +780,34 @@ def _task_rows_of_first_task(orig):
     return f
 
 
+def _rope_theta_fixed(orig):
+    return lambda x, positions, theta: orig(x, positions, 1.0e4)
+
+
+def _softmax_without_shift(orig):
+    def f(s):
+        e = np.exp(s)
+        return e / e.sum(axis=-1, keepdims=True)
+    return f
+
+
+def _sequence_ids_ignored(orig):
+    def f(layer, cache, seq_ids, rows=None, traces=None, hidden=None):
+        return orig(layer, cache, np.arange(len(seq_ids)), rows, traces, hidden)
+    return f
+
+
+def _readout_eps_dropped(orig):
+    def f(self, h2):
+        saved = self.shape
+        self.shape = dataclasses.replace(saved, rms_eps=0.0)
+        try:
+            return orig(self, h2)
+        finally:
+            self.shape = saved
+    return f
+
+
 def _attention_step_mask_off_by_one(orig):
     def f(shape, cache, seq_ids, q, k_new, v_new):
         kr = q.shape[1]
@@ -783,6 +856,10 @@ MUTANTS = {
     "post_norm_takes_input_gain": (so.Layer, "finish", _post_norm_takes_input_gain),
     "input_norm_takes_post_gain": (so.Layer, "project_qkv", _input_norm_takes_post_gain),
     "task_rows_of_first_task": (so, "classify_tasks", _task_rows_of_first_task),
+    "rope_theta_fixed_at_1e4": (so, "rope", _rope_theta_fixed),
+    "softmax_without_max_shift": (so, "softmax_rows", _softmax_without_shift),
+    "sequence_ids_ignored": (so, "classify", _sequence_ids_ignored),
+    "lm_readout_eps_dropped": (so.Layer, "readout", _readout_eps_dropped),
 }
 
 
