@@ -202,6 +202,55 @@ def check_uniform_keys_give_mean_of_values():
                                        rtol=1e-12, atol=1e-12)
 
 
+def check_head_blocks_and_group_map():
+    """Head layout of Eq. 1-3 with G = Hq / Hkv = 2, dh = 2, d = Hq * dh: rows
+    h*dh..h*dh+dh-1 of W_q form query head h, which reads KV head h // G, and
+    the attention output enters W_o head-major.  With W_k = W_v = 0 (new keys and
+    values are zero), cache values constant per KV head (c_j) and W_q nonzero for
+    head 0 only, every head but 0 scores all keys equal, so its output is
+    L / (L + r + 1) * c_{h // G}; head 0's is a different multiple of c_0.  W_o = I
+    and W_down = 0 put the outputs in h2 - x."""
+    hq, hkv, dh, L = 4, 2, 2, 5
+    d = hq * dh
+    sh, w = random_layer(67, d=d, hq=hq, hkv=hkv, dh=dh, f=3, k=2)
+    rng = np.random.default_rng(68)
+    wq = np.zeros((hq * dh, d))
+    wq[:dh] = rng.standard_normal((dh, d)) * 2.0
+    w = dataclasses.replace(w, w_q=f32(wq), w_k=f32(np.zeros((hkv * dh, d))),
+                            w_v=f32(np.zeros((hkv * dh, d))), w_o=f32(np.eye(d)),
+                            w_down=f32(np.zeros((d, sh.d_ff))))
+    layer = so.Layer(sh, w)
+    c = np.array([[1.0, -2.0], [3.0, 0.5]])                  # value of KV head j
+    kc = rng.standard_normal((L, hkv, dh)) * 2.0
+    vc = np.repeat(c[None], L, axis=0)
+    x = rng.standard_normal((sh.k_rows, d))
+    o = (layer.rows_with_cache(x, kc, vc) - x).reshape(sh.k_rows, hq, dh)
+    for r in range(sh.k_rows):
+        for h in range(1, hq):
+            np.testing.assert_allclose(o[r, h], L / (L + r + 1) * c[h // 2], rtol=1e-12, atol=1e-12)
+        a = o[r, 0] / c[0]
+        np.testing.assert_allclose(a[0], a[1], rtol=1e-12)
+        assert 0.0 < a[0] < 1.0 and abs(a[0] - L / (L + r + 1)) > 1e-3
+
+
+def check_hand_built_cache_matches_full_recompute():
+    """A one-token cache built by hand in the [token][KV head][dh] layout: the
+    context row has unit rms, the input gain is 1 and eps 0, so its normalised
+    row is itself, and rotation at position 0 is the identity; its key and value
+    are then W_k x and W_v x split head-major.  The cached pass of the soft rows
+    must equal the full causal pass over [context; soft rows] (Eq. 1-3)."""
+    sh, w = random_layer(69, d=16, hq=4, hkv=2, dh=4, k=3, eps=0.0)
+    w = dataclasses.replace(w, g_in=f32(np.ones(16)))
+    layer = so.Layer(sh, w)
+    xc = np.random.default_rng(70).standard_normal(16)
+    xc = xc / np.sqrt(np.mean(xc * xc))
+    kc = (np.asarray(w.w_k, np.float64) @ xc).reshape(1, 2, 4)
+    vc = (np.asarray(w.w_v, np.float64) @ xc).reshape(1, 2, 4)
+    full = layer.full_causal(np.vstack([xc[None], layer.soft_prompt]))[1:]
+    np.testing.assert_allclose(layer.rows_with_cache(layer.soft_prompt, kc, vc), full,
+                               rtol=1e-10, atol=1e-12)
+
+
 def check_rms_norm():
     rng = np.random.default_rng(8)
     x = rng.standard_normal((5, 32))
@@ -286,6 +335,17 @@ def check_fusion_hand_example():
     layer = so.Layer(sh, w)
     x = layer.fuse(np.array([g["h"]]), np.array([g["e"]]))
     np.testing.assert_allclose(x.ravel(), g["x"], atol=1e-9)
+
+
+def check_fusion_eps_inside_the_root():
+    # constant rows 0.5 with eps = 0.75 and unit gains normalise to
+    # 0.5 / sqrt(0.25 + 0.75) = 0.5 each; W_fc = [I | I] adds the two halves
+    sh = wl.Shape(2, 1, 1, 2, 1, 1, 2, rms_eps=0.75, w_dtype=wl.F32, kv_dtype=wl.F32)
+    _, w = random_layer(31, d=2, hq=1, hkv=1, dh=2, f=1, k=1, C=2)
+    w = dataclasses.replace(w, w_fc=f32(np.concatenate([np.eye(2), np.eye(2)], axis=1)),
+                            g_h=f32([1.0, 1.0]), g_e=f32([1.0, 1.0]))
+    x = so.Layer(sh, w).fuse(np.full((1, 2), 0.5), np.full((1, 2), 0.5))
+    np.testing.assert_allclose(x, [[1.0, 1.0]], rtol=1e-12)
 
 
 def fused_layer(seed, w_fc_kind, unit_rows=False):
@@ -567,7 +627,8 @@ ALL_CHECKS = [check_bf16_decode_fixed_patterns, check_attention_step_matches_the
               check_one_task_is_the_single_task_path, check_tasks_are_isolated_and_permutable,
               check_task_rows_belong_to_their_task, check_norm_gains_fold_into_the_next_projection,
               check_rope_frequencies_follow_theta, check_classify_follows_the_sequence_ids,
-              check_lm_head_readout_eps_inside_the_root,
+              check_lm_head_readout_eps_inside_the_root, check_fusion_eps_inside_the_root,
+              check_head_blocks_and_group_map, check_hand_built_cache_matches_full_recompute,
               check_recursive_k1_equals_parallel_fused,
               check_recursive_equals_stepwise_reconstruction,
               check_recursive_embedding_only_is_the_row_path,
@@ -808,6 +869,37 @@ def _readout_eps_dropped(orig):
     return f
 
 
+def _o_flattened_dim_major(orig):
+    def f(self, x, o):
+        return orig(self, x, np.ascontiguousarray(o.transpose(0, 2, 1)).reshape(o.shape))
+    return f
+
+
+def _query_heads_reversed(orig):
+    def f(self, x, positions):
+        q, k, v = orig(self, x, positions)
+        return q[:, ::-1].copy(), k, v
+    return f
+
+
+def _kv_heads_reversed(orig):
+    def f(self, x, positions):
+        q, k, v = orig(self, x, positions)
+        return q, k[:, ::-1].copy(), v[:, ::-1].copy()
+    return f
+
+
+def _fusion_eps_dropped(orig):
+    def f(self, hidden, embed):
+        saved = self.shape
+        self.shape = dataclasses.replace(saved, rms_eps=0.0)
+        try:
+            return orig(self, hidden, embed)
+        finally:
+            self.shape = saved
+    return f
+
+
 def _attention_step_mask_off_by_one(orig):
     def f(shape, cache, seq_ids, q, k_new, v_new):
         kr = q.shape[1]
@@ -860,6 +952,10 @@ MUTANTS = {
     "softmax_without_max_shift": (so, "softmax_rows", _softmax_without_shift),
     "sequence_ids_ignored": (so, "classify", _sequence_ids_ignored),
     "lm_readout_eps_dropped": (so.Layer, "readout", _readout_eps_dropped),
+    "o_flattened_dim_major": (so.Layer, "finish", _o_flattened_dim_major),
+    "query_heads_reversed": (so.Layer, "project_qkv", _query_heads_reversed),
+    "kv_heads_reversed": (so.Layer, "project_qkv", _kv_heads_reversed),
+    "fusion_eps_dropped": (so.Layer, "fuse", _fusion_eps_dropped),
 }
 
 
