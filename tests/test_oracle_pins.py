@@ -308,13 +308,14 @@ def check_k1_mean_equals_last():
 
 def check_paged_gather_matches_contiguous():
     sh = wl.Shape(64, 4, 2, 16, 64, 2, 2, w_dtype=wl.BF16, kv_dtype=wl.BF16)
-    w = wl.custom(sh, [0, 1, 15, 16, 17, 40], wl.LAYOUT_CONTIGUOUS, 21)
-    paged = wl.contiguous_to_paged(w.cache, 16, 5)
-    for b in range(6):
-        k1, v1 = so.sequence_kv(w.cache, b)
-        k2, v2 = so.sequence_kv(paged, b)
-        assert k1.shape == (int(w.cache.seq_lens[b]), 2, 16)
-        assert np.array_equal(k1, k2) and np.array_equal(v1, v2)
+    w = wl.custom(sh, [0, 1, 15, 16, 17, 40, 65, 130], wl.LAYOUT_CONTIGUOUS, 21)
+    for P in (16, 32, 64):  # every page size the classify path takes
+        paged = wl.contiguous_to_paged(w.cache, P, 5 + P)
+        for b in range(8):
+            k1, v1 = so.sequence_kv(w.cache, b)
+            k2, v2 = so.sequence_kv(paged, b)
+            assert k1.shape == (int(w.cache.seq_lens[b]), 2, 16)
+            assert np.array_equal(k1, k2) and np.array_equal(v1, v2)
 
 
 def check_cache_untouched():
@@ -900,6 +901,21 @@ def _fusion_eps_dropped(orig):
     return f
 
 
+def _page_size_fixed_at_16(orig):
+    def f(cache, seq_id):
+        if cache.layout != so.LAYOUT_PAGED or cache.page_size == 16:
+            return orig(cache, seq_id)
+        # the pool's slots read as if pages held 16 tokens
+        L = int(cache.seq_lens[seq_id])
+        n_pg = (L + 15) // 16
+        pages = cache.page_table[seq_id, :n_pg]
+        hkv, dh = cache.k_pool.shape[1], cache.k_pool.shape[3]
+        kp = cache.k_pool[pages][:, :, :16].transpose(0, 2, 1, 3).reshape(n_pg * 16, hkv, dh)[:L]
+        vp = cache.v_pool[pages][:, :, :16].transpose(0, 2, 1, 3).reshape(n_pg * 16, hkv, dh)[:L]
+        return so.to_f64(kp, cache.dtype), so.to_f64(vp, cache.dtype)
+    return f
+
+
 def _attention_step_mask_off_by_one(orig):
     def f(shape, cache, seq_ids, q, k_new, v_new):
         kr = q.shape[1]
@@ -956,6 +972,7 @@ MUTANTS = {
     "query_heads_reversed": (so.Layer, "project_qkv", _query_heads_reversed),
     "kv_heads_reversed": (so.Layer, "project_qkv", _kv_heads_reversed),
     "fusion_eps_dropped": (so.Layer, "fuse", _fusion_eps_dropped),
+    "page_size_fixed_at_16": (so, "sequence_kv", _page_size_fixed_at_16),
 }
 
 
