@@ -395,6 +395,25 @@ def check_fusion_with_hidden_only_ignores_the_prompt():
     assert np.max(np.abs(a - c)) > 1e-6
 
 
+def check_tasks_with_hidden_fuse_their_own_prompt():
+    """Several tasks over MTP inputs: task t fuses the hidden state with its own
+    prompt (task 0 equals the single-task fused path with its prompt and head;
+    changing task 1's prompt changes task 1 only)."""
+    sh, w = fused_layer(37, "mixed")
+    layer = so.Layer(sh, w)
+    cw = wl.custom(sh, [5, 12], wl.LAYOUT_PAGED, 38)
+    hidden = f32(np.random.default_rng(39).standard_normal((2, sh.d_model)))
+    prompts, heads, biases = _tasks(40, 2, sh)
+    a = so.classify_tasks(layer, cw.cache, cw.seq_ids, prompts, heads, biases, hidden=hidden)
+    t0 = so.Layer(sh, dataclasses.replace(w, soft_prompt=prompts[0], head_w=heads[0], head_b=biases[0]))
+    np.testing.assert_array_equal(a[:, 0], so.classify(t0, cw.cache, cw.seq_ids, hidden=hidden))
+    p2 = prompts.copy()
+    p2[1] = p2[1][::-1] * 2
+    b = so.classify_tasks(layer, cw.cache, cw.seq_ids, p2, heads, biases, hidden=hidden)
+    np.testing.assert_array_equal(a[:, 0], b[:, 0])
+    assert np.max(np.abs(a[:, 1] - b[:, 1])) > 1e-6
+
+
 def check_recursive_k1_equals_parallel_fused():
     sh, w = fused_layer(40, "random")
     sh = dataclasses.replace(sh, k_rows=1)
@@ -598,6 +617,11 @@ def check_attention_step_matches_the_layer_trace():
         q.append(tr["q"]); kn.append(tr["k_new"]); vn.append(tr["v_new"]); want.append(tr["o"])
     got = so.attention_step(sh, w.cache, w.seq_ids, np.array(q), np.array(kn), np.array(vn))
     np.testing.assert_allclose(got, np.array(want), rtol=1e-12, atol=1e-12)
+    # batch slot i reads the cache of seq_ids[i]: a permuted batch permutes the outputs
+    perm = np.array([3, 0, 4, 1, 2])
+    got_p = so.attention_step(sh, w.cache, w.seq_ids[perm], np.array(q)[perm], np.array(kn)[perm],
+                              np.array(vn)[perm])
+    np.testing.assert_allclose(got_p, np.array(want)[perm], rtol=1e-12, atol=1e-12)
 
 
 def check_attention_step_uniform_keys_closed_form():
@@ -630,6 +654,7 @@ ALL_CHECKS = [check_bf16_decode_fixed_patterns, check_attention_step_matches_the
               check_rope_frequencies_follow_theta, check_classify_follows_the_sequence_ids,
               check_lm_head_readout_eps_inside_the_root, check_fusion_eps_inside_the_root,
               check_head_blocks_and_group_map, check_hand_built_cache_matches_full_recompute,
+              check_tasks_with_hidden_fuse_their_own_prompt,
               check_recursive_k1_equals_parallel_fused,
               check_recursive_equals_stepwise_reconstruction,
               check_recursive_embedding_only_is_the_row_path,
@@ -916,6 +941,20 @@ def _page_size_fixed_at_16(orig):
     return f
 
 
+def _tasks_fuse_the_layer_prompt(orig):
+    def f(layer, cache, seq_ids, prompts, heads, biases=None, rows=None, hidden=None):
+        if hidden is not None:  # every task fuses with the handle's own prompt
+            prompts = np.repeat(layer.soft_prompt[None].astype(np.float32), len(prompts), axis=0)
+        return orig(layer, cache, seq_ids, prompts, heads, biases, rows, hidden)
+    return f
+
+
+def _attention_step_ids_ignored(orig):
+    def f(shape, cache, seq_ids, q, k_new, v_new):
+        return orig(shape, cache, np.arange(len(seq_ids)), q, k_new, v_new)
+    return f
+
+
 def _attention_step_mask_off_by_one(orig):
     def f(shape, cache, seq_ids, q, k_new, v_new):
         kr = q.shape[1]
@@ -973,6 +1012,8 @@ MUTANTS = {
     "kv_heads_reversed": (so.Layer, "project_qkv", _kv_heads_reversed),
     "fusion_eps_dropped": (so.Layer, "fuse", _fusion_eps_dropped),
     "page_size_fixed_at_16": (so, "sequence_kv", _page_size_fixed_at_16),
+    "tasks_fuse_the_layer_prompt": (so, "classify_tasks", _tasks_fuse_the_layer_prompt),
+    "attention_step_ids_ignored": (so, "attention_step", _attention_step_ids_ignored),
 }
 
 
