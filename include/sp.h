@@ -416,6 +416,30 @@ SP_API size_t sp_project_workspace_bytes(int M, int N, int K);
  * SP_ERR_UNSUPPORTED otherwise), 0 = tensor cores when supported.  The tensor
  * path splits X into bf16 hi + lo parts and may split K across CTAs; both live
  * in d_workspace (>= sp_project_workspace_bytes, 256-byte aligned). */
+/* Test hook, host only (needs no GPU): the launch plan of the tensor-core
+ * projection y[M][N] = x[M][K] W^T on n_sm SMs, as sp_classify and sp_project
+ * would choose it.  lo: 1 = hi + lo bf16 activation planes, 0 = plain bf16;
+ * schedule: an SP_OPT_GEMM_SCHEDULE value (0 automatic, 1 tile kernel,
+ * 2 persistent stream-K); capacity_bytes: room for fp32 partial planes
+ * [splits][M][N] (SIZE_MAX: unbounded).  Fills *out; SP_ERR_INVALID_ARG for
+ * M, N, K or n_sm < 1, a NULL out or a bad lo / schedule; SP_ERR_UNSUPPORTED
+ * when the shape has no tensor path (N % 128 or K % 64 nonzero). */
+typedef struct sp_gemm_plan {
+    int rows_per_tile;   /* activation rows per tile (16, 32, 64, 128 or 256)  */
+    int m_tiles;         /* ceil(M / rows_per_tile)                            */
+    int n_tiles;         /* N / 128 weight tiles                               */
+    int n_kblocks;       /* K / 64                                             */
+    int tiles_per_cta;   /* tile kernel: 1, or 2 weight tiles sharing each
+                            activation block                                   */
+    int persistent;      /* 1: stream-K kernel over (tile, k-block) units      */
+    int kblocks_per_cta; /* tile kernel: k-blocks per K split; persistent:
+                            units per CTA                                      */
+    int splits;          /* fp32 partial planes written                        */
+    int grid;            /* CTAs launched                                      */
+} sp_gemm_plan;
+SP_API sp_status sp_debug_gemm_plan(int M, int N, int K, int n_sm, int lo, int schedule,
+                                    size_t capacity_bytes, sp_gemm_plan *out);
+
 SP_API sp_status sp_project(sp_stream stream, int M, int N, int K, const float *d_x,
                             const void *d_w, float *d_y, int path, void *d_workspace,
                             size_t workspace_bytes);

@@ -34,7 +34,7 @@ EXPORTED = ["sp_create", "sp_destroy", "sp_classify", "sp_classify_host", "sp_ch
             "sp_last_error", "sp_set_option", "sp_last_launch_count", "sp_attend_workspace_bytes",
             "sp_attend", "sp_stage_times", "sp_project_workspace_bytes", "sp_project",
             "sp_attend_static", "sp_classify_hidden", "sp_classify_hidden_host",
-            "sp_debug_gathered_pages"]
+            "sp_debug_gathered_pages", "sp_debug_gemm_plan"]
 
 
 class sp_config(C.Structure):
@@ -56,6 +56,12 @@ class sp_kv_cache(C.Structure):
                 ("k_pool", C.c_void_p), ("v_pool", C.c_void_p), ("page_table", C.c_void_p),
                 ("page_size", C.c_int), ("n_pages", C.c_int), ("max_pages_per_seq", C.c_int),
                 ("n_seqs", C.c_int)]
+
+
+class sp_gemm_plan(C.Structure):
+    _fields_ = [(n, C.c_int) for n in ("rows_per_tile", "m_tiles", "n_tiles", "n_kblocks",
+                                       "tiles_per_cta", "persistent", "kblocks_per_cta", "splits",
+                                       "grid")]
 
 
 class sp_attn_dims(C.Structure):
@@ -107,6 +113,7 @@ def load_library(path: str | None = None):
     lib.sp_attend.argtypes = [vp, C.POINTER(sp_attn_dims), i, vp, vp, C.POINTER(sp_kv_cache), vp,
                               vp, vp, vp, i, vp, C.c_size_t, vp, vp]
     lib.sp_debug_gathered_pages.argtypes = [vp, vp, C.c_size_t]
+    lib.sp_debug_gemm_plan.argtypes = [i, i, i, i, i, i, C.c_size_t, C.POINTER(sp_gemm_plan)]
     for name in EXPORTED:
         if name not in ("sp_last_error", "sp_last_launch_count", "sp_attend_workspace_bytes",
                         "sp_project_workspace_bytes"):
@@ -220,6 +227,15 @@ def sp_attend_static(stream, dims, batch, seq_ids, seq_lens, kv, q, k_new, v_new
 
 def sp_project_workspace_bytes(M, N, K) -> int:
     return load_library().sp_project_workspace_bytes(int(M), int(N), int(K))
+
+
+def sp_debug_gemm_plan(M, N, K, n_sm, lo, schedule=0, capacity_bytes=None) -> dict:
+    """The tensor-core projection plan for y[M][N] = x[M][K] W^T (host only)."""
+    plan = sp_gemm_plan()
+    cap = C.c_size_t(-1).value if capacity_bytes is None else int(capacity_bytes)
+    _check(load_library().sp_debug_gemm_plan(int(M), int(N), int(K), int(n_sm), int(lo),
+                                             int(schedule), cap, C.byref(plan)))
+    return {name: getattr(plan, name) for name, _ in sp_gemm_plan._fields_}
 
 
 def sp_project(stream, M, N, K, x, w, y, path, workspace, workspace_bytes):

@@ -1049,6 +1049,25 @@ size_t sp_project_workspace_bytes(int M, int N, int K) {
     return planes + align256((size_t)p.splits * M * N * sizeof(float));
 }
 
+sp_status sp_debug_gemm_plan(int M, int N, int K, int n_sm, int lo, int schedule,
+                             size_t capacity_bytes, sp_gemm_plan *out) {
+    if (M < 1 || N < 1 || K < 1 || n_sm < 1 || !out || (lo != 0 && lo != 1) || schedule < 0 ||
+        schedule > 2)
+        return fail(SP_ERR_INVALID_ARG, "bad plan query");
+    if (!tc_supported(N, K)) return fail(SP_ERR_UNSUPPORTED, "no tensor path for N %d, K %d", N, K);
+    const TcPlan p = tc_plan(M, N, K, n_sm, capacity_bytes, lo != 0, schedule);
+    out->rows_per_tile = p.bn;
+    out->m_tiles = p.m_tiles;
+    out->n_tiles = p.n_tiles;
+    out->n_kblocks = p.n_kb;
+    out->tiles_per_cta = p.persistent ? 1 : p.nt;
+    out->persistent = p.persistent ? 1 : 0;
+    out->kblocks_per_cta = p.units_per_cta;
+    out->splits = p.splits;
+    out->grid = p.grid;
+    return SP_OK;
+}
+
 sp_status sp_project(sp_stream stream, int M, int N, int K, const float *d_x, const void *d_w,
                      float *d_y, int path, void *d_workspace, size_t workspace_bytes) {
     if (M < 1 || N < 1 || K < 1) return fail(SP_ERR_INVALID_ARG, "M, N, K must be >= 1");
