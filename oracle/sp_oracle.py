@@ -56,6 +56,10 @@ Readings where the paper is silent (each is listed in the design notes):
    frozen LM head and the pooled state first passes the head's final RMSNorm
    (gain g_final, the layer's eps): logits = W_head RMSNorm(pool(h2); g_final)
    (+ bias).  The yes/no difference is logits[yes] - logits[no].
+13. head layout (grouped-query attention with no storage order in the paper):
+   rows h*dh..h*dh+dh-1 of W_q are query head h, rows j*dh.. of W_k and W_v
+   are KV head j, cached tokens hold [KV head][dh] in that order, and the
+   attention output reaches W_o concatenated head-major.
 """
 from __future__ import annotations
 
